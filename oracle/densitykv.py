@@ -1,0 +1,371 @@
+"""Plain CPU oracle of the DensityKV bank update and of bank-reading attention.
+
+TEST INFRASTRUCTURE ONLY.  This module is the slow, obviously-correct
+reference that the CUDA path is checked against.  It may be imported only by
+``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py``; the product path never calls it, and it shares no code with the
+CUDA library (it imports numpy only).
+
+Arithmetic is float64 throughout.  The paper fixes the storage precision of
+the two per-state density scalars as FP32 (App. D "Persistent-storage
+accounting"), so the cached density rho and the frozen baseline b are rounded
+to float32 when they are stored in the bank; every sum and comparison is
+evaluated in float64.  Keys and values are taken exactly as given (bf16 inputs
+arrive as their exactly-representable float32 values).
+
+What each function follows (paper sections / equations):
+
+* ``soft_riesz``         Eq. 2 (Soft-Riesz interaction), App. B Eq. B.2.
+* ``sq_dist``            squared Euclidean key distance (Sec. 3.2; the
+                         expansion ||a||^2 + ||b||^2 - 2 a.b is the one written
+                         out in App. A, Eq. "supp-unitnorm-equivalence").
+* ``density``            Eq. 3, Soft-Riesz density over an indexed multiset,
+                         self excluded by index.
+* ``update_layer``       Algorithm 1 (App. C) with Eqs. 5-12 and C.1-C.4:
+                         empty-bank initialisation, mean-normalised candidate
+                         score, stable sort, projected growth ratios for every
+                         prefix length, shared cross-head prefix r*,
+                         mandatory-then-densest eviction, commit, exact density
+                         maintenance and frozen insertion baselines.
+* ``attend``             softmax attention of queries over [bank | window]
+                         with scale 1/sqrt(d_k) (Sec. 3.2 logit definition,
+                         App. A Eq. "supp-logit"; Fig. 2 caption).
+* ``storage_bytes``      App. D persistent-storage accounting.
+
+Readings taken where the paper is silent or ambiguous (each is restated in
+the design notes of the repository):
+
+* Ties in the "decreasing projected density" fill are broken by provenance:
+  the older state (smaller (step, src)) is evicted first (the paper allows any
+  tie rule, Alg. 1).
+* ``g >= tau`` is inclusive and evaluated as a float64 ratio rho~ / b.
+* r = 0 is always treated as feasible, and R is empty when r* = 0, even if
+  rounding made some g(0) reach tau (the invariant that makes r = 0 feasible
+  holds in exact arithmetic; Sec. 3.4 Step 2).
+* Per-head budgets M_h generalise e_r = max(0, m + r - M) to
+  e_r^h = max(0, m_h + r - M_h) with r <= min(N, min_h M_h); a head whose bank
+  is empty takes the empty-bank path (first min(N, M_h) candidates in source
+  order) and does not take part in the shared prefix search.
+* sync_heads=False gives the "independent per-head prefix" ablation
+  (App. E "Cross-head synchronization").
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+__all__ = [
+    "Params", "HeadBank", "LayerBank", "HeadRecord", "UpdateRecord",
+    "soft_riesz", "sq_dist", "density", "potential_against",
+    "update_layer", "attend", "storage_bytes", "GIB",
+]
+
+GIB = float(1 << 30)
+
+
+@dataclasses.dataclass(frozen=True)
+class Params:
+    """Method parameters; defaults from Sec. 4.1 and App. D ("Default DensityKV configuration")."""
+
+    tau: float = 2.0          # allowed density-growth factor, tau > 1
+    sigma: Optional[float] = None  # None -> sqrt(d_k / 2) (App. B, Eq. "supp-bandwidth")
+    p: float = 2.0            # decay exponent
+    eps: float = 1.0          # regulariser
+    delta: float = 1e-6       # baseline floor
+    sync_heads: bool = True   # shared cross-head prefix (default policy)
+
+    def sigma_for(self, d: int) -> float:
+        return math.sqrt(d / 2.0) if self.sigma is None else float(self.sigma)
+
+
+def sq_dist(A: np.ndarray, B: np.ndarray) -> np.ndarray:
+    """||a_i - b_j||^2 for all rows of A against all rows of B, float64 [len(A), len(B)].
+
+    Uses ||a||^2 + ||b||^2 - 2 a.b (App. A) with a library matmul, then clamps
+    at zero because a squared distance is non-negative.
+    """
+    A = np.asarray(A, dtype=np.float64)
+    B = np.asarray(B, dtype=np.float64)
+    na = np.einsum("ij,ij->i", A, A)
+    nb = np.einsum("ij,ij->i", B, B)
+    d2 = na[:, None] + nb[None, :] - 2.0 * (A @ B.T)
+    return np.maximum(d2, 0.0)
+
+
+def soft_riesz(d2: np.ndarray, prm: Params, d: int) -> np.ndarray:
+    """Eq. 2: w = (eps + ||k_i - k_j||^2 / sigma^2)^(-p)."""
+    s = prm.sigma_for(d)
+    return np.power(prm.eps + np.asarray(d2, dtype=np.float64) / (s * s), -prm.p)
+
+
+def density(K: np.ndarray, prm: Params) -> np.ndarray:
+    """Eq. 3: Phi_A(i) = sum_{j != i} w(k_i, k_j) over the indexed multiset K (rows)."""
+    K = np.asarray(K, dtype=np.float64)
+    n = K.shape[0]
+    if n == 0:
+        return np.zeros(0)
+    W = soft_riesz(sq_dist(K, K), prm, K.shape[1])
+    W[np.arange(n), np.arange(n)] = 0.0        # j != i, by index (duplicates still count)
+    return W.sum(axis=1)
+
+
+def potential_against(x: np.ndarray, A: np.ndarray, prm: Params) -> np.ndarray:
+    """App. B Eq. "supp-insertion-energy": Phi_A(k_x) = sum_j w(k_x, k_j) for each row x."""
+    x = np.atleast_2d(np.asarray(x, dtype=np.float64))
+    A = np.asarray(A, dtype=np.float64)
+    if A.shape[0] == 0:
+        return np.zeros(x.shape[0])
+    return soft_riesz(sq_dist(x, A), prm, x.shape[1]).sum(axis=1)
+
+
+@dataclasses.dataclass
+class HeadBank:
+    """Bank of one (layer, head): Eq. 4 plus the cached density and provenance (App. C, App. D)."""
+
+    M: int                      # per-head budget
+    d: int
+    dv: int
+    K: np.ndarray = None        # [m, d] float64 (exact copies of the admitted keys)
+    V: np.ndarray = None        # [m, dv]
+    rho: np.ndarray = None      # [m] float32, cached current density Phi_{K(B)}(i)
+    base: np.ndarray = None     # [m] float32, frozen insertion baseline b_i
+    step: np.ndarray = None     # [m] int64, update step that admitted the state
+    src: np.ndarray = None      # [m] int64, source index of the state within its block
+    store: type = np.float32    # storage type of rho and b (FP32 per App. D; float64 for pins)
+
+    def __post_init__(self):
+        if self.K is None:
+            self.K = np.zeros((0, self.d))
+            self.V = np.zeros((0, self.dv))
+            self.rho = np.zeros(0, self.store)
+            self.base = np.zeros(0, self.store)
+            self.step = np.zeros(0, np.int64)
+            self.src = np.zeros(0, np.int64)
+
+    @property
+    def m(self) -> int:
+        return int(self.K.shape[0])
+
+    def copy(self) -> "HeadBank":
+        return HeadBank(self.M, self.d, self.dv, self.K.copy(), self.V.copy(), self.rho.copy(),
+                        self.base.copy(), self.step.copy(), self.src.copy(), self.store)
+
+
+@dataclasses.dataclass
+class LayerBank:
+    heads: List[HeadBank]
+
+    @staticmethod
+    def empty(budgets: Sequence[int], d: int, dv: Optional[int] = None, store=np.float32) -> "LayerBank":
+        return LayerBank([HeadBank(int(M), d, d if dv is None else dv, store=store) for M in budgets])
+
+    def copy(self) -> "LayerBank":
+        return LayerBank([h.copy() for h in self.heads])
+
+
+@dataclasses.dataclass
+class HeadRecord:
+    """Intermediate quantities of one head's update, exposed for parity checks."""
+
+    empty_init: bool
+    s: Optional[np.ndarray] = None          # [N] Eq. 6 / C.1 scores
+    pi: Optional[np.ndarray] = None         # [N] stable ascending order of s
+    counts: Optional[np.ndarray] = None     # [rmax+1] c_r^h for every tested prefix
+    e: Optional[np.ndarray] = None          # [rmax+1] e_r^h
+    cross: Optional[np.ndarray] = None      # [m] min{r : g_i(r) >= tau}, or -1 if none <= rmax
+    r_used: int = 0                         # number of candidates admitted in this head
+    rho_tilde: Optional[np.ndarray] = None  # [m] rho~_i(r*) (float64)
+    g_star: Optional[np.ndarray] = None     # [m] g_i(r*)
+    mandatory: Optional[np.ndarray] = None  # [m] bool, g_i(r*) >= tau (and r* > 0)
+    evicted: Optional[np.ndarray] = None    # indices (pre-update bank order) of R, mandatory first
+    admitted: Optional[np.ndarray] = None   # candidate indices admitted, in admission order
+
+
+@dataclasses.dataclass
+class UpdateRecord:
+    r_star: int
+    rmax: int
+    heads: List[HeadRecord]
+
+
+def _prefix_rho_tilde(hb: HeadBank, Kc_pi: np.ndarray, prm: Params, rmax: int) -> np.ndarray:
+    """Eq. C.2 for every prefix length r = 0..rmax: rho~_i(r) = rho_i + sum_{j<=r} w(kbar_i, k_pi(j)).
+
+    Returns float64 [m, rmax+1].  Column-wise cumulative sums over the
+    pi-ordered candidate interactions give all prefix contributions (App. C,
+    "Decision granularity versus computational tiling").
+    """
+    Wmat = soft_riesz(sq_dist(hb.K, Kc_pi[:rmax]), prm, hb.d)          # [m, rmax]
+    out = np.empty((hb.m, rmax + 1))
+    out[:, 0] = hb.rho.astype(np.float64)
+    out[:, 1:] = hb.rho.astype(np.float64)[:, None] + np.cumsum(Wmat, axis=1)
+    return out
+
+
+def _prefix_rho_tilde_literal(hb: HeadBank, Kc_pi: np.ndarray, prm: Params, rmax: int) -> np.ndarray:
+    """Same quantity as ``_prefix_rho_tilde``, recomputed from scratch for each r with plain loops.
+
+    Tiny inputs only; used to pin the cumulative-sum form (Alg. 1 tests every prefix length).
+    """
+    s = prm.sigma_for(hb.d)
+    out = np.empty((hb.m, rmax + 1))
+    for i in range(hb.m):
+        for r in range(rmax + 1):
+            acc = float(hb.rho[i])
+            for j in range(r):
+                diff = hb.K[i] - Kc_pi[j]
+                d2 = float(np.dot(diff, diff))
+                acc += (prm.eps + d2 / (s * s)) ** (-prm.p)
+            out[i, r] = acc
+    return out
+
+
+def _empty_init(hb: HeadBank, Kc: np.ndarray, Vc: np.ndarray, step: int, prm: Params) -> HeadRecord:
+    """Alg. 1, m = 0 branch: admit the first min(N, M) source-ordered candidates, then set
+    rho_i = Phi over the resulting bank and b_i = max(rho_i, delta)."""
+    N = Kc.shape[0]
+    r = min(N, hb.M)
+    hb.K = np.asarray(Kc[:r], dtype=np.float64).copy()
+    hb.V = np.asarray(Vc[:r], dtype=np.float64).copy()
+    rho = density(hb.K, prm)
+    hb.rho = rho.astype(hb.store)
+    hb.base = np.maximum(rho, prm.delta).astype(hb.store)
+    hb.step = np.full(r, step, np.int64)
+    hb.src = np.arange(r, dtype=np.int64)
+    return HeadRecord(empty_init=True, r_used=r, admitted=np.arange(r), evicted=np.zeros(0, np.int64))
+
+
+def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
+                 prm: Params = Params(), literal: bool = False) -> UpdateRecord:
+    """One DensityKV update of one layer (Algorithm 1, App. C), in place on ``bank``.
+
+    Kc, Vc: candidate keys/values of the finalized block, [H][N][d] and [H][N][dv],
+    in source order.  ``step`` is recorded as the provenance of admitted states.
+    ``literal=True`` recomputes every prefix sum from scratch (tiny inputs).
+    """
+    H = len(bank.heads)
+    Kc = np.asarray(Kc, dtype=np.float64)
+    Vc = np.asarray(Vc, dtype=np.float64)
+    assert Kc.shape[0] == H and Vc.shape[0] == H
+    N = Kc.shape[1]
+    recs: List[Optional[HeadRecord]] = [None] * H
+
+    live = [h for h in range(H) if bank.heads[h].m > 0]
+    for h in range(H):
+        if bank.heads[h].m == 0:
+            recs[h] = _empty_init(bank.heads[h], Kc[h], Vc[h], step, prm)
+
+    rmax = min([N] + [bank.heads[h].M for h in live]) if live else 0
+    if not live:
+        return UpdateRecord(r_star=min(N, min(hb.M for hb in bank.heads)) if H else 0,
+                            rmax=rmax, heads=recs)
+
+    # Steps 1-2 per head: score, stable sort, projected growth for every prefix length.
+    tables = {}
+    for h in live:
+        hb = bank.heads[h]
+        m = hb.m
+        # Eq. 6 / C.1: s_h(x) = (1/m) sum_i w(kbar_i, k_x) / b_i
+        Wxb = soft_riesz(sq_dist(Kc[h], hb.K), prm, hb.d)              # [N, m]
+        s = (Wxb / hb.base.astype(np.float64)[None, :]).sum(axis=1) / m
+        # stable ascending sort, ties broken by source order
+        pi = np.argsort(s, kind="stable")
+        Kc_pi = Kc[h][pi]
+        if literal:
+            rt = _prefix_rho_tilde_literal(hb, Kc_pi, prm, rmax)
+        else:
+            rt = _prefix_rho_tilde(hb, Kc_pi, prm, rmax)
+        g = rt / hb.base.astype(np.float64)[:, None]                    # Eq. C.3
+        viol = g >= prm.tau
+        counts = viol.sum(axis=0)                                        # c_r^h, Eq. 9
+        r_all = np.arange(rmax + 1)
+        e = np.maximum(0, m + r_all - hb.M)                              # e_r^h, Eq. 10
+        feasible = counts <= e
+        feasible[0] = True                                               # r = 0 always feasible
+        anyv = viol.any(axis=1)
+        cross = np.where(anyv, np.argmax(viol, axis=1), -1)
+        tables[h] = (s, pi, rt, g, counts, e, feasible, cross)
+
+    # Eq. 11: largest prefix length feasible for every head (or per head when not synchronised).
+    if prm.sync_heads:
+        allf = np.logical_and.reduce([tables[h][6] for h in live])
+        r_star = int(np.nonzero(allf)[0].max())
+        r_of = {h: r_star for h in live}
+    else:
+        r_of = {h: int(np.nonzero(tables[h][6])[0].max()) for h in live}
+        r_star = max(r_of.values())
+
+    # Step 3 per head: evict, commit, maintain densities.
+    for h in live:
+        hb = bank.heads[h]
+        s, pi, rt, g, counts, e, feasible, cross = tables[h]
+        r = r_of[h]
+        m = hb.m
+        e_r = int(e[r])
+        rho_t = rt[:, r]
+        g_r = g[:, r]
+        mand = (g_r >= prm.tau) if r > 0 else np.zeros(m, bool)
+        mand_idx = np.nonzero(mand)[0]
+        assert mand_idx.shape[0] <= e_r, "feasibility violated"
+        rest = np.nonzero(~mand)[0]
+        # decreasing rho~(r*); ties: older provenance (smaller step, then src) first
+        order = np.lexsort((hb.src[rest], hb.step[rest], -rho_t[rest]))
+        fill = rest[order[:e_r - mand_idx.shape[0]]]
+        R = np.concatenate([mand_idx, fill]).astype(np.int64)
+        keep = np.ones(m, bool)
+        keep[R] = False
+        adm = pi[:r]
+
+        # Eq. C.4: survivors' cached density, exactly: rho~(r*) minus interactions with R.
+        if R.shape[0] > 0 and keep.any():
+            sub = soft_riesz(sq_dist(hb.K[keep], hb.K[R]), prm, hb.d).sum(axis=1)
+        else:
+            sub = np.zeros(int(keep.sum()))
+        rho_surv = rho_t[keep] - sub
+
+        # Eq. 12 commit: (B \ R) followed by the admitted prefix in pi order.
+        K_new = np.concatenate([hb.K[keep], Kc[h][adm]], axis=0)
+        V_new = np.concatenate([hb.V[keep], Vc[h][adm]], axis=0)
+        # Eq. 5 / C.4: new states' density over the final bank (co-admitted included), frozen as b.
+        n_surv = int(keep.sum())
+        if r > 0:
+            W_new = soft_riesz(sq_dist(K_new[n_surv:], K_new), prm, hb.d)    # [r, m']
+            W_new[np.arange(r), n_surv + np.arange(r)] = 0.0                  # exclude self by index
+            rho_new = W_new.sum(axis=1)
+        else:
+            rho_new = np.zeros(0)
+        hb.K, hb.V = K_new, V_new
+        hb.rho = np.concatenate([rho_surv, rho_new]).astype(hb.store)
+        hb.base = np.concatenate([hb.base[keep], np.maximum(rho_new, prm.delta)]).astype(hb.store)
+        hb.step = np.concatenate([hb.step[keep], np.full(r, step, np.int64)])
+        hb.src = np.concatenate([hb.src[keep], adm.astype(np.int64)])
+        recs[h] = HeadRecord(empty_init=False, s=s, pi=pi, counts=counts, e=e, cross=cross,
+                             r_used=r, rho_tilde=rho_t, g_star=g_r, mandatory=mand,
+                             evicted=R, admitted=adm)
+    return UpdateRecord(r_star=r_star, rmax=rmax, heads=recs)
+
+
+def attend(hb: HeadBank, Q: np.ndarray, Kw: np.ndarray, Vw: np.ndarray) -> np.ndarray:
+    """Softmax attention of Q over [bank keys | window keys], logits q.k / sqrt(d_k), no mask."""
+    Q = np.asarray(Q, dtype=np.float64)
+    Kall = np.concatenate([hb.K, np.asarray(Kw, dtype=np.float64)], axis=0)
+    Vall = np.concatenate([hb.V, np.asarray(Vw, dtype=np.float64)], axis=0)
+    if Kall.shape[0] == 0:
+        return np.zeros((Q.shape[0], hb.dv))
+    S = (Q @ Kall.T) / math.sqrt(Q.shape[1])
+    S -= S.max(axis=1, keepdims=True)
+    P = np.exp(S)
+    P /= P.sum(axis=1, keepdims=True)
+    return P @ Vall
+
+
+def storage_bytes(L: int, H: int, n: int, dk: int = 128, dv: int = 128,
+                  kv_bytes: int = 2, meta_bytes: int = 4 + 4 + 8 + 4) -> dict:
+    """App. D accounting: S_KV(n) = L H n (d_k + d_v) x 2 bytes, plus per-state metadata
+    (two FP32 density scalars, int64 + int32 provenance = 20 bytes)."""
+    kv = L * H * n * (dk + dv) * kv_bytes
+    meta = L * H * n * meta_bytes
+    return {"kv": kv, "meta": meta, "total": kv + meta}

@@ -1,0 +1,44 @@
+"""The seeded input generator: determinism, shapes, bf16 exactness and the vMF law."""
+import numpy as np
+from scipy.special import ive
+
+import synth
+
+
+def test_vmf_mean_resultant_length_matches_theory():
+    # E[mu . x] = A_d(kappa) = I_{d/2}(kappa) / I_{d/2-1}(kappa) for x ~ vMF(mu, kappa) on S^{d-1}
+    rng = np.random.default_rng(0)
+    for d, kappa in ((64, 20.0), (128, 2560.0), (16, 5.0)):
+        mu = np.zeros(d)
+        mu[3] = 1.0
+        x = synth.sample_vmf(rng, mu, kappa, 20000)
+        assert np.allclose(np.linalg.norm(x, axis=1), 1.0, atol=1e-12)
+        theory = ive(d / 2, kappa) / ive(d / 2 - 1, kappa)
+        assert abs(x[:, 3].mean() - theory) < 4 * x[:, 3].std() / np.sqrt(len(x)) + 1e-4
+
+
+def test_blocks_are_deterministic_and_bf16_exact():
+    wl = synth.get_workload("wan13b_layer_h12", N=64, Nq=32, H=3)
+    a = synth.LayerRollout(wl, 0)
+    b = synth.LayerRollout(wl, 0, heads=[2])
+    K, V = a.block(5)
+    K2, V2 = b.block(5)
+    assert K.shape == (3, 64, 128) and np.array_equal(K[2], K2[0]) and np.array_equal(V[2], V2[0])
+    assert np.array_equal(synth.round_to_bf16(K), K)
+    assert not np.array_equal(a.block(6)[0], K)
+    assert abs(np.linalg.norm(K, axis=-1).mean() - np.sqrt(128)) < 0.2
+
+
+def test_round_to_bf16_ties_to_even():
+    x = np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -1.5, 3.0e38], np.float32)
+    r = synth.round_to_bf16(x)
+    assert r[0] == 1.0 and r[1] == 1.0 + 2 ** -6 and r[2] == -1.5
+
+
+def test_workload_shapes():
+    wl = synth.get_workload("wan14b_headwise_l40h40")
+    assert len(wl.budgets) == 1600 and set(wl.budgets) <= {2340, 4680, 9360, 18720}
+    assert set(wl.clusters) <= {8, 32, 128, 512} and 5.0 <= min(wl.kappa) and max(wl.kappa) <= 50.0
+    wl0 = synth.get_workload("tiny_fp32_l1h2_d64")
+    assert (wl0.L, wl0.H, wl0.d, wl0.N, wl0.budgets, wl0.dtype) == (1, 2, 64, 256, (512, 512), "fp32")
+    assert wl0.admitted_block(0) == 0 and synth.get_workload("wan13b_layer_h12").admitted_block(0) is None
