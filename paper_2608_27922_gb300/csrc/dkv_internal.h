@@ -1,0 +1,94 @@
+// Internal (non-ABI) declarations shared by the host API and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "dkv_device.cuh"
+
+namespace dkv {
+
+// Caller-owned bank buffers plus their dimensions.
+struct Bank {
+  void* k;
+  void* v;
+  float* rho;
+  float* base;
+  float* knorm;
+  int64_t* prov_step;
+  int32_t* prov_src;
+  int32_t* occ;
+  int H, d, M_max, n_max;
+  int bf16;   // 1: bf16 keys/values, 0: fp32
+};
+
+// Device workspace, carved from the caller's workspace buffer (dkv_api.cu).
+struct Ws {
+  DevLayer* L;
+  DevHead* hd;          // [H]
+  int32_t* budgets;     // [H]
+  float* cnorm;         // [H][n_max]     ||k_x||^2 of the candidates (source order)
+  float* score;         // [H][n_max]     Eq. 6 scores
+  int32_t* perm;        // [H][n_max]     stable ascending order of the scores (pi)
+  void* kperm;          // [H][n_max][d]  candidate keys in pi order
+  float* kperm_norm;    // [H][n_max]
+  int32_t* cross;       // [H][M_max]     first prefix length with g >= tau (INT32_MAX: none)
+  int32_t* hist;        // [H][hist_stride] histogram of cross over 0..rmax+1
+  uint32_t* feas;       // [H][feas_words] bit r set: prefix r feasible in head h
+  float* snap;          // [H][M_max][snap_stride] running prefix sums every SNAP columns
+  float* rho_t;         // [H][M_max]     projected density rho~(r_h) (Eq. C.2)
+  int32_t* evict_list;  // [H][n_max]     evicted slots, ascending
+  int32_t* surv_list;   // [H][M_max]     surviving slots, ascending
+  void* kevict;         // [H][n_max][d]  keys of evicted states (gathered before commit)
+  float* kevict_norm;   // [H][n_max]
+  void* ksurv;          // [H][M_max][d]  keys of surviving states
+  float* ksurv_norm;    // [H][M_max]
+  int32_t* slot_new;    // [H][n_max]     bank slot of the j-th admitted candidate
+  int hist_stride, snap_stride, feas_words;
+};
+
+// Computes the sub-buffer offsets of the workspace; returns the total bytes.
+size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* base);
+
+// Kernel timing hook (dkv_api.cu): brackets a launch with events when enabled.
+struct Timer;
+void timer_begin(Timer* t, const char* name, cudaStream_t s);
+void timer_end(Timer* t, cudaStream_t s);
+
+// ---- launches (each returns cudaGetLastError() of its launch) ----
+// update front half (admit)
+cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cudaStream_t s, Timer* t);
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t);
+cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_cross_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+// update back half (compress)
+cudaError_t launch_project_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_select(const Bank& b, const Ws& w, cudaStream_t s, Timer* t);
+cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t);
+cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_subtract_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_newbase_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+// tensor-core (tcgen05) versions of the pair passes, bf16 and d = 128 only
+cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+// bank maintenance
+cudaError_t launch_bank_norms(const Bank& b, cudaStream_t s, Timer* t);
+cudaError_t launch_set_occupancy(const Bank& b, const int32_t* occ_dev_src, int value, cudaStream_t s);
+// attention
+cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,
+                               void* O, cudaStream_t s, Timer* t);
+cudaError_t launch_attend_tc(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,
+                             void* O, cudaStream_t s, Timer* t);
+bool tc_supported(int d, int bf16);
+cudaError_t simt_set_smem_limits();
+cudaError_t update_set_smem_limits();
+cudaError_t tc_set_smem_limits();
+
+}  // namespace dkv

@@ -1,0 +1,507 @@
+// Selection, ordering and compaction kernels of the bank update (no pair math).
+//
+//   prepare      snapshot of occupancy, budgets and the prefix range of this update
+//   cand_norms   ||k_x||^2 of the candidates (fp32)
+//   sort         stable ascending order of the Eq. 6 scores, ties by source index (Alg. 1)
+//   permute      candidate keys copied into pi order (operand of the prefix passes)
+//   rstar_*      violator counts c_r = #{cross <= r}, budgets e_r (Eq. 10), feasibility,
+//                and the largest prefix feasible for every head (Eq. 11)
+//   select       mandatory set {g(r*) >= tau} plus the densest rho~(r*) (Step 3), via a
+//                radix select on the fp32 bit patterns; ties evict the older state
+//   gather       keys of the surviving and of the evicted states (operands of Eq. C.4)
+//   commit       Eq. 12: admitted keys/values into the evicted slots, the rest appended
+#include "dkv_internal.h"
+
+#include <climits>
+
+namespace dkv {
+
+namespace {
+
+constexpr int BIG = 1024;   // threads of the one-block-per-head kernels
+
+__device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
+__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
+
+// Copies one row of `bytes` bytes (a multiple of 16) with one warp.
+__device__ __forceinline__ void warp_copy_row(void* dst, const void* src, int bytes) {
+  const uint4* s = reinterpret_cast<const uint4*>(src);
+  uint4* d = reinterpret_cast<uint4*>(dst);
+  for (int i = lane_id(); i < bytes / 16; i += 32) d[i] = s[i];
+}
+
+__global__ void k_prepare(Bank b, Ws w, int N, int64_t step) {
+  __shared__ int s_min_budget, s_live;
+  if (threadIdx.x == 0) { s_min_budget = INT_MAX; s_live = 0; }
+  __syncthreads();
+  for (int h = threadIdx.x; h < b.H; h += blockDim.x) {
+    int m = b.occ[h];
+    const int M = w.budgets[h];
+    if (m < 0 || m > M) {
+      dev_fail(w.L, DEV_INCONSISTENT, 1000 + h);
+      m = m < 0 ? 0 : M;
+    }
+    DevHead hd;
+    hd.m_old = m; hd.M = M; hd.r = 0; hd.e = 0; hd.n_mand = 0; hd.n_pre = 0; hd.m_new = m;
+    hd.empty = (m == 0);
+    w.hd[h] = hd;
+    if (m > 0) { atomicMin(&s_min_budget, M); atomicAdd(&s_live, 1); }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    w.L->N = N;
+    w.L->step = step;
+    w.L->empty_all = (s_live == 0);
+    w.L->rmax = s_live ? min(N, s_min_budget) : 0;
+    w.L->r_star = 0;
+  }
+}
+
+template <typename T>
+__global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
+                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d) {
+  const int h = blockIdx.y;
+  const int row = blockIdx.x * (blockDim.x / 32) + warp_id();
+  const int n = count_is_occ ? count[h] : N;
+  if (row < 0 || row >= n || row >= rows_cap) return;
+  const T* r = K + (int64_t)h * head_stride + (int64_t)row * d;
+  float a = 0.f;
+  for (int k = lane_id(); k < d; k += 32) {
+    const float x = to_f<T>(r[k]);
+    a = fmaf(x, x, a);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+  if (lane_id() == 0) out[(int64_t)h * out_hs + row] = a;
+}
+
+// Bitonic sort of (fkey(score) << 32 | source index) per head: ascending score,
+// equal scores in source order.
+__global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
+  extern __shared__ unsigned long long keys[];
+  const int h = blockIdx.x;
+  const int N = w.L->N;
+  int32_t* perm = w.perm + (int64_t)h * n_max;
+  if (w.hd[h].empty) {   // empty bank: source order (Alg. 1, m = 0 branch)
+    for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = i;
+    return;
+  }
+  int n = 2;
+  while (n < N) n <<= 1;
+  const float* sc = w.score + (int64_t)h * n_max;
+  for (int i = threadIdx.x; i < n; i += blockDim.x)
+    keys[i] = i < N ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
+  __syncthreads();
+  for (int k = 2; k <= n; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const int ix = i ^ j;
+        if (ix > i) {
+          const unsigned long long a = keys[i], c = keys[ix];
+          const bool up = (i & k) == 0;
+          if ((a > c) == up) { keys[i] = c; keys[ix] = a; }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = (int32_t)(keys[i] & 0xffffffffu);
+}
+
+__global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int esize) {
+  const int h = blockIdx.y;
+  const int j = blockIdx.x * (blockDim.x / 32) + warp_id();
+  if (j >= N) return;
+  const int rb = b.d * esize;
+  const int src = w.perm[(int64_t)h * b.n_max + j];
+  warp_copy_row((char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, Kc + ((int64_t)h * N + src) * rb, rb);
+  if (lane_id() == 0) w.kperm_norm[(int64_t)h * b.n_max + j] = w.cnorm[(int64_t)h * b.n_max + src];
+}
+
+// Per head: c_r = #{i : cross_i <= r} and feasibility c_r <= e_r for r in [0, rmax].
+__global__ void __launch_bounds__(BIG) k_rstar_head(Ws w) {
+  __shared__ int s_tot[BIG];
+  __shared__ int s_best;
+  const int h = blockIdx.x;
+  const DevHead hd = w.hd[h];
+  const int rmax = w.L->rmax;
+  uint32_t* feas = w.feas + (int64_t)h * w.feas_words;
+  const int nw = (rmax + 1 + 31) / 32;
+  if (hd.empty) {   // an empty head does not constrain the shared prefix
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) feas[i] = 0xffffffffu;
+    return;
+  }
+  for (int i = threadIdx.x; i < nw; i += blockDim.x) feas[i] = 0u;
+  if (threadIdx.x == 0) s_best = 0;
+  const int n = rmax + 1;
+  const int chunk = (n + blockDim.x - 1) / blockDim.x;
+  const int lo = threadIdx.x * chunk, hi = min(n, lo + chunk);
+  const int32_t* hist = w.hist + (int64_t)h * w.hist_stride;
+  int tot = 0;
+  for (int r = lo; r < hi; ++r) tot += hist[r];
+  s_tot[threadIdx.x] = tot;
+  __syncthreads();
+  for (int o = 1; o < (int)blockDim.x; o <<= 1) {   // inclusive Hillis-Steele scan
+    const int v = threadIdx.x >= o ? s_tot[threadIdx.x - o] : 0;
+    __syncthreads();
+    s_tot[threadIdx.x] += v;
+    __syncthreads();
+  }
+  int c = s_tot[threadIdx.x] - tot;   // exclusive prefix
+  int best = 0;
+  for (int r = lo; r < hi; ++r) {
+    c += hist[r];
+    const int e = max(0, hd.m_old + r - hd.M);
+    const bool ok = (r == 0) || (c <= e);   // r = 0 is always feasible (Sec. 3.4 Step 2)
+    if (ok) {
+      atomicOr(&feas[r >> 5], 1u << (r & 31));
+      best = r;
+    }
+  }
+  atomicMax(&s_best, best);
+  __syncthreads();
+  if (threadIdx.x == 0) w.hd[h].r = s_best;   // largest feasible prefix of this head alone
+}
+
+__global__ void __launch_bounds__(BIG) k_rstar_layer(Bank b, Ws w, int sync_heads) {
+  __shared__ int s_best;
+  const int rmax = w.L->rmax;
+  const int N = w.L->N;
+  const int nw = (rmax + 1 + 31) / 32;
+  if (threadIdx.x == 0) s_best = 0;
+  __syncthreads();
+  if (sync_heads) {
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
+      uint32_t a = 0xffffffffu;
+      for (int h = 0; h < b.H; ++h) a &= w.feas[(int64_t)h * w.feas_words + i];
+      if (i == nw - 1 && ((rmax + 1) & 31)) a &= (1u << ((rmax + 1) & 31)) - 1u;
+      if (i == 0) a |= 1u;
+      if (a) atomicMax(&s_best, i * 32 + 31 - __clz(a));
+    }
+  }
+  __syncthreads();
+  const int rstar = s_best;
+  __shared__ int s_rmax_used, s_rmin_used;
+  if (threadIdx.x == 0) { s_rmax_used = 0; s_rmin_used = INT_MAX; }
+  __syncthreads();
+  for (int h = threadIdx.x; h < b.H; h += blockDim.x) {
+    DevHead hd = w.hd[h];
+    int r;
+    if (hd.empty) r = min(N, hd.M);
+    else r = sync_heads ? rstar : hd.r;
+    hd.r = r;
+    hd.e = hd.empty ? 0 : max(0, hd.m_old + r - hd.M);
+    w.hd[h] = hd;
+    atomicMax(&s_rmax_used, r);
+    atomicMin(&s_rmin_used, r);
+  }
+  __syncthreads();
+  // reported r*: Alg. 1's min(N, M) when every head starts empty (min over per-head budgets),
+  // the shared prefix when synchronised, else the largest per-head prefix
+  if (threadIdx.x == 0)
+    w.L->r_star = w.L->empty_all ? s_rmin_used : (sync_heads ? rstar : s_rmax_used);
+}
+
+// Block-wide exclusive scan of one flag per thread; returns this thread's offset and
+// writes the block total to *total.
+__device__ int block_scan_flag(int flag, int* s_warp, int* total) {
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  const int within = __popc(bal & ((1u << lane_id()) - 1u));
+  if (lane_id() == 0) s_warp[warp_id()] = __popc(bal);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int run = 0;
+    for (int i = 0; i < (int)(blockDim.x / 32); ++i) { const int v = s_warp[i]; s_warp[i] = run; run += v; }
+    s_warp[32] = run;
+  }
+  __syncthreads();
+  const int off = s_warp[warp_id()] + within;
+  *total = s_warp[32];
+  __syncthreads();
+  return off;
+}
+
+__global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
+  __shared__ int s_hist[256];
+  __shared__ int s_warp[33];
+  __shared__ int s_cnt[2];
+  __shared__ unsigned s_prefix, s_kk;
+  __shared__ unsigned long long s_tprefix;
+  const int h = blockIdx.x;
+  const DevHead hd = w.hd[h];
+  const int64_t bh = (int64_t)h * b.M_max;
+  const int m = hd.m_old;
+  const int r = hd.r;
+  const int e = hd.e;
+  const int32_t* cross = w.cross + bh;
+  const float* rt = w.rho_t + bh;
+  if (hd.empty) return;
+  if (threadIdx.x == 0) { s_cnt[0] = 0; s_cnt[1] = 0; }
+  __syncthreads();
+  // mandatory set and pre-violators
+  int nm = 0, npre = 0;
+  for (int i = threadIdx.x; i < m; i += blockDim.x) {
+    const int c = cross[i];
+    npre += (c == 0);
+    nm += (r > 0 && c <= r);
+  }
+  atomicAdd(&s_cnt[0], nm);
+  atomicAdd(&s_cnt[1], npre);
+  __syncthreads();
+  int n_mand = s_cnt[0];
+  if (threadIdx.x == 0) { w.hd[h].n_mand = n_mand; w.hd[h].n_pre = s_cnt[1]; }
+  if (e == 0) return;
+  if (n_mand > e) {   // the prefix was feasible, so this cannot happen
+    if (threadIdx.x == 0) dev_fail(w.L, DEV_INCONSISTENT, 2000 + h);
+    return;
+  }
+  const int k = e - n_mand;   // states to evict by decreasing rho~(r)
+  // radix select of the k-th largest key among non-mandatory states
+  unsigned prefix = 0, mask = 0;
+  if (threadIdx.x == 0) { s_prefix = 0; s_kk = (unsigned)k; }
+  __syncthreads();
+  if (k > 0) {
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = threadIdx.x; i < 256; i += blockDim.x) s_hist[i] = 0;
+      __syncthreads();
+      for (int i = threadIdx.x; i < m; i += blockDim.x) {
+        if (r > 0 && cross[i] <= r) continue;
+        const unsigned key = fkey(rt[i]);
+        if ((key & mask) == prefix) atomicAdd(&s_hist[(key >> shift) & 255u], 1);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned kk = s_kk, cum = 0;
+        for (int bin = 255; bin >= 0; --bin) {
+          const unsigned c = (unsigned)s_hist[bin];
+          if (cum + c >= kk) { s_kk = kk - cum; s_prefix = prefix | ((unsigned)bin << shift); break; }
+          cum += c;
+        }
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      mask |= 255u << shift;
+    }
+  }
+  const unsigned T = prefix;          // key of the k-th largest
+  const unsigned take_eq = s_kk;      // how many states with key == T to evict
+  // ties at the threshold: evict the older states (smaller (step, src)) first
+  int n_eq_local = 0;
+  if (k > 0)
+    for (int i = threadIdx.x; i < m; i += blockDim.x)
+      if (!(r > 0 && cross[i] <= r) && fkey(rt[i]) == T) ++n_eq_local;
+  __syncthreads();
+  if (threadIdx.x == 0) s_cnt[0] = 0;
+  __syncthreads();
+  atomicAdd(&s_cnt[0], n_eq_local);
+  __syncthreads();
+  const unsigned n_eq = (unsigned)s_cnt[0];
+  unsigned long long tprefix = 0, tmask = 0;
+  const bool need_tie = k > 0 && n_eq > take_eq;
+  if (need_tie) {
+    if (threadIdx.x == 0) { s_tprefix = 0; s_kk = take_eq; }
+    __syncthreads();
+    for (int shift = 56; shift >= 0; shift -= 8) {
+      for (int i = threadIdx.x; i < 256; i += blockDim.x) s_hist[i] = 0;
+      __syncthreads();
+      for (int i = threadIdx.x; i < m; i += blockDim.x) {
+        if ((r > 0 && cross[i] <= r) || fkey(rt[i]) != T) continue;
+        const unsigned long long tk = ((unsigned long long)(uint32_t)b.prov_step[bh + i] << 32) |
+                                      (uint32_t)b.prov_src[bh + i];
+        if ((tk & tmask) == tprefix) atomicAdd(&s_hist[(tk >> shift) & 255ull], 1);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {   // smallest first
+        unsigned kk = s_kk, cum = 0;
+        for (int bin = 0; bin < 256; ++bin) {
+          const unsigned c = (unsigned)s_hist[bin];
+          if (cum + c >= kk) { s_kk = kk - cum; s_tprefix = tprefix | ((unsigned long long)bin << shift); break; }
+          cum += c;
+        }
+      }
+      __syncthreads();
+      tprefix = s_tprefix;
+      tmask |= 255ull << shift;
+    }
+  }
+  // provenance keys are unique per head, so "<= tprefix" selects exactly take_eq states
+  int n_ev = 0, n_sv = 0;
+  for (int base = 0; base < m; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    int ev = 0;
+    if (i < m) {
+      const bool mand = r > 0 && cross[i] <= r;
+      if (mand) ev = 1;
+      else if (k > 0) {
+        const unsigned key = fkey(rt[i]);
+        if (key > T) ev = 1;
+        else if (key == T) {
+          if (!need_tie) ev = 1;
+          else {
+            const unsigned long long tk = ((unsigned long long)(uint32_t)b.prov_step[bh + i] << 32) |
+                                          (uint32_t)b.prov_src[bh + i];
+            ev = tk <= tprefix;
+          }
+        }
+      }
+    }
+    int tot;
+    const int off = block_scan_flag(ev, s_warp, &tot);
+    if (i < m && ev && n_ev + off < e) w.evict_list[(int64_t)h * b.n_max + n_ev + off] = i;
+    const int offs = (threadIdx.x - off);   // survivors before this thread in the chunk
+    if (i < m && !ev && n_sv + offs < m) w.surv_list[bh + n_sv + offs] = i;
+    n_ev += tot;
+    n_sv += min((int)blockDim.x, m - base) - tot;
+  }
+  if (threadIdx.x == 0 && n_ev != e) dev_fail(w.L, DEV_INCONSISTENT, 3000 + h);
+}
+
+// Keys of the surviving states (rows of Eq. C.4's subtraction) and of the evicted
+// states (its columns), copied before the commit overwrites the evicted slots.
+__global__ void k_gather(Bank b, Ws w, int esize) {
+  const int h = blockIdx.y;
+  const DevHead hd = w.hd[h];
+  if (hd.empty || hd.e == 0) return;
+  const int row = blockIdx.x * (blockDim.x / 32) + warp_id();
+  const int rb = b.d * esize;
+  const int64_t bh = (int64_t)h * b.M_max;
+  const int ns = hd.m_old - hd.e;
+  if (row < ns) {
+    const int slot = w.surv_list[bh + row];
+    if (slot < 0 || slot >= hd.m_old) {
+      if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
+      return;
+    }
+    warp_copy_row((char*)w.ksurv + (bh + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
+    if (lane_id() == 0) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
+  }
+  if (row < hd.e) {
+    const int slot = w.evict_list[(int64_t)h * b.n_max + row];
+    if (slot < 0 || slot >= hd.m_old) {
+      if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 7500 + h);
+      return;
+    }
+    warp_copy_row((char*)w.kevict + ((int64_t)h * b.n_max + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
+    if (lane_id() == 0) w.kevict_norm[(int64_t)h * b.n_max + row] = b.knorm[bh + slot];
+  }
+}
+
+// Eq. 12: the j-th admitted candidate (pi order) goes to the j-th evicted slot, the
+// rest are appended after the old occupancy; keys and values are copied bit for bit.
+__global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int esize) {
+  const int h = blockIdx.y;
+  const DevHead hd = w.hd[h];
+  const int j = blockIdx.x * (blockDim.x / 32) + warp_id();
+  const int64_t bh = (int64_t)h * b.M_max;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    const int m_new = hd.m_old - hd.e + hd.r;
+    w.hd[h].m_new = m_new;
+    b.occ[h] = m_new;
+    if (m_new > hd.M) dev_fail(w.L, DEV_INCONSISTENT, 4000 + h);
+  }
+  if (j >= hd.r) return;
+  const int slot = j < hd.e ? w.evict_list[(int64_t)h * b.n_max + j] : hd.m_old + (j - hd.e);
+  if (slot < 0 || slot >= hd.M) {
+    if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
+    return;
+  }
+  const int rb = b.d * esize;
+  const int src = w.perm[(int64_t)h * b.n_max + j];
+  warp_copy_row((char*)b.k + (bh + slot) * rb, (const char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, rb);
+  warp_copy_row((char*)b.v + (bh + slot) * rb, Vc + ((int64_t)h * N + src) * rb, rb);
+  if (lane_id() == 0) {
+    b.knorm[bh + slot] = w.kperm_norm[(int64_t)h * b.n_max + j];
+    b.prov_step[bh + slot] = w.L->step;
+    b.prov_src[bh + slot] = src;
+    w.slot_new[(int64_t)h * b.n_max + j] = slot;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cudaStream_t s, Timer* t) {
+  timer_begin(t, "prepare", s);
+  k_prepare<<<1, 256, 0, s>>>(b, w, N, step);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
+  dim3 grid((N + 7) / 8, b.H);
+  timer_begin(t, "cand_norms", s);
+  if (b.bf16)
+    k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)Kc, (int64_t)N * b.d, N, nullptr, 0, N,
+                                                    w.cnorm, b.n_max, b.d);
+  else
+    k_row_norms<float><<<grid, 256, 0, s>>>((const float*)Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm,
+                                            b.n_max, b.d);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bank_norms(const Bank& b, cudaStream_t s, Timer* t) {
+  dim3 grid((b.M_max + 7) / 8, b.H);
+  timer_begin(t, "bank_norms", s);
+  if (b.bf16)
+    k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)b.k, (int64_t)b.M_max * b.d, b.M_max,
+                                                    b.occ, 1, 0, b.knorm, b.M_max, b.d);
+  else
+    k_row_norms<float><<<grid, 256, 0, s>>>((const float*)b.k, (int64_t)b.M_max * b.d, b.M_max, b.occ, 1, 0,
+                                            b.knorm, b.M_max, b.d);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
+  int n = 2;
+  while (n < b.n_max) n <<= 1;
+  timer_begin(t, "sort", s);
+  k_sort<<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
+  dim3 grid((N + 7) / 8, b.H);
+  timer_begin(t, "permute", s);
+  k_permute<<<grid, 256, 0, s>>>(b, w, (const char*)Kc, N, b.bf16 ? 2 : 4);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  timer_begin(t, "rstar", s);
+  k_rstar_head<<<b.H, BIG, 0, s>>>(w);
+  k_rstar_layer<<<1, BIG, 0, s>>>(b, w, kp.sync_heads);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
+  timer_begin(t, "select", s);
+  k_select<<<b.H, BIG, 0, s>>>(b, w);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
+  dim3 grid((b.M_max + 7) / 8, b.H);
+  timer_begin(t, "gather", s);
+  k_gather<<<grid, 256, 0, s>>>(b, w, b.bf16 ? 2 : 4);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t) {
+  dim3 grid((N + 7) / 8, b.H);
+  timer_begin(t, "commit", s);
+  k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4);
+  timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t update_set_smem_limits() {
+  return cudaFuncSetAttribute(k_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8);
+}
+
+}  // namespace dkv

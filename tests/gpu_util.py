@@ -1,0 +1,218 @@
+"""Helpers of the GPU parity tests: teacher forcing and oracle-vs-CUDA comparison.
+
+The CUDA path is driven only through the C ABI binding (paper_2608_27922_gb300.dkv);
+expected values come only from the CPU oracle (oracle/) on the same seeded inputs.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, List, Optional, Tuple
+
+import numpy as np
+import torch
+
+import oracle
+import synth
+from paper_2608_27922_gb300 import dkv
+
+INT_MAX = 2 ** 31 - 1
+
+
+def to_dev(x: np.ndarray, dtype: torch.dtype) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to("cuda", dtype)
+
+
+def oracle_params(bank: dkv.BankLayer) -> oracle.Params:
+    p = bank.params
+    return oracle.Params(tau=float(p.tau), sigma=float(p.sigma), p=float(p.p), eps=float(p.eps),
+                         delta=float(np.float32(p.delta)), sync_heads=bool(p.sync_heads))
+
+
+def load_state(bank: dkv.BankLayer, ob: oracle.LayerBank) -> None:
+    """Writes the oracle's bank into the GPU bank buffers (slots 0..m-1) and imports it."""
+    for h, hb in enumerate(ob.heads):
+        m = hb.m
+        if m:
+            bank.k[h, :m] = to_dev(hb.K, bank.dtype)
+            bank.v[h, :m] = to_dev(hb.V, bank.dtype)
+            bank.rho[h, :m] = torch.from_numpy(hb.rho.astype(np.float32)).cuda()
+            bank.base[h, :m] = torch.from_numpy(hb.base.astype(np.float32)).cuda()
+            bank.prov_step[h, :m] = torch.from_numpy(hb.step.astype(np.int64)).cuda()
+            bank.prov_src[h, :m] = torch.from_numpy(hb.src.astype(np.int32)).cuda()
+    bank.import_state([hb.m for hb in ob.heads])
+
+
+def gpu_heads(bank: dkv.BankLayer) -> List[Dict[Tuple[int, int], tuple]]:
+    occ = bank.occupancy_host()
+    out = []
+    K = bank.k.float().cpu().numpy()
+    V = bank.v.float().cpu().numpy()
+    rho = bank.rho.cpu().numpy()
+    base = bank.base.cpu().numpy()
+    st = bank.prov_step.cpu().numpy()
+    sr = bank.prov_src.cpu().numpy()
+    kn = bank.knorm.cpu().numpy()
+    for h in range(bank.H):
+        d = {}
+        for i in range(occ[h]):
+            key = (int(st[h, i]), int(sr[h, i]))
+            assert key not in d, f"duplicate provenance {key} in head {h}"
+            d[key] = (K[h, i], V[h, i], float(rho[h, i]), float(base[h, i]), float(kn[h, i]), i)
+        out.append(d)
+    return out
+
+
+def oracle_heads(ob: oracle.LayerBank) -> List[Dict[Tuple[int, int], tuple]]:
+    out = []
+    for hb in ob.heads:
+        out.append({(int(a), int(b)): (hb.K[i], hb.V[i], float(hb.rho[i]), float(hb.base[i]))
+                    for i, (a, b) in enumerate(zip(hb.step, hb.src))})
+    return out
+
+
+@dataclasses.dataclass
+class Report:
+    rstar_gpu: int = 0
+    rstar_oracle: int = 0
+    score_max_rel: float = 0.0
+    perm_mismatch: int = 0
+    perm_unexplained: int = 0
+    cross_mismatch: int = 0
+    cross_unexplained: int = 0
+    set_mismatch: int = 0
+    set_unexplained: int = 0
+    rho_max_rel: float = 0.0
+    base_max_rel: float = 0.0
+    rho_tilde_max_rel: float = 0.0
+    kv_bit_exact: bool = True
+    notes: List[str] = dataclasses.field(default_factory=list)
+
+    def ok(self) -> bool:
+        return (self.perm_unexplained == 0 and self.cross_unexplained == 0 and self.set_unexplained == 0
+                and self.kv_bit_exact)
+
+
+def _g_row(hb: oracle.HeadBank, i: int, Kpi: np.ndarray, r: int, prm: oracle.Params) -> float:
+    """Oracle g_i(r) for one bank row and a given candidate order (Eq. C.3)."""
+    if r == 0:
+        return float(hb.rho[i]) / float(hb.base[i])
+    w = oracle.soft_riesz(oracle.sq_dist(hb.K[i:i + 1], Kpi[:r]), prm, hb.d)[0]
+    return (float(hb.rho[i]) + float(w.sum())) / float(hb.base[i])
+
+
+def update_and_compare(bank: dkv.BankLayer, ob: oracle.LayerBank, K: np.ndarray, V: np.ndarray, step: int,
+                       tol: float, dens_tol: float) -> Tuple[Report, oracle.UpdateRecord]:
+    """Teacher-forced update: the GPU starts from the oracle's bank; both apply one update.
+
+    tol: relative window within which a decision may differ (near-tie of s, g vs tau,
+    rho~ vs the fill cutoff).  dens_tol: relative tolerance of s, rho~, rho and b.
+    ``ob`` is advanced by the oracle's update.
+    """
+    prm = oracle_params(bank)
+    before = ob.copy()
+    load_state(bank, before)
+    Kd, Vd = to_dev(K, bank.dtype), to_dev(V, bank.dtype)
+    bank.admit(Kd, Vd, step)
+    bank.compress()
+    bank.sync()
+    rec = oracle.update_layer(ob, K, V, step, prm)
+    L, hs = bank.stats()
+    inter = {k: v.cpu().numpy().copy() for k, v in bank.intermediates().items()}
+    rep = Report(rstar_gpu=L.r_star, rstar_oracle=rec.r_star)
+    N = K.shape[1]
+    Kq = K.astype(np.float64)
+    for h, (hb, hr) in enumerate(zip(before.heads, rec.heads)):
+        if hr.empty_init:
+            continue
+        s_g = inter["score"][h, :N]
+        rel = np.abs(s_g - hr.s) / np.maximum(np.abs(hr.s), 1e-30)
+        rep.score_max_rel = max(rep.score_max_rel, float(rel.max()))
+        pg = inter["perm"][h, :N]
+        diff = np.nonzero(pg != hr.pi)[0]
+        rep.perm_mismatch += len(diff)
+        for j in diff:
+            a, b = hr.s[pg[j]], hr.s[hr.pi[j]]
+            if abs(a - b) > tol * max(abs(a), abs(b)):
+                rep.perm_unexplained += 1
+        # crossing index per bank row (only comparable when both orders agree)
+        if len(diff) == 0:
+            cg = inter["cross"][h, :hb.m].astype(np.int64)
+            co = np.where(hr.cross < 0, INT_MAX, hr.cross)
+            bad = np.nonzero(cg != co)[0]
+            rep.cross_mismatch += len(bad)
+            Kpi = Kq[h][hr.pi]
+            for i in bad:
+                rs = [int(x) for x in (cg[i], co[i]) if x != INT_MAX]
+                near = any(abs(_g_row(hb, i, Kpi, r, prm) - prm.tau) <= tol * prm.tau for r in rs)
+                near |= any(abs(_g_row(hb, i, Kpi, r - 1, prm) - prm.tau) <= tol * prm.tau for r in rs if r > 0)
+                if not near:
+                    rep.cross_unexplained += 1
+            if rec.r_star == L.r_star:
+                rt = inter["rho_tilde"][h, :hb.m]
+                rel = np.abs(rt - hr.rho_tilde) / np.maximum(np.abs(hr.rho_tilde), 1e-30)
+                rep.rho_tilde_max_rel = max(rep.rho_tilde_max_rel, float(rel.max()))
+    if rep.rstar_gpu != rep.rstar_oracle:
+        rep.notes.append(f"r* gpu {rep.rstar_gpu} oracle {rep.rstar_oracle}")
+    else:
+        for h, (st, hr) in enumerate(zip(hs, rec.heads)):
+            if st.admitted != hr.r_used or st.evicted != len(hr.evicted):
+                rep.set_unexplained += 1
+                rep.notes.append(f"head {h}: admitted/evicted gpu {st.admitted}/{st.evicted} "
+                                 f"oracle {hr.r_used}/{len(hr.evicted)}")
+            if not hr.empty_init and st.mandatory != int(hr.mandatory.sum()):
+                rep.notes.append(f"head {h}: mandatory gpu {st.mandatory} oracle {int(hr.mandatory.sum())}")
+    # committed banks, compared as sets keyed by provenance
+    G = gpu_heads(bank)
+    Oh = oracle_heads(ob)
+    for h in range(bank.H):
+        g, o = G[h], Oh[h]
+        only_g = set(g) - set(o)
+        only_o = set(o) - set(g)
+        rep.set_mismatch += len(only_g) + len(only_o)
+        if only_g or only_o:
+            hr = rec.heads[h]
+            hb = before.heads[h]
+            ok = rep.rstar_gpu == rep.rstar_oracle and hr.rho_tilde is not None
+            if ok:
+                # an eviction decision within `tol` of its cutoff explains the difference
+                e = len(hr.evicted)
+                fill = [i for i in hr.evicted if not hr.mandatory[i]]
+                cut = min(hr.rho_tilde[fill]) if fill else None
+                prov_index = {(int(a), int(b)): i for i, (a, b) in enumerate(zip(hb.step, hb.src))}
+                for key in only_g | only_o:
+                    i = prov_index.get(key)
+                    if i is None:      # a candidate admitted on one side only
+                        ok = False
+                        break
+                    gi = hr.g_star[i]
+                    near_tau = abs(gi - prm.tau) <= tol * prm.tau
+                    near_cut = cut is not None and abs(hr.rho_tilde[i] - cut) <= tol * abs(cut)
+                    if not (near_tau or near_cut):
+                        ok = False
+                        break
+            if not ok:
+                rep.set_unexplained += len(only_g) + len(only_o)
+        for key in set(g) & set(o):
+            kg, vg, rg, bg, kn, _ = g[key]
+            ko, vo, ro, bo = o[key]
+            if not (np.array_equal(kg, ko.astype(np.float32)) and np.array_equal(vg, vo.astype(np.float32))):
+                rep.kv_bit_exact = False
+            rep.rho_max_rel = max(rep.rho_max_rel, abs(rg - ro) / max(abs(ro), 1e-30))
+            rep.base_max_rel = max(rep.base_max_rel, abs(bg - bo) / max(abs(bo), 1e-30))
+    return rep, rec
+
+
+def attention_error(bank: dkv.BankLayer, ob: oracle.LayerBank, Q: np.ndarray, Kw: Optional[np.ndarray],
+                    Vw: Optional[np.ndarray]) -> float:
+    """Max abs error of the CUDA attention against the oracle on the GPU bank's current contents."""
+    O = bank.attend(to_dev(Q, bank.dtype), None if Kw is None else to_dev(Kw, bank.dtype),
+                    None if Vw is None else to_dev(Vw, bank.dtype)).float().cpu().numpy()
+    H = Q.shape[0]
+    err = 0.0
+    for h in range(H):
+        kw = np.zeros((0, Q.shape[2])) if Kw is None else Kw[h]
+        vw = np.zeros((0, Q.shape[2])) if Vw is None else Vw[h]
+        ref = oracle.attend(ob.heads[h], Q[h], kw, vw)
+        err = max(err, float(np.abs(O[h] - ref).max()))
+    return err

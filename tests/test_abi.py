@@ -1,0 +1,116 @@
+"""The C ABI library builds, loads and exports every symbol include/*.h declares.
+
+CPU only: no call here launches GPU work.  Struct layouts of the ctypes binding are
+checked against a C compiler's view of include/dkv.h.
+"""
+import ctypes
+import glob
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = sorted(glob.glob(os.path.join(ROOT, "include", "*.h")))
+
+
+def _built_lib():
+    from paper_2608_27922_gb300 import build as B
+    if not os.path.exists(B.LIB):
+        if not (shutil.which("nvcc") or os.path.exists("/usr/local/cuda/bin/nvcc")):
+            pytest.skip("nvcc unavailable and the library is not built")
+        B.build()
+    from paper_2608_27922_gb300 import dkv
+    return dkv
+
+
+def _declared_functions():
+    names = set()
+    for h in HEADERS:
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w\s\*]*?\b(dkv_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+def test_header_declares_the_hot_path():
+    names = _declared_functions()
+    for required in ("dkv_bank_create", "dkv_bank_admit", "dkv_bank_compress", "dkv_bank_attend",
+                     "dkv_bank_destroy", "dkv_bank_workspace_size"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported():
+    dkv = _built_lib()
+    L = dkv.lib()
+    declared = _declared_functions()
+    missing = [n for n in sorted(declared) if not hasattr(L, n)]
+    assert not missing, missing
+    bound = {n for n, _, _ in dkv.SIGNATURES}
+    assert declared <= bound, sorted(declared - bound)
+
+
+def test_struct_layouts_match_c():
+    dkv = _built_lib()
+    if not shutil.which("gcc"):
+        pytest.skip("gcc unavailable")
+    src = r"""
+#include <stdio.h>
+#include <stddef.h>
+#include "dkv.h"
+int main(void) {
+  printf("%zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t), sizeof(dkv_layer_stats_t),
+         sizeof(dkv_head_stats_t), sizeof(dkv_intermediates_t), offsetof(dkv_buffers_t, workspace_bytes));
+  return 0;
+}
+"""
+    tmp = os.path.join(ROOT, "tests", "_abi_layout_probe")
+    with open(tmp + ".c", "w") as f:
+        f.write(src)
+    try:
+        subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), tmp + ".c", "-o", tmp])
+        out = subprocess.check_output([tmp]).decode().split()
+    finally:
+        for p in (tmp + ".c", tmp):
+            if os.path.exists(p):
+                os.remove(p)
+    sizes = [int(x) for x in out]
+    assert sizes == [ctypes.sizeof(dkv.dkv_params_t), ctypes.sizeof(dkv.dkv_buffers_t),
+                     ctypes.sizeof(dkv.dkv_layer_stats_t), ctypes.sizeof(dkv.dkv_head_stats_t),
+                     ctypes.sizeof(dkv.dkv_intermediates_t), dkv.dkv_buffers_t.workspace_bytes.offset]
+
+
+def test_host_only_entry_points():
+    dkv = _built_lib()
+    L = dkv.lib()
+    for s in range(9):
+        assert L.dkv_status_str(s)
+    assert dkv.dkv_version() >= 100
+    p = dkv.dkv_params_default(128)
+    assert (p.tau, p.sigma, p.p, p.eps, p.sync_heads) == (2.0, 8.0, 2.0, 1.0, 1)
+    assert abs(p.delta - 1e-6) < 1e-12
+    assert dkv.dkv_params_default(64).sigma == pytest.approx(32 ** 0.5)
+    # workspace size: positive for valid shapes, zero for invalid ones
+    assert dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16) > 0
+    assert dkv.dkv_bank_workspace_size(12, 96, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16) == 0
+    assert dkv.dkv_bank_workspace_size(2, 64, [0, 5], 16, dkv.DKV_DTYPE_FP32) == 0
+    assert dkv.dkv_bank_workspace_size(2, 64, [5, 5], 1 << 20, dkv.DKV_DTYPE_FP32) == 0
+    # argument errors are reported before any CUDA call
+    h = ctypes.c_void_p()
+    assert L.dkv_bank_create(ctypes.byref(h), 2, 64, None, 16, 1, None, None) == 1
+    assert L.dkv_bank_admit(None, None, None, 1, 0, None) == 1
+    assert L.dkv_bank_compress(None, None) == 1
+    assert L.dkv_bank_attend(None, None, 1, None, None, 0, None, None) == 1
+    assert L.dkv_bank_sync(None) == 1
+    L.dkv_bank_destroy(None)
+
+
+def test_binding_has_no_fallback(monkeypatch):
+    from paper_2608_27922_gb300 import dkv
+    monkeypatch.setattr(dkv, "LIB_PATH", "/nonexistent/libdkv.so")
+    monkeypatch.setattr(dkv, "_LIB", None)
+    with pytest.raises(RuntimeError):
+        dkv.lib()

@@ -1,0 +1,197 @@
+"""GPU parity of the bank update and attention against the CPU oracle (through the C ABI).
+
+Teacher-forced: before every update the GPU bank is loaded with the oracle's bank,
+both apply the same update, and s, pi, cross, r*, the retained sets, the K/V bits and
+rho / b are compared.  In the fp32 score mode the decisions must be identical up to
+near-ties of fp32 rounding; in the tensor-core mode (bf16 operands, fp32 accumulation)
+they may differ only within 1e-3 relative of a cutoff, and densities agree to 1e-2.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_util import attention_error, load_state, to_dev, update_and_compare, oracle_params
+
+pytestmark = pytest.mark.gpu
+
+# fp32 score mode: sums of up to ~1e4 fp32 terms; near-tie window well above their rounding
+FP32_TOL, FP32_DENS = 2e-4, 2e-4
+# tensor-core mode: bf16 inputs exact, products exact, fp32 accumulation (spec bounds)
+TC_TOL, TC_DENS = 1e-3, 1e-2
+
+
+@pytest.fixture(scope="module")
+def dkv():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_27922_gb300 import dkv as d
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    return d
+
+
+def _mode(dkv, name):
+    return {"fp32": dkv.DKV_SCORE_FP32, "tc": dkv.DKV_SCORE_TENSOR}[name]
+
+
+def _tols(name):
+    return (FP32_TOL, FP32_DENS) if name == "fp32" else (TC_TOL, TC_DENS)
+
+
+def _bank(dkv, wl, mode, layer=0, n_max=None, **kw):
+    dt = torch.float32 if wl.dtype == "fp32" else torch.bfloat16
+    try:
+        b = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(layer), n_max or wl.N, dt, score_mode=mode, **kw)
+    except dkv.DkvError as e:
+        if e.status == 7:
+            pytest.skip("tensor-core mode unavailable in this build")
+        raise
+    b.reset()
+    return b
+
+
+def _rollout(dkv, wl, mode_name, steps=None, check_attn=True, layer=0, **kw):
+    bank = _bank(dkv, wl, _mode(dkv, mode_name), layer, **kw)
+    tol, dens = _tols(mode_name)
+    ro = synth.LayerRollout(wl, layer)
+    ob = oracle.LayerBank.empty(wl.budgets_of_layer(layer), wl.d)
+    reports = []
+    for t in range(steps or wl.steps):
+        if check_attn:
+            Q = ro.queries(t)
+            Kw, Vw = ro.window(t)
+            load_state(bank, ob)
+            err = attention_error(bank, ob, Q, Kw, Vw)
+            assert err < (1e-4 if wl.dtype == "fp32" and mode_name == "fp32" else 2e-2), (t, err)
+        b = wl.admitted_block(t)
+        if b is None:
+            continue
+        K, V = ro.block(b)
+        rep, rec = update_and_compare(bank, ob, K, V, b, tol, dens)
+        reports.append(rep)
+        assert rep.ok(), (t, rep)
+        assert rep.rstar_gpu == rep.rstar_oracle, (t, rep)
+        assert rep.score_max_rel <= dens and rep.rho_tilde_max_rel <= dens, (t, rep)
+        assert rep.rho_max_rel <= dens * 5 and rep.base_max_rel <= dens * 5, (t, rep)
+    bank.close()
+    return reports
+
+
+@pytest.mark.parametrize("mode", ["fp32"])
+def test_tiny_fp32_workload_full_rollout(dkv, mode):
+    """1 layer x 2 heads, d = 64, fp32, 256-token blocks into a 512-token bank, 6 steps."""
+    wl = synth.get_workload("tiny_fp32_l1h2_d64")
+    reps = _rollout(dkv, wl, mode)
+    # eviction happens and the retained sets are identical in fp32 mode
+    assert sum(r.set_mismatch for r in reps) == 0
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_ragged_bf16_rollout(dkv, mode):
+    """d = 128 bf16, sizes off the tile grid (N = 300, M = 700, 3 heads)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=3, N=300, W=200, Nq=130, budgets=700, steps=7)
+    _rollout(dkv, wl, mode)
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_frozen_regime_literal_kappa(dkv, mode):
+    """Literal kappa (near-isotropic keys): the bank saturates and r* drops to 0 (no change)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=200, W=64, Nq=64, budgets=400, steps=6,
+                            kappa_per_dim=False)
+    reps = _rollout(dkv, wl, mode, check_attn=False)
+    assert any(r.rstar_oracle == 0 for r in reps)
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_empty_bank_with_more_candidates_than_budget(dkv, mode):
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=300, W=32, Nq=32, budgets=200, steps=4)
+    reps = _rollout(dkv, wl, mode, check_attn=False)
+    assert reps[0].rstar_oracle == 200
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_heterogeneous_budgets_shared_and_independent(dkv, mode):
+    budgets = (150, 300, 450, 600)
+    for sync in (1, 0):
+        wl = synth.get_workload("wan14b_headwise_l40h40", L=1, H=4, N=220, W=64, Nq=64, budgets=budgets,
+                                steps=6)
+        _rollout(dkv, wl, mode, check_attn=False, sync_heads=sync)
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+@pytest.mark.parametrize("p,sigma,tau", [(1.0, 8.0, 2.0), (4.0, 16.0, 1.5), (2.0, 4.0, 3.0)])
+def test_parameter_sweeps(dkv, mode, p, sigma, tau):
+    """Table 2a ranges: p in {1, 2, 4}, sigma in {4, 8, 16}, tau in {1.5, 2, 3}."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=140, W=32, Nq=32, budgets=260, steps=5)
+    _rollout(dkv, wl, mode, check_attn=False, p=p, sigma=sigma, tau=tau)
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_single_candidate_and_duplicates(dkv, mode):
+    """N = 1 updates, and blocks made of repeated keys (score ties -> source order;
+    fill ties -> the older state is evicted first)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=1, W=8, Nq=8, budgets=3, steps=8)
+    _rollout(dkv, wl, mode, check_attn=False)
+    import gpu_util
+    bank = _bank(dkv, synth.get_workload("wan13b_layer_h12", H=1, N=8, budgets=12), _mode(dkv, mode))
+    ob = oracle.LayerBank.empty([12], 128)
+    rng = np.random.default_rng(0)
+    base_key = synth.round_to_bf16(rng.standard_normal((1, 1, 128)).astype(np.float32) * 3)
+    for t in range(5):
+        K = np.repeat(base_key, 8, axis=1) if t % 2 == 0 else \
+            synth.round_to_bf16(rng.standard_normal((1, 8, 128)).astype(np.float32) * 11)
+        V = synth.round_to_bf16(rng.standard_normal((1, 8, 128)).astype(np.float32))
+        tol, dens = _tols(mode)
+        rep, _ = gpu_util.update_and_compare(bank, ob, K, V, t, tol, dens)
+        assert rep.ok() and rep.rstar_gpu == rep.rstar_oracle, (t, rep)
+    bank.close()
+
+
+def test_call_order_and_argument_errors(dkv):
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=16, budgets=32)
+    bank = _bank(dkv, wl, dkv.DKV_SCORE_FP32)
+    K = torch.zeros(2, 16, 128, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(dkv.DkvError) as e:
+        bank.compress()
+    assert e.value.status == 3
+    bank.admit(K, K, 0)
+    with pytest.raises(dkv.DkvError) as e:
+        bank.admit(K, K, 1)
+    assert e.value.status == 3
+    bank.compress()
+    big = torch.zeros(2, 17, 128, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(dkv.DkvError) as e:
+        bank.admit(big, big, 2)
+    assert e.value.status == 2
+    with pytest.raises(dkv.DkvError) as e:
+        dkv.dkv_bank_admit(bank.handle, K, K, 16, -1)
+    assert e.value.status == 1
+    with pytest.raises(dkv.DkvError) as e:
+        bank.import_state([33, 0])
+    assert e.value.status == 2
+    bank.sync()
+    assert bank.occupancy_host() == [16, 16]
+    bank.reset()
+    assert bank.occupancy_host() == [0, 0]
+    bank.close()
+
+
+def test_device_error_word_reports_inconsistent_bank(dkv):
+    """A bank whose occupancy exceeds its budget (written behind the library's back) is
+    reported by dkv_bank_sync as a device-side consistency failure, and the handle stays usable."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=16, budgets=32)
+    bank = _bank(dkv, wl, dkv.DKV_SCORE_FP32)
+    bank.occupancy.fill_(40)
+    K = torch.zeros(2, 16, 128, dtype=torch.bfloat16, device="cuda")
+    bank.admit(K, K, 0)
+    bank.compress()
+    with pytest.raises(dkv.DkvError) as e:
+        bank.sync()
+    assert e.value.status == 8
+    bank.sync()   # the word is cleared once reported
+    bank.reset()
+    bank.update(K, K, 1)
+    bank.sync()
+    bank.close()
