@@ -334,7 +334,7 @@ dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const v
   if (!aligned(Q, 16) || !aligned(O, 16) || (W > 0 && (!aligned(Kw, 16) || !aligned(Vw, 16)))) return DKV_ERR_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   bank->last = s;
-  cudaError_t e = bank->tc ? launch_attend_tc(bank->b, Q, Nq, Kw, Vw, W, O, s, &bank->timer)
+  cudaError_t e = bank->tc ? launch_attend_tc(bank->b, bank->w.L, Q, Nq, Kw, Vw, W, O, s, &bank->timer)
                            : launch_attend_fp32(bank->b, Q, Nq, Kw, Vw, W, O, s, &bank->timer);
   return cuda_status(e);
 }

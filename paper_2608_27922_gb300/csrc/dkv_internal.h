@@ -84,8 +84,8 @@ cudaError_t launch_set_occupancy(const Bank& b, const int32_t* occ_dev_src, int 
 // attention
 cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,
                                void* O, cudaStream_t s, Timer* t);
-cudaError_t launch_attend_tc(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,
-                             void* O, cudaStream_t s, Timer* t);
+cudaError_t launch_attend_tc(const Bank& b, DevLayer* L, const void* Q, int Nq, const void* Kw, const void* Vw,
+                             int W, void* O, cudaStream_t s, Timer* t);
 bool tc_supported(int d, int bf16);
 cudaError_t simt_set_smem_limits();
 cudaError_t update_set_smem_limits();
