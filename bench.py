@@ -1,0 +1,473 @@
+#!/usr/bin/env python3
+"""Benchmark of the DensityKV hot path on GB300: bank update + bank-reading attention.
+
+One step = one rollout step of one layer (all H heads): attention of the current
+block's queries over [bank | window], then admit + compress of the block leaving
+the window (Sec. 3.4, Alg. 1), all through the C ABI (libdkv.so).
+
+Default workload: the Wan-1.3B-shaped single layer (12 heads, d = 128, bf16,
+4,680-token blocks, 9,360-token bank, window = previous block, 4,680 queries),
+synthetic clustered keys from ``synth``.  W warm-up steps start from an empty bank
+(the first two fill it, eviction starts at the third), then K steps are timed one
+by one with CUDA events on the launching stream; a 256 MiB buffer is written
+between timed steps to flush the 129 MB L2.
+
+Metric: bank keys scored per second = sum over heads of (m_h + N) per update
+(every bank key's projected growth and every candidate are scored) / step time.
+
+``--impl reference`` times the CPU oracle (oracle/, numpy float64) on the host
+cores, each step a bounded sample of the same workload (one head).
+
+Multi-GPU (torchrun): every rank runs an independent layer of the same shape (the
+bank update and attention are per layer and head, with no exchange), so no
+collective is on the data path; ranks meet only at the barriers around the timed
+region and in a max-reduction of the elapsed time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "bank keys scored/s (update+attention)"
+UNIT = "keys/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=17)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="wan13b_layer_h12")
+    ap.add_argument("--score-mode", choices=["tensor", "fp32"], default="tensor")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between steps")
+    ap.add_argument("--heads", type=int, default=0, help="override the head count (profiling runs)")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, enabled: bool = True):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f".clocks_{os.getpid()}.csv")
+        self.idx = gpu_index
+        if not enabled:
+            return
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-i", str(gpu_index), "-lms", "200"], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, v in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"),
+                               parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------- helpers
+def peaks():
+    if os.path.exists(PEAKS_FILE):
+        p = json.load(open(PEAKS_FILE))
+        return p, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def source_sha1(*names):
+    h = hashlib.sha1()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2608_27922_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def traffic_for(kernel: str, src_files):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    t = json.load(open(TRAFFIC_FILE)).get(kernel)
+    if not t or t.get("source_sha1") != source_sha1(*src_files):
+        return None
+    return t.get("bytes_per_launch")
+
+
+def make_workload(name, world, heads=0):
+    import synth
+    over = {}
+    if heads:
+        over["H"] = heads
+    wl = synth.get_workload(name, **over)
+    if world > wl.L:
+        wl = synth.get_workload(name, L=world, **over)
+    return wl
+
+
+class Inputs:
+    """Host copies of the blocks and queries of steps [0, n) of one layer's rollout."""
+
+    def __init__(self, wl, layer, n_steps):
+        import synth
+        self.wl = wl
+        ro = synth.LayerRollout(wl, layer)
+        need = set()
+        for t in range(n_steps):
+            need.add(wl.window_block(t))
+            b = wl.admitted_block(t)
+            if b is not None:
+                need.add(b)
+        self.blocks = {b: ro.block(b) for b in sorted(need)}
+        self.queries = [ro.queries(t) for t in range(n_steps)]
+
+
+# --------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    import __graft_entry__
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    from paper_2608_27922_gb300 import dkv
+
+    wl = make_workload(args.workload, world, args.heads)
+    layer = rank
+    W, K = args.warmup, args.steps
+    n_total = W + K + (0 if args.no_e2e else K)
+    inp = Inputs(wl, layer, n_total)
+    bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    dblocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
+    dq = [torch.from_numpy(q).to(dev, bf) for q in inp.queries[:W + K]]
+    mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
+    bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(layer), wl.N, bf, score_mode=mode, device=dev)
+    bank.reset()
+    out = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(t, Q, KW, VW, KC, VC):
+        bank.attend(Q, KW, VW, out=out)
+        b = wl.admitted_block(t)
+        if b is not None:
+            bank.admit(KC, VC, b)
+            bank.compress()
+
+    def device_step(t):
+        kw, vw = dblocks[wl.window_block(t)]
+        b = wl.admitted_block(t)
+        kc, vc = dblocks[b] if b is not None else (None, None)
+        step(t, dq[t], kw, vw, kc, vc)
+
+    for t in range(W):
+        device_step(t)
+    bank.sync()
+
+    # ---- timed region: K steps, CUDA events on the launching stream, L2 flushed between steps
+    clocks = ClockSampler(local, enabled=(not args.no_clocks) and rank == 0)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    bank.set_timing(True)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    keys = 0
+    stats = []
+    wall0 = time.perf_counter()
+    for i in range(K):
+        t = W + i
+        if not args.no_flush:
+            flush.fill_(float(i))
+        ev[i][0].record(stream)
+        device_step(t)
+        ev[i][1].record(stream)
+        ev[i][1].synchronize()
+        L, hs = bank.stats()
+        if wl.admitted_block(t) is not None:
+            keys += sum(h.occupancy_before + wl.N for h in hs)
+        # occupancy_before is the bank this step's attention read
+        stats.append((L.r_star, sum(h.evicted for h in hs), sum(h.mandatory for h in hs),
+                      sum(h.occupancy_before for h in hs)))
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    ktimes = bank.kernel_times()
+    bank.set_timing(False)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    clk = clocks.stop()
+    bank.sync()
+    total_ms = sum(step_ms)
+    if world > 1:
+        tt = torch.tensor([total_ms, keys], dtype=torch.float64, device=dev)
+        mx = tt.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        sm = tt.clone()
+        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+        total_ms_max, keys_all = float(mx[0]), float(sm[1])
+    else:
+        total_ms_max, keys_all = total_ms, float(keys)
+    value = keys_all / (total_ms_max / 1e3)
+
+    # ---- end to end through the C ABI with host buffers: H2D inputs, compute, D2H output
+    e2e = None
+    if not args.no_e2e:
+        host_blocks = {b: (torch.from_numpy(k).to(bf).pin_memory(), torch.from_numpy(v).to(bf).pin_memory())
+                       for b, (k, v) in inp.blocks.items()}
+        host_q = [torch.from_numpy(q).to(bf).pin_memory() for q in inp.queries[W + K:]]
+        host_out = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf).pin_memory()
+        kbuf = torch.empty(wl.H, wl.N, wl.d, dtype=bf, device=dev)
+        vbuf = torch.empty_like(kbuf)
+        kw_buf = torch.empty(wl.H, wl.W, wl.d, dtype=bf, device=dev)
+        vw_buf = torch.empty_like(kw_buf)
+        qbuf = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
+        e2e_keys = 0
+        e2e_ms = 0.0
+        h2d = d2h = 0
+        for i in range(K):
+            t = W + K + i
+            if not args.no_flush:
+                flush.fill_(float(i))
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            s0.record(stream)
+            wb = wl.window_block(t)
+            ab = wl.admitted_block(t)
+            kw_buf.copy_(host_blocks[wb][0], non_blocking=True)
+            vw_buf.copy_(host_blocks[wb][1], non_blocking=True)
+            qbuf.copy_(host_q[i], non_blocking=True)
+            h2d_i = qbuf.numel() * qbuf.element_size() + 2 * kw_buf.numel() * kw_buf.element_size()
+            if ab is not None and ab != wb:
+                kbuf.copy_(host_blocks[ab][0], non_blocking=True)
+                vbuf.copy_(host_blocks[ab][1], non_blocking=True)
+                kc, vc = kbuf, vbuf
+                h2d_i += 2 * kbuf.numel() * kbuf.element_size()
+            else:
+                kc, vc = kw_buf, vw_buf   # the block leaving the window is the window block
+            step(t, qbuf, kw_buf, vw_buf, kc, vc)
+            host_out.copy_(out, non_blocking=True)
+            s1.record(stream)
+            s1.synchronize()
+            e2e_ms += s0.elapsed_time(s1)
+            L, hs = bank.stats()
+            if ab is not None:
+                e2e_keys += sum(h.occupancy_before + wl.N for h in hs)
+            h2d += h2d_i
+            d2h += host_out.numel() * host_out.element_size()
+        if world > 1:
+            tt = torch.tensor([e2e_ms, e2e_keys], dtype=torch.float64, device=dev)
+            mx = tt.clone()
+            dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+            sm = tt.clone()
+            dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+            e2e_ms, e2e_keys = float(mx[0]), float(sm[1])
+        e2e = {"value": e2e_keys / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d // K,
+               "d2h_bytes_per_step": d2h // K, "ms_per_step": e2e_ms / K}
+
+    # ---- roofline of the dominant kernel (largest share of the timed region)
+    pk, pk_src = peaks()
+    launches = sum(v[0] for v in ktimes.values())
+    dom = max(ktimes.items(), key=lambda kv: kv[1][1])
+    dom_name, (dom_n, dom_ms) = dom
+    roof = None
+    m_bank = statistics.mean([s[3] / wl.H for s in stats]) if stats else 0
+    if dom_name.startswith("attend"):
+        # 2 flops per multiply-add in Q K^T and in P V over (m + W) keys per query
+        flops = 4.0 * wl.H * wl.Nq * (m_bank + wl.W) * wl.d
+        achieved = flops / (dom_ms / dom_n / 1e3) / 1e12
+        peak = float(pk["bf16_tflops"])
+        roof = {"kernel": dom_name, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "peak_source": f"{pk_src} bf16 dense (burst)",
+                "algorithmic_per_launch": {"flops": flops, "keys_per_query": m_bank + wl.W},
+                "traffic": traffic_for(dom_name, ["k_tc_attn.cu", "tc_ptx.cuh"])}
+    else:
+        roof = {"kernel": dom_name, "bound": "tensor", "achieved": None, "peak": float(pk["bf16_tflops"]),
+                "unit": "TFLOP/s", "frac": None, "traffic": None}
+    per_kernel = {k: {"launches": n, "avg_ms": ms / max(n, 1), "share": ms / max(sum(v[1] for v in ktimes.values()), 1e-9)}
+                  for k, (n, ms) in sorted(ktimes.items(), key=lambda kv: -kv[1][1])}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_sample(wl, layer)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+            "ms_per_step": total_ms_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": f"{wl.name}: {wl.L if world > 1 else 1} layer(s) x {wl.H} heads, d={wl.d}, "
+                                   f"N={wl.N}, M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
+                       "score_mode": args.score_mode, "layers_per_gpu": 1,
+                       "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
+                       "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
+            "blocks_per_s": world * K / (total_ms_max / 1e3),
+            "interaction_pairs_per_s": None,
+            "wall_s_timed": wall,
+            "e2e": e2e, "gpu_launches": launches * world, "roofline": roof, "cpu_baseline": cpu,
+            "clocks": clk, "per_kernel": per_kernel,
+            "update": {"r_star": [s[0] for s in stats], "evicted": [s[1] for s in stats],
+                       "mandatory": [s[2] for s in stats]},
+        }
+        print(json.dumps(line), flush=True)
+    bank.close()
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+# --------------------------------------------------------------------------- oracle timing
+def oracle_threads():
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(k):
+            return int(os.environ[k])
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def _oracle_head_setup(wl, layer, head):
+    """Oracle bank of one head brought to steady state (untimed): first two updates."""
+    import oracle
+    import synth
+    ro = synth.LayerRollout(wl, layer, heads=[head])
+    ob = oracle.LayerBank.empty([wl.budgets[layer * wl.H + head]], wl.d)
+    t = 0
+    while True:
+        b = wl.admitted_block(t)
+        if b is not None:
+            K, V = ro.block(b)
+            oracle.update_layer(ob, K, V, b)
+            if ob.heads[0].m >= ob.heads[0].M:
+                return ro, ob, t + 1
+        t += 1
+        if t > 8:
+            return ro, ob, t
+
+
+def _oracle_step(wl, ro, ob, t):
+    """One step of one head in the oracle: attention of all queries, then the update."""
+    import oracle
+    Q = ro.queries(t)
+    Kw, Vw = ro.window(t)
+    b = wl.admitted_block(t)
+    K, V = ro.block(b)
+    t0 = time.perf_counter()
+    oracle.attend(ob.heads[0], Q[0], Kw[0], Vw[0])
+    m = ob.heads[0].m
+    oracle.update_layer(ob, K, V, b)
+    return time.perf_counter() - t0, m + wl.N
+
+
+def cpu_baseline_sample(wl, layer):
+    ro, ob, t = _oracle_head_setup(wl, layer, 0)
+    dt, keys = _oracle_step(wl, ro, ob, t)
+    return {"value": keys / dt, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
+            "sample": f"1 head (of {wl.H}), 1 steady-state step of {wl.name}: attention of {wl.Nq} queries "
+                      f"+ bank update, {keys} keys scored in {dt:.2f} s (numpy float64)"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    wl = make_workload(args.workload, 1)
+    ro, ob, t = _oracle_head_setup(wl, 0, 0)
+    for i in range(args.warmup):
+        _oracle_step(wl, ro, ob, t)
+        t += 1
+    tot, keys = 0.0, 0
+    for i in range(args.steps):
+        dt, k = _oracle_step(wl, ro, ob, t)
+        tot += dt
+        keys += k
+        t += 1
+    value = keys / tot
+    cpu = {"value": value, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
+           "sample": f"each step: 1 head (of {wl.H}) of {wl.name} at steady state, attention of {wl.Nq} "
+                     f"queries + bank update (numpy float64)"}
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": f"{wl.name} (one head per step on the host CPU)"},
+            "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.warmup < 3:
+        print("warning: --warmup < 3 does not reach the steady state of the bank", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -470,8 +470,10 @@ cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cu
 }
 
 cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  timer_begin(t, "rstar", s);
+  timer_begin(t, "rstar_head", s);
   k_rstar_head<<<b.H, BIG, 0, s>>>(w);
+  timer_end(t, s);
+  timer_begin(t, "rstar_layer", s);
   k_rstar_layer<<<1, BIG, 0, s>>>(b, w, kp.sync_heads);
   timer_end(t, s);
   return cudaGetLastError();
