@@ -235,6 +235,42 @@ dkv_status_t dkv_bank_set_timing(dkv_bank_t bank, int32_t enable);
 dkv_status_t dkv_bank_kernel_times(dkv_bank_t bank, int32_t max_kernels, char* names /* [max][48] */,
                                    int32_t* launches, double* total_ms, int32_t* n_kernels);
 
+/* Largest candidate count accepted by dkv_candidate_order_noalloc. */
+#define DKV_NOALLOC_MAX_N 16384
+
+/* Candidate scores and order for ONE head, without any device allocation.
+ *
+ * The paper has no counterpart of this call; it exists for callers that cannot
+ * allocate device memory and so cannot provide the workspace of dkv_bank_create:
+ * code inside a framework whose pool owns every device byte, hosts that forbid
+ * allocation after start-up (real-time or embedded deployments), or plugins that
+ * are handed only fixed input and output buffers.  It computes what the first half
+ * of dkv_bank_admit computes for one head in the fp32 score mode: the Eq. 6 score
+ * of every candidate and the stable ascending order of those scores (ties in source
+ * order; an empty bank, m = 0, gives the source order and zero scores).
+ *
+ *   K_bank   : device [m][d] bank keys of the head, dtype
+ *   base     : device [m] frozen baselines b_i (fp32)
+ *   Kc       : device [N][d] candidate keys in source order, dtype
+ *   params   : host; tau, sigma, p, eps, delta as for dkv_bank_create (the other
+ *              fields are ignored)
+ *   scores_out : device [N] fp32, or NULL
+ *   perm_out : device [N] int32: perm_out[j] = candidate at sorted position j
+ *
+ * Limits: 1 <= N <= DKV_NOALLOC_MAX_N (else DKV_ERR_SHAPE, nothing is launched),
+ * 0 <= m <= 262144, d in {64, 128}.
+ * Memory: the scores live in a fixed 64 KiB device array inside the library (one
+ * per GPU that loads it, kept until the process exits); the call allocates nothing,
+ * on the device or through any library.  The first call on each device looks up
+ * that array's device address and sets a kernel attribute, once; make that first
+ * call before any stream capture.  Nothing in the array needs clearing: every
+ * entry a call reads is written earlier in the same call.  All calls on a device
+ * share the array, so calls whose work overlaps on the GPU (different streams
+ * without ordering between them) race; order them on one stream.               */
+dkv_status_t dkv_candidate_order_noalloc(const void* K_bank, const float* base, int32_t m, const void* Kc,
+                                         int32_t N, int32_t d, int32_t dtype, const dkv_params_t* params,
+                                         float* scores_out, int32_t* perm_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -79,7 +79,10 @@ SIGNATURES = [
     ("dkv_bank_set_timing", _I, [_P, _I]),
     ("dkv_bank_kernel_times", _I, [_P, _I, ctypes.c_char_p, ctypes.POINTER(ctypes.c_int32),
                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int32)]),
+    ("dkv_candidate_order_noalloc", _I, [_P, _P, _I, _P, _I, _I, _I, ctypes.POINTER(dkv_params_t), _P, _P, _P]),
 ]
+
+DKV_NOALLOC_MAX_N = 16384
 
 _LIB: Optional[ctypes.CDLL] = None
 
@@ -220,6 +223,15 @@ def dkv_bank_kernel_times(bank: int) -> Dict[str, Tuple[int, float]]:
         nm = names.raw[48 * i:48 * (i + 1)].split(b"\0", 1)[0].decode()
         out[nm] = (int(launches[i]), float(ms[i]))
     return out
+
+
+def dkv_candidate_order_noalloc(K_bank, base, m: int, Kc, N: int, d: int, dtype: int, params: dkv_params_t,
+                                scores_out, perm_out, stream=None) -> None:
+    """Eq. 6 scores and their stable order for one head, with no device allocation
+    (for callers that cannot allocate; see include/dkv.h)."""
+    _check(lib().dkv_candidate_order_noalloc(_ptr(K_bank) if m > 0 else 0, _ptr(base) if m > 0 else 0, m,
+                                             _ptr(Kc), N, d, dtype, ctypes.byref(params), _ptr(scores_out),
+                                             _ptr(perm_out), _stream(stream)), "dkv_candidate_order_noalloc")
 
 
 # ----------------------------------------------------------------- buffer owner
