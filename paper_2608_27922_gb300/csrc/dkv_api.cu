@@ -111,6 +111,11 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* ba
   w.ksurv = take(Hh * Mm * d * es);
   w.ksurv_norm = (float*)take(Hh * Mm * 4);
   w.slot_new = (int32_t*)take(Hh * Nm * 4);
+  w.cext = take(Hh * Nm * 64);
+  w.kperm_ext = take(Hh * Nm * 64);
+  w.bext = take(Hh * Mm * 64);
+  w.ksurv_ext = take(Hh * Mm * 64);
+  w.kevict_ext = take(Hh * Nm * 64);
   w.hist_stride = hist_stride;
   w.snap_stride = snap_stride;
   w.feas_words = feas_words;
@@ -291,7 +296,7 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   bank->last = s;
   cudaError_t e = cudaMemsetAsync(w.hist, 0, sizeof(int32_t) * (size_t)b.H * w.hist_stride, s);
   if (e == cudaSuccess) e = launch_prepare(b, w, N, step, s, t);
-  if (e == cudaSuccess) e = launch_cand_norms(b, w, Kc, N, s, t);
+  if (e == cudaSuccess) e = launch_cand_norms(b, w, Kc, N, bank->kp, s, t);
   if (e == cudaSuccess)
     e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_sort(b, w, s, t);
@@ -347,7 +352,7 @@ dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* st
   cudaStream_t s = (cudaStream_t)stream;
   bank->last = s;
   cudaError_t e = cudaMemcpyAsync(bank->b.occ, occupancy, sizeof(int32_t) * bank->b.H, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = launch_bank_norms(bank->b, s, &bank->timer);
+  if (e == cudaSuccess) e = launch_bank_norms(bank->b, bank->w, bank->kp, s, &bank->timer);
   return cuda_status(e);
 }
 

@@ -45,6 +45,12 @@ struct Ws {
   void* ksurv;          // [H][M_max][d]  keys of surviving states
   float* ksurv_norm;    // [H][M_max]
   int32_t* slot_new;    // [H][n_max]     bank slot of the j-th admitted candidate
+  // extension rows of the tensor-core passes, bf16 [..][32]: row form | column form
+  void* cext;           // [H][n_max][32] candidates, source order
+  void* kperm_ext;      // [H][n_max][32] candidates, pi order
+  void* bext;           // [H][M_max][32] bank (derived from the bank keys, kept in step)
+  void* ksurv_ext;      // [H][M_max][32]
+  void* kevict_ext;     // [H][n_max][32]
   int hist_stride, snap_stride, feas_words;
 };
 
@@ -59,7 +65,8 @@ void timer_end(Timer* t, cudaStream_t s);
 // ---- launches (each returns cudaGetLastError() of its launch) ----
 // update front half (admit)
 cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cudaStream_t s, Timer* t);
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
+                              Timer* t);
 cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t);
 cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t);
@@ -79,7 +86,7 @@ cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cud
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // bank maintenance
-cudaError_t launch_bank_norms(const Bank& b, cudaStream_t s, Timer* t);
+cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_set_occupancy(const Bank& b, const int32_t* occ_dev_src, int value, cudaStream_t s);
 // attention
 cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,

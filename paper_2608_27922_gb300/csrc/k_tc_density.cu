@@ -1,23 +1,39 @@
 // Tensor-core (tcgen05) pair passes of the bank update, bf16 keys, d = 128.
 //
-// Every pass contracts a tile of 128 "row" keys against a run of "column" keys:
-//   acc[i][j] = k_i . k_j                       (tcgen05.mma, bf16 in, fp32 in TMEM)
-//   u = eps + (|k_i|^2 + |k_j|^2 - 2 acc) / sigma^2,  w = u^-p     (Eq. 2, fp32 epilogue)
-// and folds w into a per-row quantity in the epilogue, so no row-by-column matrix
-// ever reaches global memory (App. C "Decision granularity versus computational
-// tiling"):
-//   SCORE    rows = candidates, cols = bank:         s(x) = (1/m) sum_i w / b_i   (Eq. 6)
-//   CROSS    rows = bank, cols = candidates in pi order: running rho~_i(r) (Eq. C.2),
-//            first r with rho~ >= tau b_i (Eqs. 8-9), snapshots every 128 columns
+// Every pass contracts a tile of 128 "row" keys against a run of "column" keys and
+// folds the Soft-Riesz interaction (Eq. 2) into a per-row quantity in the
+// epilogue, so no row-by-column matrix reaches global memory (App. C, "Decision
+// granularity versus computational tiling"):
+//   SCORE    rows = candidates, cols = bank:     s(x) = (1/m) sum_i w / b_i        (Eq. 6)
+//   CROSS    rows = bank, cols = candidates in pi order: running rho~_i(r) (Eq. C.2)
+//            and the first r with rho~_i(r) >= tau b_i (Eqs. 8-9); snapshots every
+//            128 columns
 //   PROJECT  rows = bank, cols = pi-ordered candidates [128 floor(r/128), r):
-//            rho~_i(r) resumed from the snapshot (same tiles, same arithmetic)
-//   SUB      rows = survivors, cols = evicted: rho_i = rho~_i - sum_R w     (Eq. C.4)
-//   NEWBASE  rows = admitted, cols = final bank (self excluded by index):
-//            rho_x = Phi(x), b_x = max(rho_x, delta)                 (Eq. 5 / C.4)
+//            rho~_i(r), resumed from the snapshot with the same arithmetic
+//   SUB      rows = survivors, cols = evicted:   rho_i = rho~_i - sum_R w       (Eq. C.4)
+//   NEWBASE  rows = admitted, cols = final bank, self excluded by index:
+//            rho_x = Phi(x), b_x = max(rho_x, delta)                     (Eq. 5 / C.4)
 //
-// CTA layout (192 threads, 2 CTAs per SM): warp 0 issues TMA (row tile once, column
-// tiles through a 2-stage ring), warp 1 issues tcgen05.mma into two 128-column TMEM
-// accumulators, warps 2-5 are the epilogue (thread = row = TMEM lane).
+// Distances inside the MMA.  Each key carries 32 extension bf16 values (two forms
+// of 16): row form [-g_hi, -g_mid, -g_lo, 1, 1, 1, 0..], column form
+// [1, 1, 1, -h_hi, -h_mid, -h_lo, 0..] with g = |k|^2/2 + eps sigma^2/2 and
+// h = |k|^2/2 split into three bf16 parts.  A ninth MMA k-step (K = 16) adds the
+// product of the row form and the column form, so the fp32 accumulator holds
+//   A = a.b - g_a - h_b = -(sigma^2/2) (eps + |a - b|^2 / sigma^2) = -(sigma^2/2) u,
+// and w = u^-p = c |A|^-p with c = (sigma^2/2)^p.  Sums are kept in units of
+// |A|^-p and scaled by c once per row.
+//
+// Epilogue arithmetic.  Two interactions share one reciprocal:
+//   |A1|^-2 + |A2|^-2 = (A1^2 + A2^2) / (A1 A2)^2,
+// and the 16 pair terms of a 32-column chunk are summed as a fixed binary tree, so
+// there is no serial dependence inside a chunk.  The crossing pass tests each
+// chunk total against the row's threshold and rescans a chunk term by term only
+// when the threshold falls inside it (at most once per row).
+//
+// CTA (320 threads, 2 per SM): warp 0 TMA producer, warp 1 MMA issuer, warps 2-9
+// epilogue.  Epilogue warps w and w+4 share TMEM lanes 32 (w % 4) .. +31 (one row
+// per lane) and split each 128-column tile into halves of 64 columns; the crossing
+// and projection passes exchange half totals through shared memory every tile.
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
@@ -32,21 +48,29 @@ using namespace tc;
 
 enum TMode { TM_SCORE = 0, TM_CROSS = 1, TM_PROJECT = 2, TM_SUB = 3, TM_NEWBASE = 4 };
 
-constexpr int BM = 128;          // rows per CTA (TMEM lanes)
-constexpr int BN = 128;          // columns per tile
-constexpr int TILE_BYTES = BM * 128 * 2;   // 128 rows x 128 bf16
-constexpr int HALF_BYTES = TILE_BYTES / 2; // one 64-column swizzle panel
+constexpr int BM = 128;                     // rows per CTA (TMEM lanes)
+constexpr int BN = 128;                     // columns per tile
+constexpr int TILE_BYTES = BM * 128 * 2;    // 128 rows x 128 bf16
+constexpr int HALF_BYTES = TILE_BYTES / 2;  // one 64-column 128-byte-swizzle panel
+constexpr int EXT_BYTES = BM * 16 * 2;      // 128 rows x 16 bf16 (32-byte swizzle)
 constexpr int STAGES = 2;
-constexpr int THREADS = 192;
-constexpr uint32_t TMEM_COLS = 256;        // two 128-column accumulators
-constexpr size_t SMEM_BYTES = 1024 /*align*/ + TILE_BYTES * (1 + STAGES) + 2 * 2 * BN * 4 /*meta*/ + 256;
+constexpr int EPI_WARPS = 8;
+constexpr int THREADS = 64 + 32 * EPI_WARPS;
+constexpr uint32_t TMEM_COLS = 256;         // two 128-column accumulators
+constexpr int OFF_A = 0;
+constexpr int OFF_AX = TILE_BYTES;
+constexpr int OFF_B = OFF_AX + EXT_BYTES;                 // [STAGES] tiles
+constexpr int OFF_BX = OFF_B + STAGES * TILE_BYTES;       // [STAGES] extension tiles
+constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [2][BN]
+constexpr int OFF_XCH = OFF_META + 2 * BN * 4;            // float [2][2][BM]
+constexpr int OFF_BAR = OFF_XCH + 2 * 2 * BM * 4;
+constexpr size_t SMEM_BYTES = 1024 + OFF_BAR + 128;
+constexpr uint32_t LOAD_BYTES = TILE_BYTES + EXT_BYTES;
 
 struct TcJob {
   Bank b;
   Ws w;
   KParams kp;
-  const float* rnorm;   // row key norms, head stride rn_hs
-  int64_t rn_hs;
 };
 
 __device__ __forceinline__ void job_range(int MODE, const DevHead& hd, const DevLayer& L, int& nrows, int& c0,
@@ -59,15 +83,84 @@ __device__ __forceinline__ void job_range(int MODE, const DevHead& hd, const Dev
   if (MODE == TM_NEWBASE) { nrows = hd.r; c1 = hd.m_new; }
 }
 
-template <int MODE>
+// |a|^-P for a < 0 (one reciprocal).
+template <int P>
+__device__ __forceinline__ float term1(float a) {
+  const float r = rcp_approx(a);
+  if (P == 1) return -r;
+  const float r2 = r * r;
+  return P == 2 ? r2 : r2 * r2;
+}
+
+// |a|^-P + |b|^-P for a, b < 0 (one reciprocal).
+template <int P>
+__device__ __forceinline__ float term2(float a, float b) {
+  const float R = rcp_approx(a * b);
+  if (P == 1) return -(a + b) * R;
+  const float R2 = R * R;
+  if (P == 2) return R2 * fmaf(a, a, b * b);
+  const float a2 = a * a, b2 = b * b;
+  return (R2 * R2) * fmaf(a2, a2, b2 * b2);
+}
+
+// wa |a|^-P + wb |b|^-P (one reciprocal).
+template <int P>
+__device__ __forceinline__ float term2w(float a, float b, float wa, float wb) {
+  const float R = rcp_approx(a * b);
+  if (P == 1) return -R * fmaf(wa, b, wb * a);
+  const float R2 = R * R;
+  if (P == 2) return R2 * fmaf(wa, b * b, wb * (a * a));
+  const float a2 = a * a, b2 = b * b;
+  return (R2 * R2) * fmaf(wa, b2 * b2, wb * (a2 * a2));
+}
+
+// Fixed-order binary tree over 16 values.
+__device__ __forceinline__ float tree16(float (&t)[16]) {
+#pragma unroll
+  for (int s = 8; s > 0; s >>= 1)
+#pragma unroll
+    for (int k = 0; k < s; ++k) t[k] += t[k + s];
+  return t[0];
+}
+
+// Sum of |v_j|^-P over a full 32-column chunk.
+template <int P>
+__device__ __forceinline__ float chunk_sum(const float (&v)[32]) {
+  float t[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) t[k] = term2<P>(v[2 * k], v[2 * k + 1]);
+  return tree16(t);
+}
+
+// Same over the first `lim` columns (lim < 32), term by term.
+template <int P>
+__device__ __forceinline__ float chunk_sum_partial(const float (&v)[32], int lim) {
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (j < lim) s += term1<P>(v[j]);
+  return s;
+}
+
+// Sum over `lim` columns skipping column `skip` (-1: none), term by term.
+template <int P>
+__device__ __forceinline__ float chunk_sum_skip(const float (&v)[32], int lim, int skip) {
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (j < lim && j != skip) s += term1<P>(v[j]);
+  return s;
+}
+
+template <int MODE, int P>
 __global__ void __launch_bounds__(THREADS, 2)
-    tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcJob j) {
+    tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
+             const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx, TcJob j) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + TILE_BYTES;
-  float* meta = reinterpret_cast<float*>(smem + TILE_BYTES * (1 + STAGES));   // [2 buf][2][BN]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(meta + 2 * 2 * BN);
+  float* meta = reinterpret_cast<float*>(smem + OFF_META);
+  float* xch = reinterpret_cast<float*>(smem + OFF_XCH);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* bar_a = bars + 0;
   uint64_t* bar_full = bars + 1;    // [STAGES]
   uint64_t* bar_empty = bars + 3;   // [STAGES]
@@ -89,7 +182,7 @@ __global__ void __launch_bounds__(THREADS, 2)
   if (threadIdx.x == 0) {
     mbar_init(bar_a, 1);
     for (int s = 0; s < STAGES; ++s) { mbar_init(bar_full + s, 1); mbar_init(bar_empty + s, 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(bar_accf + b, 1); mbar_init(bar_acce + b, 4); }
+    for (int b = 0; b < 2; ++b) { mbar_init(bar_accf + b, 1); mbar_init(bar_acce + b, EPI_WARPS); }
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -101,21 +194,22 @@ __global__ void __launch_bounds__(THREADS, 2)
 
   if (warp == 0) {
     if (lane == 0 && ntiles > 0) {
-      // ---------------- TMA producer
-      prefetch_map(&tmA);
-      prefetch_map(&tmB);
-      mbar_arrive_expect_tx(bar_a, TILE_BYTES);
-      tma_load_3d(sA, &tmA, bar_a, 0, row0, h);
-      tma_load_3d(sA + HALF_BYTES, &tmA, bar_a, 64, row0, h);
+      // ---------------- TMA producer: row tile (+ row-form extension) once, column tiles
+      prefetch_map(&tmA); prefetch_map(&tmAx); prefetch_map(&tmB); prefetch_map(&tmBx);
+      mbar_arrive_expect_tx(bar_a, LOAD_BYTES);
+      tma_load_3d(smem + OFF_A, &tmA, bar_a, 0, row0, h);
+      tma_load_3d(smem + OFF_A + HALF_BYTES, &tmA, bar_a, 64, row0, h);
+      tma_load_3d(smem + OFF_AX, &tmAx, bar_a, 0, row0, h);
       int issued = 0;
       for (int t = 0; t < ntiles; ++t) {
         const int s = t % STAGES;
-        const uint32_t ph = (t / STAGES) & 1;
-        if (!mbar_wait(bar_empty + s, ph ^ 1, abort_flag)) break;
-        mbar_arrive_expect_tx(bar_full + s, TILE_BYTES);
+        if (!mbar_wait(bar_empty + s, ((t / STAGES) & 1) ^ 1, abort_flag)) break;
+        mbar_arrive_expect_tx(bar_full + s, LOAD_BYTES);
         const int col = c0 + t * BN;
-        tma_load_3d(sB + s * TILE_BYTES, &tmB, bar_full + s, 0, col, h);
-        tma_load_3d(sB + s * TILE_BYTES + HALF_BYTES, &tmB, bar_full + s, 64, col, h);
+        uint8_t* dst = smem + OFF_B + s * TILE_BYTES;
+        tma_load_3d(dst, &tmB, bar_full + s, 0, col, h);
+        tma_load_3d(dst + HALF_BYTES, &tmB, bar_full + s, 64, col, h);
+        tma_load_3d(smem + OFF_BX + s * EXT_BYTES, &tmBx, bar_full + s, 16, col, h);
         issued = t + 1;
       }
       if (issued < ntiles) {
@@ -130,23 +224,26 @@ __global__ void __launch_bounds__(THREADS, 2)
     }
   } else if (warp == 1) {
     if (lane == 0 && ntiles > 0) {
-      // ---------------- MMA issuer
+      // ---------------- MMA issuer: 8 k-steps of the keys + 1 of the extension
       constexpr uint32_t idesc = idesc_bf16(BM, BN);
       bool ok = mbar_wait(bar_a, 0, abort_flag);
-      const uint32_t a_base = smem_u32(sA);
+      const uint32_t a_base = smem_u32(smem + OFF_A);
+      const uint32_t ax_base = smem_u32(smem + OFF_AX);
       int done = 0;
       for (int t = 0; ok && t < ntiles; ++t) {
         const int s = t % STAGES;
         const int b = t & 1;
-        if (!mbar_wait(bar_full + s, (t / STAGES) & 1, abort_flag)) { ok = false; break; }
-        if (!mbar_wait(bar_acce + b, ((t >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        if (!(ok = mbar_wait(bar_full + s, (t / STAGES) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait(bar_acce + b, ((t >> 1) & 1) ^ 1, abort_flag))) break;
         fence_after_sync();
-        const uint32_t b_base = smem_u32(sB + s * TILE_BYTES);
+        const uint32_t b_base = smem_u32(smem + OFF_B + s * TILE_BYTES);
+        const uint32_t bx_base = smem_u32(smem + OFF_BX + s * EXT_BYTES);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t koff = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
           mma_bf16(tmem + b * BN, desc_sw128(a_base + koff), desc_sw128(b_base + koff), idesc, kk > 0);
         }
+        mma_bf16(tmem + b * BN, desc_sw32(ax_base), desc_sw32(bx_base), idesc, 1u);
         mma_commit(bar_empty + s);
         mma_commit(bar_accf + b);
         done = t + 1;
@@ -162,118 +259,171 @@ __global__ void __launch_bounds__(THREADS, 2)
       }
     }
   } else {
-    // ---------------- epilogue: one thread per row (TMEM lane)
-    const int q = warp & 3;                       // TMEM lane quarter accessible to this warp
+    // ---------------- epilogue: thread = row (TMEM lane); two warps per row quarter
+    const int ew = warp - 2;                      // 0..7
+    const int half = ew >> 2;                     // columns [64 half, 64 half + 64) of each tile
+    const int q = warp & 3;                       // TMEM lane quarter
     const int r_local = q * 32 + lane;
     const int row = row0 + r_local;
     const bool active = row < nrows;
-    const int et = threadIdx.x - 64;              // 0..127 among the epilogue threads
+    const int et = threadIdx.x - 64;              // 0..255
     const int64_t bh = (int64_t)h * j.b.M_max;
     const KParams kp = j.kp;
-    const float k2 = -2.0f * kp.inv_s2;
-    // per-row state
-    float cr = kp.eps, S = 0.f, acc = 0.f, thr = 0.f;
-    int cross = INT_MAX, self = -1, slot = row;
+    const float hs2 = 0.5f / kp.inv_s2;           // sigma^2 / 2
+    float c = hs2;                                // (sigma^2 / 2)^p
+    if (P >= 2) c = hs2 * hs2;
+    if (P == 4) c = c * c;
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    // per-row state (sums in units of |A|^-p)
+    float S = 0.f, acc = 0.f, thr = 0.f;
+    int cross = INT_MAX, self = -1;
     float* snap_row = nullptr;
     if (active) {
-      cr = fmaf(j.rnorm[(int64_t)h * j.rn_hs + row], kp.inv_s2, kp.eps);
       if (MODE == TM_CROSS) {
-        S = j.b.rho[bh + row];
-        thr = __fmul_rn(kp.tau, j.b.base[bh + row]);
-        if (S >= thr) cross = 0;
+        const float rho = j.b.rho[bh + row];
+        thr = (__fmul_rn(kp.tau, j.b.base[bh + row]) - rho) / c;
+        if (thr <= 0.f) cross = 0;
         snap_row = j.w.snap + (bh + row) * j.w.snap_stride;
-        snap_row[0] = S;
       } else if (MODE == TM_PROJECT) {
         S = j.w.snap[(bh + row) * j.w.snap_stride + c0 / SNAP];
-      } else if (MODE == TM_SUB) {
-        slot = hd.e == 0 ? row : j.w.surv_list[bh + row];
       } else if (MODE == TM_NEWBASE) {
         self = j.w.slot_new[(int64_t)h * j.b.n_max + row];
       }
     }
-    // column metadata source
-    const float* cnorm = nullptr;
-    const float* cbase = nullptr;
-    if (MODE == TM_SCORE || MODE == TM_NEWBASE) cnorm = j.b.knorm + bh;
-    if (MODE == TM_SCORE) cbase = j.b.base + bh;
-    if (MODE == TM_CROSS || MODE == TM_PROJECT) cnorm = j.w.kperm_norm + (int64_t)h * j.b.n_max;
-    if (MODE == TM_SUB) cnorm = j.w.kevict_norm + (int64_t)h * j.b.n_max;
+    if (MODE == TM_CROSS && active && half == 0) snap_row[0] = 0.f;
 
     bool ok = true;
     for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
       const int col0 = c0 + t * BN;
       const int nc = min(BN, c1 - col0);
-      // stage this tile's column terms: cc = |k_j|^2 / sigma^2, and 1 / b_j for SCORE
-      float* mc = meta + b * 2 * BN;
-      {
-        const int c = col0 + et;
-        mc[et] = et < nc ? cnorm[c] * kp.inv_s2 : 0.f;
-        if (MODE == TM_SCORE) mc[BN + et] = et < nc ? 1.0f / cbase[c] : 0.f;
+      if (MODE == TM_SCORE) {   // 1 / b_j of this tile's columns
+        if (et < BN) meta[b * BN + et] = et < nc ? 1.0f / j.b.base[bh + col0 + et] : 0.f;
+        named_bar(5, 32 * EPI_WARPS);
       }
-      // every epilogue warp takes this barrier on every tile, also after a failed wait,
-      // so no warp is ever left waiting here
-      named_bar(1, 128);
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_accf + b, (t >> 1) & 1, abort_flag));
-      if (!ok) continue;
-      fence_after_sync();
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * BN;
-#pragma unroll 1
-      for (int c32 = 0; c32 < BN; c32 += 32) {
-        if (c32 >= nc) break;
-        float v[32];
-        tmem_ld32(tbase + c32, v);
-        tmem_wait_ld();
-        if (!active) continue;
-        const int lim = min(32, nc - c32);
+      float tot[2] = {0.f, 0.f};
+      if (ok) {
+        fence_after_sync();
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-          if (jj < lim) {
-            const float u = fmaxf(fmaf(v[jj], k2, cr + mc[c32 + jj]), kp.eps);
-            const float r = rcp_approx(u);
-            float w = r;
-            if (kp.p >= 2) w = r * r;
-            if (kp.p == 4) w = w * w;
-            const int col = col0 + c32 + jj;
-            if (MODE == TM_SCORE) {
-              acc = fmaf(w, mc[BN + c32 + jj], acc);
-            } else if (MODE == TM_CROSS) {
-              S += w;
-              if (cross == INT_MAX && S >= thr) cross = col + 1;
-            } else if (MODE == TM_PROJECT) {
-              S += w;
-            } else if (MODE == TM_SUB) {
-              acc += w;
+        for (int ch = 0; ch < 2; ++ch) {
+          const int cs = half * 64 + ch * 32;     // first column of the chunk within the tile
+          if (cs >= nc) continue;                 // warp-uniform
+          float v[32];
+          tmem_ld32(lane_base + b * BN + cs, v);
+          tmem_wait_ld();
+          const int lim = min(32, nc - cs);
+          if (MODE == TM_SCORE) {
+            const float* ib = meta + b * BN + cs;
+            if (lim == 32) {
+              float tt[16];
+#pragma unroll
+              for (int k = 0; k < 16; ++k) tt[k] = term2w<P>(v[2 * k], v[2 * k + 1], ib[2 * k], ib[2 * k + 1]);
+              tot[ch] = tree16(tt);
             } else {
-              if (col != self) S += w;
+              float s = 0.f;
+#pragma unroll
+              for (int jj = 0; jj < 32; ++jj)
+                if (jj < lim) s = fmaf(term1<P>(v[jj]), ib[jj], s);
+              tot[ch] = s;
             }
+          } else if (MODE == TM_NEWBASE) {
+            const int sk = self - (col0 + cs);
+            if (lim == 32 && (sk < 0 || sk >= 32)) tot[ch] = chunk_sum<P>(v);
+            else tot[ch] = chunk_sum_skip<P>(v, lim, sk);
+          } else {
+            tot[ch] = lim == 32 ? chunk_sum<P>(v) : chunk_sum_partial<P>(v, lim);
           }
         }
       }
-      if (MODE == TM_CROSS && active && nc == BN) snap_row[(col0 + BN) / SNAP] = S;
-      fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar_acce + b);
+      if (MODE == TM_CROSS || MODE == TM_PROJECT) {
+        // exchange the half totals of this row, so both warps carry the same running sum
+        const float mine = tot[0] + tot[1];
+        xch[(b * 2 + half) * BM + r_local] = mine;
+        named_bar(1 + q, 64);
+        const float other = xch[(b * 2 + (half ^ 1)) * BM + r_local];
+        const float T0 = half == 0 ? mine : other;
+        const float T1 = half == 0 ? other : mine;
+        if (MODE == TM_CROSS && ok) {
+          const float base0 = half == 0 ? S : S + T0;
+          int hit = -1;
+          float run = base0;
+          if (active && cross == INT_MAX) {
+            if (base0 + tot[0] >= thr) hit = 0;
+            else if ((base0 + tot[0]) + tot[1] >= thr) { hit = 1; run = base0 + tot[0]; }
+          }
+          // exact position inside the chunk, term by term (at most once per row); the
+          // TMEM load is warp-collective, so the whole warp takes part for each chunk hit
+#pragma unroll
+          for (int hc = 0; hc < 2; ++hc) {
+            const int cs = half * 64 + hc * 32;
+            if (cs < nc && __any_sync(0xffffffffu, hit == hc)) {
+              float v[32];
+              tmem_ld32(lane_base + b * BN + cs, v);
+              tmem_wait_ld();
+              if (hit == hc) {
+                const int lim = min(32, nc - cs);
+                int pos = lim;
+#pragma unroll
+                for (int jj = 0; jj < 32; ++jj) {
+                  if (jj < lim && pos == lim) {
+                    run += term1<P>(v[jj]);
+                    if (run >= thr) pos = jj + 1;
+                  }
+                }
+                cross = col0 + cs + pos;
+              }
+            }
+          }
+        }
+        S = (S + T0) + T1;
+        if (MODE == TM_CROSS && ok && active && half == 0 && nc == BN) snap_row[(col0 + BN) / SNAP] = S;
+      } else {
+        acc += tot[0] + tot[1];
+      }
+      if (ok) {
+        fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_acce + b);
+      }
     }
     if (!ok) {
       *abort_flag = 1;
-      dev_fail(j.w.L, DEV_TIMEOUT, 300 + MODE);
-    } else if (active) {
+      if (lane == 0) dev_fail(j.w.L, DEV_TIMEOUT, 300 + MODE);
+    }
+    if (MODE == TM_SCORE || MODE == TM_SUB || MODE == TM_NEWBASE) {
+      // combine the two column halves of each row (no per-tile exchange in these passes)
+      xch[half * BM + r_local] = acc;
+      named_bar(1 + q, 64);
+      acc = xch[r_local] + xch[BM + r_local];
+    }
+    if (MODE == TM_CROSS) {
+      // each half saw only its own columns: the row's first crossing is the earlier one.
+      // The exchange slots of parity (ntiles & 1) were last read before the final tile's
+      // barrier, so they are free.
+      int* xi = reinterpret_cast<int*>(xch) + (ntiles & 1) * 2 * BM;
+      xi[half * BM + r_local] = cross;
+      named_bar(1 + q, 64);
+      cross = min(xi[r_local], xi[BM + r_local]);
+    }
+    if (ok && active && half == 0) {
       if (MODE == TM_SCORE) {
-        j.w.score[(int64_t)h * j.b.n_max + row] = acc / (float)hd.m_old;
+        j.w.score[(int64_t)h * j.b.n_max + row] = (acc * c) / (float)hd.m_old;
       } else if (MODE == TM_CROSS) {
         j.w.cross[bh + row] = cross;
         const int bin = cross == INT_MAX ? L.rmax + 1 : cross;
         atomicAdd(&j.w.hist[(int64_t)h * j.w.hist_stride + bin], 1);
       } else if (MODE == TM_PROJECT) {
-        j.w.rho_t[bh + row] = S;
+        j.w.rho_t[bh + row] = fmaf(c, S, j.b.rho[bh + row]);
       } else if (MODE == TM_SUB) {
-        if (slot >= 0 && slot < hd.m_old) j.b.rho[bh + slot] = j.w.rho_t[bh + slot] - acc;
+        const int slot = hd.e == 0 ? row : j.w.surv_list[bh + row];
+        if (slot >= 0 && slot < hd.m_old) j.b.rho[bh + slot] = fmaf(-c, acc, j.w.rho_t[bh + slot]);
         else dev_fail(j.w.L, DEV_INCONSISTENT, 6003);
       } else {
         if (self >= 0 && self < hd.M) {
-          j.b.rho[bh + self] = S;
-          j.b.base[bh + self] = fmaxf(S, kp.delta);
+          const float rho = c * acc;
+          j.b.rho[bh + self] = rho;
+          j.b.base[bh + self] = fmaxf(rho, kp.delta);
         } else {
           dev_fail(j.w.L, DEV_INCONSISTENT, 6004);
         }
@@ -307,34 +457,53 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-}  // namespace
-
-// bf16 [heads][rows][128] tensor, boxes of 64 columns x box_rows rows, 128-byte swizzle.
-bool make_map_rows(CUtensorMap* m, const void* base, int64_t rows, int64_t heads, int box_rows) {
+bool encode(CUtensorMap* m, const void* base, uint64_t inner, int64_t rows, int64_t heads, uint32_t box_inner,
+            uint32_t box_rows, CUtensorMapSwizzle sw) {
   EncodeTiledFn fn = encode_fn();
   if (!fn || rows < 1 || heads < 1) return false;
-  cuuint64_t dims[3] = {128, (cuuint64_t)rows, (cuuint64_t)heads};
-  cuuint64_t strides[2] = {256, (cuuint64_t)rows * 256};
-  cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  cuuint64_t dims[3] = {inner, (cuuint64_t)rows, (cuuint64_t)heads};
+  cuuint64_t strides[2] = {inner * 2, (cuuint64_t)rows * inner * 2};
+  cuuint32_t box[3] = {box_inner, box_rows, 1};
   cuuint32_t es[3] = {1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+// bf16 [heads][rows][128] keys: boxes of 64 columns x box_rows rows, 128-byte swizzle.
+bool make_map_rows(CUtensorMap* m, const void* base, int64_t rows, int64_t heads, int box_rows) {
+  return encode(m, base, 128, rows, heads, 64, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+// bf16 [heads][rows][32] extension rows: boxes of 16 columns x box_rows rows, 32-byte swizzle.
+bool make_map_ext(CUtensorMap* m, const void* base, int64_t rows, int64_t heads, int box_rows) {
+  return encode(m, base, 32, rows, heads, 16, box_rows, CU_TENSOR_MAP_SWIZZLE_32B);
 }
 
 namespace {
 
+template <int MODE, int P>
+void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap& ax, const CUtensorMap& b,
+              const CUtensorMap& bx, const TcJob& job) {
+  tc_pairs<MODE, P><<<grid, THREADS, SMEM_BYTES, s>>>(a, ax, b, bx, job);
+}
+
 template <int MODE>
-cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void* rk, int64_t rk_rows,
-                      const float* rnorm, int64_t rn_hs, const void* ck, int64_t ck_rows, int max_rows,
-                      cudaStream_t s, Timer* t, const char* name) {
-  CUtensorMap ma, mb;
-  if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_rows(&mb, ck, ck_rows, b.H, BN))
+cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void* rk, const void* rx, int64_t rk_rows,
+                      const void* ck, const void* cx, int64_t ck_rows, int max_rows, cudaStream_t s, Timer* t,
+                      const char* name) {
+  CUtensorMap ma, max_, mb, mbx;
+  if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_ext(&max_, rx, rk_rows, b.H, BM) ||
+      !make_map_rows(&mb, ck, ck_rows, b.H, BN) || !make_map_ext(&mbx, cx, ck_rows, b.H, BN))
     return cudaErrorInvalidValue;
-  TcJob job{b, w, kp, rnorm, rn_hs};
+  TcJob job{b, w, kp};
   dim3 grid((max_rows + BM - 1) / BM, b.H);
   timer_begin(t, name, s);
-  tc_pairs<MODE><<<grid, THREADS, SMEM_BYTES, s>>>(ma, mb, job);
+  if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, job);
+  else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, job);
+  else launch_p<MODE, 2>(grid, s, ma, max_, mb, mbx, job);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -347,13 +516,18 @@ cudaError_t tc_attn_set_smem_limits();
 
 cudaError_t tc_set_smem_limits() {
   cudaError_t e = cudaSuccess;
-#define DKV_OPT(K) \
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(K, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES)
-  DKV_OPT(tc_pairs<TM_SCORE>);
-  DKV_OPT(tc_pairs<TM_CROSS>);
-  DKV_OPT(tc_pairs<TM_PROJECT>);
-  DKV_OPT(tc_pairs<TM_SUB>);
-  DKV_OPT(tc_pairs<TM_NEWBASE>);
+#define DKV_OPT(M)                                                                                             \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_pairs<M, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);    \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_pairs<M, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);    \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_pairs<M, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  DKV_OPT(TM_SCORE)
+  DKV_OPT(TM_CROSS)
+  DKV_OPT(TM_PROJECT)
+  DKV_OPT(TM_SUB)
+  DKV_OPT(TM_NEWBASE)
 #undef DKV_OPT
   if (e == cudaSuccess) e = tc_attn_set_smem_limits();
   return e;
@@ -361,26 +535,26 @@ cudaError_t tc_set_smem_limits() {
 
 cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
                             Timer* t) {
-  return launch_tc<TM_SCORE>(b, w, kp, Kc, N, w.cnorm, b.n_max, b.k, b.M_max, N, s, t, "score_tc");
+  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc");
 }
 
 cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  return launch_tc<TM_CROSS>(b, w, kp, b.k, b.M_max, b.knorm, b.M_max, w.kperm, b.n_max, b.M_max, s, t,
+  return launch_tc<TM_CROSS>(b, w, kp, b.k, w.bext, b.M_max, w.kperm, w.kperm_ext, b.n_max, b.M_max, s, t,
                              "cross_tc");
 }
 
 cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  return launch_tc<TM_PROJECT>(b, w, kp, b.k, b.M_max, b.knorm, b.M_max, w.kperm, b.n_max, b.M_max, s, t,
+  return launch_tc<TM_PROJECT>(b, w, kp, b.k, w.bext, b.M_max, w.kperm, w.kperm_ext, b.n_max, b.M_max, s, t,
                                "project_tc");
 }
 
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  return launch_tc<TM_SUB>(b, w, kp, w.ksurv, b.M_max, w.ksurv_norm, b.M_max, w.kevict, b.n_max, b.M_max, s, t,
-                           "subtract_tc");
+  return launch_tc<TM_SUB>(b, w, kp, w.ksurv, w.ksurv_ext, b.M_max, w.kevict, w.kevict_ext, b.n_max, b.M_max, s,
+                           t, "subtract_tc");
 }
 
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  return launch_tc<TM_NEWBASE>(b, w, kp, w.kperm, b.n_max, w.kperm_norm, b.n_max, b.k, b.M_max, b.n_max, s, t,
+  return launch_tc<TM_NEWBASE>(b, w, kp, w.kperm, w.kperm_ext, b.n_max, b.k, w.bext, b.M_max, b.n_max, s, t,
                                "newbase_tc");
 }
 

@@ -57,9 +57,21 @@ __global__ void k_prepare(Bank b, Ws w, int N, int64_t step) {
   }
 }
 
+// bf16 split x = hi + mid + lo (each rounded to nearest), ~24 significant bits.
+__device__ __forceinline__ void split3(float x, __nv_bfloat16& hi, __nv_bfloat16& mid, __nv_bfloat16& lo) {
+  hi = __float2bfloat16_rn(x);
+  const float r1 = x - __bfloat162float(hi);
+  mid = __float2bfloat16_rn(r1);
+  lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+}
+
+// ||k||^2 per row and, if ext != nullptr, the row's 32 extension values used by the
+// tensor-core passes: row form [-g_hi, -g_mid, -g_lo, 1, 1, 1, 0 x 10] and column form
+// [1, 1, 1, -h_hi, -h_mid, -h_lo, 0 x 10], g = |k|^2 / 2 + goff, h = |k|^2 / 2.
 template <typename T>
 __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
-                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d) {
+                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d,
+                            __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
   const int h = blockIdx.y;
   const int row = blockIdx.x * (blockDim.x / 32) + warp_id();
   const int n = count_is_occ ? count[h] : N;
@@ -73,6 +85,19 @@ __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int ro
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
   if (lane_id() == 0) out[(int64_t)h * out_hs + row] = a;
+  if (ext) {
+    __nv_bfloat16 g[3], hh[3];
+    split3(-(0.5f * a + goff), g[0], g[1], g[2]);
+    split3(-(0.5f * a), hh[0], hh[1], hh[2]);
+    const int l = lane_id();
+    const __nv_bfloat16 one = __float2bfloat16_rn(1.0f), zero = __float2bfloat16_rn(0.0f);
+    __nv_bfloat16 v = zero;
+    if (l < 3) v = g[l];
+    else if (l < 6) v = one;
+    else if (l >= 16 && l < 19) v = one;
+    else if (l >= 19 && l < 22) v = hh[l - 19];
+    ext[(int64_t)h * ext_hs + (int64_t)row * 32 + l] = v;
+  }
 }
 
 // Bitonic sort of (fkey(score) << 32 | source index) per head: ascending score,
@@ -115,6 +140,8 @@ __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int 
   const int rb = b.d * esize;
   const int src = w.perm[(int64_t)h * b.n_max + j];
   warp_copy_row((char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, Kc + ((int64_t)h * N + src) * rb, rb);
+  warp_copy_row((char*)w.kperm_ext + ((int64_t)h * b.n_max + j) * 64, (const char*)w.cext + ((int64_t)h * b.n_max + src) * 64,
+                64);
   if (lane_id() == 0) w.kperm_norm[(int64_t)h * b.n_max + j] = w.cnorm[(int64_t)h * b.n_max + src];
 }
 
@@ -373,6 +400,7 @@ __global__ void k_gather(Bank b, Ws w, int esize) {
       return;
     }
     warp_copy_row((char*)w.ksurv + (bh + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
+    warp_copy_row((char*)w.ksurv_ext + (bh + row) * 64, (const char*)w.bext + (bh + slot) * 64, 64);
     if (lane_id() == 0) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
   }
   if (row < hd.e) {
@@ -382,6 +410,7 @@ __global__ void k_gather(Bank b, Ws w, int esize) {
       return;
     }
     warp_copy_row((char*)w.kevict + ((int64_t)h * b.n_max + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
+    warp_copy_row((char*)w.kevict_ext + ((int64_t)h * b.n_max + row) * 64, (const char*)w.bext + (bh + slot) * 64, 64);
     if (lane_id() == 0) w.kevict_norm[(int64_t)h * b.n_max + row] = b.knorm[bh + slot];
   }
 }
@@ -409,6 +438,7 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
   const int src = w.perm[(int64_t)h * b.n_max + j];
   warp_copy_row((char*)b.k + (bh + slot) * rb, (const char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, rb);
   warp_copy_row((char*)b.v + (bh + slot) * rb, Vc + ((int64_t)h * N + src) * rb, rb);
+  warp_copy_row((char*)w.bext + (bh + slot) * 64, (const char*)w.kperm_ext + ((int64_t)h * b.n_max + j) * 64, 64);
   if (lane_id() == 0) {
     b.knorm[bh + slot] = w.kperm_norm[(int64_t)h * b.n_max + j];
     b.prov_step[bh + slot] = w.L->step;
@@ -426,28 +456,34 @@ cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cuda
   return cudaGetLastError();
 }
 
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
+static float ext_goff(const KParams& kp) { return kp.eps * 0.5f / kp.inv_s2; }   // eps sigma^2 / 2
+
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
+                              Timer* t) {
   dim3 grid((N + 7) / 8, b.H);
+  __nv_bfloat16* ext = (__nv_bfloat16*)w.cext;
   timer_begin(t, "cand_norms", s);
   if (b.bf16)
     k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)Kc, (int64_t)N * b.d, N, nullptr, 0, N,
-                                                    w.cnorm, b.n_max, b.d);
+                                                    w.cnorm, b.n_max, b.d, ext, (int64_t)b.n_max * 32, ext_goff(kp));
   else
     k_row_norms<float><<<grid, 256, 0, s>>>((const float*)Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm,
-                                            b.n_max, b.d);
+                                            b.n_max, b.d, ext, (int64_t)b.n_max * 32, ext_goff(kp));
   timer_end(t, s);
   return cudaGetLastError();
 }
 
-cudaError_t launch_bank_norms(const Bank& b, cudaStream_t s, Timer* t) {
+cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   dim3 grid((b.M_max + 7) / 8, b.H);
+  __nv_bfloat16* ext = (__nv_bfloat16*)w.bext;
   timer_begin(t, "bank_norms", s);
   if (b.bf16)
     k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)b.k, (int64_t)b.M_max * b.d, b.M_max,
-                                                    b.occ, 1, 0, b.knorm, b.M_max, b.d);
+                                                    b.occ, 1, 0, b.knorm, b.M_max, b.d, ext,
+                                                    (int64_t)b.M_max * 32, ext_goff(kp));
   else
     k_row_norms<float><<<grid, 256, 0, s>>>((const float*)b.k, (int64_t)b.M_max * b.d, b.M_max, b.occ, 1, 0,
-                                            b.knorm, b.M_max, b.d);
+                                            b.knorm, b.M_max, b.d, ext, (int64_t)b.M_max * 32, ext_goff(kp));
   timer_end(t, s);
   return cudaGetLastError();
 }

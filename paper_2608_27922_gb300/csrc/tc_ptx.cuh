@@ -147,6 +147,16 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t addr) {
          | ((uint64_t)2u << 61);               // layout: 128-byte swizzle
 }
 
+// Shared-memory matrix descriptor, 32-byte swizzle, K-major: rows of 32 bytes (16 bf16,
+// one MMA k-step), 8-row groups 256 bytes apart, base 256-byte aligned.
+__device__ __forceinline__ uint64_t desc_sw32(uint32_t addr) {
+  return (uint64_t)((addr >> 4) & 0x3FFFu)     // start address
+         | ((uint64_t)1u << 16)                // leading byte offset (unused for swizzled K-major)
+         | ((uint64_t)(256u >> 4) << 32)       // stride byte offset: 8 rows x 32 B
+         | ((uint64_t)1u << 46)                // descriptor version (tcgen05)
+         | ((uint64_t)6u << 61);               // layout: 32-byte swizzle
+}
+
 // MN-major 128-byte-swizzle descriptor (operand stored with the N/M index contiguous):
 // `lbo` = bytes between successive 64-element groups along M/N, `sbo` = bytes between
 // successive 8-row (K) groups.
