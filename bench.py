@@ -61,6 +61,8 @@ def parse_args():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between steps")
     ap.add_argument("--heads", type=int, default=0, help="override the head count (profiling runs)")
+    ap.add_argument("--no-overlap", action="store_true",
+                    help="run attention and the update on one stream instead of overlapping them")
     return ap.parse_args()
 
 
@@ -213,12 +215,29 @@ def run_ours(args):
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
+    side = torch.cuda.Stream(dev)
+
     def step(t, Q, KW, VW, KC, VC):
-        bank.attend(Q, KW, VW, out=out)
         b = wl.admitted_block(t)
+        if args.no_overlap:
+            bank.attend(Q, KW, VW, out=out)
+            if b is not None:
+                bank.admit(KC, VC, b)
+                bank.compress()
+            return
+        # attention and admit both only read the bank (the update is atomic from the
+        # reader's side), so they run concurrently; compress waits for attention
+        go = torch.cuda.Event()
+        go.record(stream)
+        side.wait_event(go)
+        bank.attend(Q, KW, VW, out=out, stream=side)
+        done = torch.cuda.Event()
+        done.record(side)
         if b is not None:
-            bank.admit(KC, VC, b)
-            bank.compress()
+            bank.admit(KC, VC, b, stream=stream)
+        stream.wait_event(done)
+        if b is not None:
+            bank.compress(stream=stream)
 
     def device_step(t):
         kw, vw = dblocks[wl.window_block(t)]
@@ -362,6 +381,7 @@ def run_ours(args):
             "config": {"workload": f"{wl.name}: {wl.L if world > 1 else 1} layer(s) x {wl.H} heads, d={wl.d}, "
                                    f"N={wl.N}, M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
                        "score_mode": args.score_mode, "layers_per_gpu": 1,
+                       "streams": "attention || admit, then compress" if not args.no_overlap else "one stream",
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                        "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
             "blocks_per_s": world * K / (total_ms_max / 1e3),

@@ -116,6 +116,12 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* ba
   w.bext = take(Hh * Mm * 64);
   w.ksurv_ext = take(Hh * Mm * 64);
   w.kevict_ext = take(Hh * Nm * 64);
+  const int part_stride = (M_max > n_max ? M_max : n_max);
+  const int cnt_stride = (part_stride + 127) / 128;
+  w.part = (float*)take(2 * Hh * part_stride * 4);
+  w.cnt = (int32_t*)take(Hh * cnt_stride * 4);
+  w.part_stride = part_stride;
+  w.cnt_stride = cnt_stride;
   w.hist_stride = hist_stride;
   w.snap_stride = snap_stride;
   w.feas_words = feas_words;
@@ -263,6 +269,7 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   // workspace header: zeroed layer state and the per-head budgets (one-time, synchronous)
   cudaError_t e = cudaMemset(bk->w.L, 0, sizeof(DevLayer));
   if (e == cudaSuccess) e = cudaMemset(bk->w.hd, 0, sizeof(DevHead) * H);
+  if (e == cudaSuccess) e = cudaMemset(bk->w.cnt, 0, sizeof(int32_t) * H * bk->w.cnt_stride);
   if (e == cudaSuccess) e = cudaMemcpy(bk->w.budgets, budgets, sizeof(int32_t) * H, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     delete bk;

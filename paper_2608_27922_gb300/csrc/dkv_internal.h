@@ -51,7 +51,9 @@ struct Ws {
   void* bext;           // [H][M_max][32] bank (derived from the bank keys, kept in step)
   void* ksurv_ext;      // [H][M_max][32]
   void* kevict_ext;     // [H][n_max][32]
-  int hist_stride, snap_stride, feas_words;
+  float* part;          // [2][H][part_stride] per-row partial sums of column-split passes
+  int32_t* cnt;         // [H][cnt_stride] arrival counters of column-split row tiles (kept 0)
+  int hist_stride, snap_stride, feas_words, part_stride, cnt_stride;
 };
 
 // Computes the sub-buffer offsets of the workspace; returns the total bytes.

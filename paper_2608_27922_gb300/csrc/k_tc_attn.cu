@@ -2,16 +2,19 @@
 //   O = softmax(Q [K_bank ; K_win]^T / sqrt(d)) [V_bank ; V_win]        (Sec. 3.2, Fig. 2)
 // over the m_h retained bank states followed by the W window states, no mask.
 //
-// One CTA owns 128 queries of one head and streams 128-key tiles (bank tiles first,
-// then window tiles).  Per tile:
-//   S = Q K^T           tcgen05.mma into one of two 128-column TMEM buffers
-//   P = exp2(S log2(e)/sqrt(d) - m)   softmax warps (thread = query row), bf16 into smem
-//   O += P V            tcgen05.mma, V read as an MN-major operand, O in TMEM
-// The running maximum m is raised only when a tile's maximum exceeds it by more than
-// 8 (log2 units); O and the running sum are then rescaled in TMEM.  Exponentials stay
-// below 2^8, and the final O / l is exact softmax algebra (the common factor cancels).
-//
-// Warps: 0 TMA producer, 1 MMA issuer, 2-5 softmax + output.  TMEM: S0, S1, O.
+// One CTA owns 128 queries of one head.  The key range (bank tiles, then window
+// tiles, 128 keys each) is split in two halves, processed concurrently by two
+// softmax warpgroups that share the query tile and one MMA-issuing thread:
+//   S_g = Q K^T            tcgen05.mma into TMEM (128 columns per group)
+//   P_g = exp2(S_g log2(e)/sqrt(d) - m_g)   softmax threads (thread = query row);
+//                          P is written back over S_g in TMEM as packed bf16
+//   O_g += P_g V           tcgen05.mma with A = P_g read from TMEM, V MN-major in smem
+// The running maximum m_g is raised only when a tile's maximum exceeds it by more
+// than 8 (log2 units); O_g and the running sum are then rescaled in TMEM.  At the
+// end the two partial results are merged exactly:
+//   O = (2^(m_0 - m) O_0 + 2^(m_1 - m) O_1) / (2^(m_0 - m) l_0 + 2^(m_1 - m) l_1).
+// Warps: 0 TMA producer, 1 MMA issuer, 2-5 softmax group 0, 6-9 softmax group 1.
+// TMEM columns: S_0 [0,128), O_0 [128,256), S_1 [256,384), O_1 [384,512).
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
@@ -29,11 +32,14 @@ constexpr int BQ = 128;                 // queries per CTA
 constexpr int BK = 128;                 // keys per tile
 constexpr int TB = 128 * 128 * 2;       // bytes of a 128 x 128 bf16 tile
 constexpr int HB = TB / 2;              // one 64-column swizzle panel
-constexpr int THREADS = 192;
-constexpr uint32_t TMEM_COLS = 512;     // S0 [0,128), S1 [128,256), O [256,384)
-constexpr uint32_t O_COL = 256;
-// Q, K[2], V[2], P[2] tiles + barriers
-constexpr size_t SMEM_BYTES = 1024 + TB * 7 + 256;
+constexpr int THREADS = 64 + 256;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int OFF_Q = 0;
+constexpr int OFF_K = TB;               // [2 groups]
+constexpr int OFF_V = 3 * TB;           // [2 groups]
+constexpr int OFF_X = 5 * TB;           // float [2 groups][2 (m, l)][BQ]
+constexpr int OFF_BAR = OFF_X + 2 * 2 * BQ * 4;
+constexpr size_t SMEM_BYTES = 1024 + OFF_BAR + 256;
 constexpr float RESCALE_LOG2 = 8.0f;
 
 __device__ __forceinline__ float ex2(float x) {
@@ -53,7 +59,7 @@ struct AttnJob {
   int Nq;
   int W;
   __nv_bfloat16* O;
-  float sl2;   // log2(e) / sqrt(d)
+  float sl2;     // log2(e) / sqrt(d)
 };
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -62,22 +68,17 @@ __global__ void __launch_bounds__(THREADS, 1)
               const __grid_constant__ CUtensorMap tmVw, AttnJob j) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;
-  uint8_t* sK = smem + TB;        // [2]
-  uint8_t* sV = smem + 3 * TB;    // [2]
-  uint8_t* sP = smem + 5 * TB;    // [2]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * TB);
+  float* xst = reinterpret_cast<float*>(smem + OFF_X);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;    // [2]
+  uint64_t* k_full = bars + 1;    // [2 groups]
   uint64_t* k_empty = bars + 3;   // [2]
   uint64_t* v_full = bars + 5;    // [2]
   uint64_t* v_empty = bars + 7;   // [2]
   uint64_t* s_full = bars + 9;    // [2]
-  uint64_t* s_free = bars + 11;   // [2]
-  uint64_t* p_full = bars + 13;   // [2]
-  uint64_t* p_free = bars + 15;   // [2]
-  uint64_t* pv_done = bars + 17;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* p_full = bars + 11;   // [2]
+  uint64_t* pv_done = bars + 13;  // [2]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 15);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int h = blockIdx.y;
@@ -86,17 +87,17 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int W = j.W;
   const int nb = (m + BK - 1) / BK;            // bank tiles
   const int nt = nb + (W + BK - 1) / BK;       // all key tiles
+  const int nh = (nt + 1) / 2;                 // tiles of group 0; group 1 takes the rest
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(k_full + i, 1); mbar_init(k_empty + i, 1);
-      mbar_init(v_full + i, 1); mbar_init(v_empty + i, 1);
-      mbar_init(s_full + i, 1); mbar_init(s_free + i, 4);
-      mbar_init(p_full + i, 4); mbar_init(p_free + i, 1);
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(k_full + g, 1); mbar_init(k_empty + g, 1);
+      mbar_init(v_full + g, 1); mbar_init(v_empty + g, 1);
+      mbar_init(s_full + g, 1); mbar_init(p_full + g, 4);
+      mbar_init(pv_done + g, 1);
     }
-    mbar_init(pv_done, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -106,32 +107,38 @@ __global__ void __launch_bounds__(THREADS, 1)
   fence_after_sync();
   const uint32_t tmem = *tmem_holder;
 
+  auto tiles_of = [&](int g) { return g == 0 ? nh : nt - nh; };
+  auto tile_index = [&](int g, int i) { return g * nh + i; };
+
   if (warp == 0) {
     if (lane == 0 && nt > 0) {
-      // ---------------- TMA producer
+      // ---------------- TMA producer: Q once; per group single-buffered K and V
       prefetch_map(&tmQ);
       mbar_arrive_expect_tx(q_full, TB);
-      tma_load_3d(sQ, &tmQ, q_full, 0, q0, h);
-      tma_load_3d(sQ + HB, &tmQ, q_full, 64, q0, h);
-      int kiss = 0, viss = 0;
+      tma_load_3d(smem + OFF_Q, &tmQ, q_full, 0, q0, h);
+      tma_load_3d(smem + OFF_Q + HB, &tmQ, q_full, 64, q0, h);
+      int kiss[2] = {0, 0}, viss[2] = {0, 0};
       bool ok = true;
-      for (int t = 0; t < nt && ok; ++t) {
-        const int s = t & 1;
-        const uint32_t ph = ((t >> 1) & 1) ^ 1;
-        const bool bank = t < nb;
-        const CUtensorMap* mk = bank ? &tmKb : &tmKw;
-        const CUtensorMap* mv = bank ? &tmVb : &tmVw;
-        const int row = bank ? t * BK : (t - nb) * BK;
-        if (!(ok = mbar_wait(k_empty + s, ph, abort_flag))) break;
-        mbar_arrive_expect_tx(k_full + s, TB);
-        tma_load_3d(sK + s * TB, mk, k_full + s, 0, row, h);
-        tma_load_3d(sK + s * TB + HB, mk, k_full + s, 64, row, h);
-        kiss = t + 1;
-        if (!(ok = mbar_wait(v_empty + s, ph, abort_flag))) break;
-        mbar_arrive_expect_tx(v_full + s, TB);
-        tma_load_3d(sV + s * TB, mv, v_full + s, 0, row, h);
-        tma_load_3d(sV + s * TB + HB, mv, v_full + s, 64, row, h);
-        viss = t + 1;
+      const int n0 = tiles_of(0), n1 = tiles_of(1);
+      for (int i = 0; ok && i < n0; ++i) {
+        for (int g = 0; g < 2 && ok; ++g) {
+          if (i >= (g == 0 ? n0 : n1)) continue;
+          const int u = tile_index(g, i);
+          const bool bank = u < nb;
+          const CUtensorMap* mk = bank ? &tmKb : &tmKw;
+          const CUtensorMap* mv = bank ? &tmVb : &tmVw;
+          const int row = bank ? u * BK : (u - nb) * BK;
+          if (!(ok = mbar_wait(k_empty + g, (i & 1) ^ 1, abort_flag))) break;
+          mbar_arrive_expect_tx(k_full + g, TB);
+          tma_load_3d(smem + OFF_K + g * TB, mk, k_full + g, 0, row, h);
+          tma_load_3d(smem + OFF_K + g * TB + HB, mk, k_full + g, 64, row, h);
+          kiss[g] = i + 1;
+          if (!(ok = mbar_wait(v_empty + g, (i & 1) ^ 1, abort_flag))) break;
+          mbar_arrive_expect_tx(v_full + g, TB);
+          tma_load_3d(smem + OFF_V + g * TB, mv, v_full + g, 0, row, h);
+          tma_load_3d(smem + OFF_V + g * TB + HB, mv, v_full + g, 64, row, h);
+          viss[g] = i + 1;
+        }
       }
       if (!ok) {
         *abort_flag = 1;
@@ -139,176 +146,226 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       volatile int no_abort = 0;
       mbar_wait(q_full, 0, &no_abort);
-      for (int t = kiss > 2 ? kiss - 2 : 0; t < kiss; ++t) mbar_wait(k_full + (t & 1), (t >> 1) & 1, &no_abort);
-      for (int t = viss > 2 ? viss - 2 : 0; t < viss; ++t) mbar_wait(v_full + (t & 1), (t >> 1) & 1, &no_abort);
+      for (int g = 0; g < 2; ++g) {
+        if (kiss[g] > 0) mbar_wait(k_full + g, (kiss[g] - 1) & 1, &no_abort);
+        if (viss[g] > 0) mbar_wait(v_full + g, (viss[g] - 1) & 1, &no_abort);
+      }
     }
   } else if (warp == 1) {
     if (lane == 0 && nt > 0) {
-      // ---------------- MMA issuer: S_t, then PV_{t-1}
+      // ---------------- MMA issuer.  Per group: S(0), then for each tile i:
+      // PV(i) once P(i) is in TMEM, then S(i+1) (which overwrites P(i) after PV(i) read it).
       constexpr uint32_t id_s = idesc_bf16(BQ, BK);
       constexpr uint32_t id_o = idesc_bf16(BQ, 128, /*b_mn_major=*/true);
+      const uint32_t q_base = smem_u32(smem + OFF_Q);
+      const int n[2] = {tiles_of(0), tiles_of(1)};
       bool ok = mbar_wait(q_full, 0, abort_flag);
-      const uint32_t q_base = smem_u32(sQ);
-      int pv_issued = 0;
-      for (int t = 0; ok && t <= nt; ++t) {
-        if (t < nt) {
-          const int s = t & 1;
-          if (!(ok = mbar_wait(k_full + s, (t >> 1) & 1, abort_flag))) break;
-          if (!(ok = mbar_wait(s_free + s, ((t >> 1) & 1) ^ 1, abort_flag))) break;
-          fence_after_sync();
-          const uint32_t k_base = smem_u32(sK + s * TB);
+      int pv_issued[2] = {0, 0};
+      auto issue_s = [&](int g, int i) -> bool {
+        if (!mbar_wait(k_full + g, i & 1, abort_flag)) return false;
+        fence_after_sync();
+        const uint32_t k_base = smem_u32(smem + OFF_K + g * TB);
+        const uint32_t sc = tmem + g * 256;
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
-            mma_bf16(tmem + s * BK, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
-          }
-          mma_commit(k_empty + s);
-          mma_commit(s_full + s);
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
+          mma_bf16(sc, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
         }
-        if (t >= 1) {
-          const int u = t - 1, s = u & 1;
-          if (!(ok = mbar_wait(p_full + s, (u >> 1) & 1, abort_flag))) break;
-          if (!(ok = mbar_wait(v_full + s, (u >> 1) & 1, abort_flag))) break;
-          fence_after_sync();
-          const uint32_t p_base = smem_u32(sP + s * TB);
-          const uint32_t v_base = smem_u32(sV + s * TB);
+        mma_commit(k_empty + g);
+        mma_commit(s_full + g);
+        return true;
+      };
+      auto issue_pv = [&](int g, int i) -> bool {
+        if (!mbar_wait(p_full + g, i & 1, abort_flag)) return false;
+        if (!mbar_wait(v_full + g, i & 1, abort_flag)) return false;
+        fence_after_sync();
+        const uint32_t v_base = smem_u32(smem + OFF_V + g * TB);
+        const uint32_t pc = tmem + g * 256;          // P: packed bf16 pairs over S columns [0, 64)
+        const uint32_t oc = tmem + g * 256 + 128;
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t aoff = (kk >> 2) * HB + (kk & 3) * 32;
-            mma_bf16(tmem + O_COL, desc_sw128(p_base + aoff), desc_sw128_mn(v_base + kk * 2048, HB, 1024), id_o,
-                     (u > 0 || kk > 0) ? 1u : 0u);
-          }
-          mma_commit(v_empty + s);
-          mma_commit(p_free + s);
-          mma_commit(pv_done);
-          pv_issued = u + 1;
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ts(oc, pc + kk * 8, desc_sw128_mn(v_base + kk * 2048, HB, 1024), id_o, (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(v_empty + g);
+        mma_commit(pv_done + g);
+        pv_issued[g] = i + 1;
+        return true;
+      };
+      for (int g = 0; g < 2 && ok; ++g)
+        if (n[g] > 0) ok = issue_s(g, 0);
+      for (int i = 0; ok && i < n[0]; ++i) {
+        for (int g = 0; g < 2 && ok; ++g) {
+          if (i >= n[g]) continue;
+          ok = issue_pv(g, i);
+          if (ok && i + 1 < n[g]) ok = issue_s(g, i + 1);
         }
       }
       if (!ok) {
         *abort_flag = 1;
         dev_fail(j.L, DEV_TIMEOUT, 401);
       }
-      if (pv_issued > 0) {
-        volatile int no_abort = 0;
-        mbar_wait(pv_done, (pv_issued - 1) & 1, &no_abort);
-      }
+      volatile int no_abort = 0;
+      for (int g = 0; g < 2; ++g)
+        if (pv_issued[g] > 0) mbar_wait(pv_done + g, (pv_issued[g] - 1) & 1, &no_abort);
     }
   } else {
-    // ---------------- softmax and output: thread = query row = TMEM lane
+    // ---------------- softmax group g, thread = query row = TMEM lane
+    const int g = (warp - 2) >> 2;
     const int qd = warp & 3;
     const int r = qd * 32 + lane;
     const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
+    const uint32_t sc = tmem + lane_off + g * 256;     // S_g (and P_g)
+    const uint32_t oc = sc + 128;                      // O_g
+    const int ng = tiles_of(g);
     float mrun = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int t = 0; t < nt; ++t) {
-      const int s = t & 1;
-      const bool bank = t < nb;
-      const int valid = bank ? min(BK, m - t * BK) : min(BK, W - (t - nb) * BK);
-      ok = ok && __all_sync(0xffffffffu, mbar_wait(s_full + s, (t >> 1) & 1, abort_flag));
+    for (int i = 0; i < ng; ++i) {
+      const int u = tile_index(g, i);
+      const bool bank = u < nb;
+      const int valid = bank ? min(BK, m - u * BK) : min(BK, W - (u - nb) * BK);
+      ok = ok && __all_sync(0xffffffffu, mbar_wait(s_full + g, i & 1, abort_flag));
       if (!ok) break;
       fence_after_sync();
-      float sv[128];
+      // pass 1: row maximum of the raw scores (masking only on a partial last tile)
+      float tmax;
+      {
+        float t[8];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        float v[32];
-        tmem_ld32(tmem + lane_off + s * BK + c * 32, v);
+        for (int k = 0; k < 8; ++k) t[k] = -INFINITY;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) sv[c * 32 + i] = v[i];
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(sc + c * 32, v);
+          tmem_wait_ld();
+          if (valid == BK) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) t[k & 7] = fmaxf(t[k & 7], v[k]);
+          } else {
+#pragma unroll
+            for (int k = 0; k < 32; ++k)
+              if (c * 32 + k < valid) t[k & 7] = fmaxf(t[k & 7], v[k]);
+          }
+        }
+        tmax = fmaxf(fmaxf(fmaxf(t[0], t[1]), fmaxf(t[2], t[3])), fmaxf(fmaxf(t[4], t[5]), fmaxf(t[6], t[7])));
       }
-      tmem_wait_ld();
-      fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free + s);
-      float tmax = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 128; ++i) {
-        sv[i] = i < valid ? sv[i] * j.sl2 : -INFINITY;
-        tmax = fmaxf(tmax, sv[i]);
-      }
-      // lazily raised running maximum; O and l are rescaled only when it moves by > 8
+      tmax *= j.sl2;
+      // lazily raised running maximum.  S_g(i) complete implies PV_g(i-1) complete
+      // (one thread issues both, in order), so O_g is idle here.
       const bool raise = tmax > mrun + RESCALE_LOG2;
       const float mnew = raise ? tmax : mrun;
-      if (__any_sync(0xffffffffu, raise && t > 0)) {
-        // O holds sum_{u < t} P_u V_u: wait for PV_{t-1}, then scale it in TMEM
-        ok = ok && __all_sync(0xffffffffu, mbar_wait(pv_done, (t - 1) & 1, abort_flag));
-        if (!ok) break;
-        fence_after_sync();
+      if (__any_sync(0xffffffffu, raise && i > 0)) {
         const float alpha = raise ? ex2(mrun - mnew) : 1.0f;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           float v[32];
-          tmem_ld32(tmem + lane_off + O_COL + c * 32, v);
+          tmem_ld32(oc + c * 32, v);
           tmem_wait_ld();
           uint32_t w32[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) w32[i] = __float_as_uint(v[i] * alpha);
-          tmem_st32(tmem + lane_off + O_COL + c * 32, w32);
+          for (int k = 0; k < 32; ++k) w32[k] = __float_as_uint(v[k] * alpha);
+          tmem_st32(oc + c * 32, w32);
         }
-        tmem_wait_st();
       }
       if (raise) {
-        l *= (t > 0) ? ex2(mrun - mnew) : 0.f;
+        l *= (i > 0) ? ex2(mrun - mnew) : 0.f;
         mrun = mnew;
       }
-      // P_t into the shared-memory buffer s once PV_{t-2} has released it
-      ok = ok && __all_sync(0xffffffffu, mbar_wait(p_free + s, ((t >> 1) & 1) ^ 1, abort_flag));
-      if (!ok) break;
-      uint8_t* pb = sP + s * TB;
+      // P_g = 2^(s log2(e)/sqrt(d) - m) as packed bf16 pairs over the first 64 columns of S_g
+      const float nm = -mrun;
+      float la = 0.f, lb = 0.f;
+      // pass 2: exponentials, 64 scores at a time
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {          // 16 chunks of 8 keys (16 bytes)
-        float p[8];
+      for (int c = 0; c < 2; ++c) {
+        float sv[64];
+        {
+          float v[32];
+          tmem_ld32(sc + c * 64, v);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          p[i] = ex2(sv[c * 8 + i] - mrun);
-          l += p[i];
+          for (int k = 0; k < 32; ++k) sv[k] = v[k];
+          tmem_ld32(sc + c * 64 + 32, v);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) sv[32 + k] = v[k];
+          tmem_wait_ld();
         }
-        uint4 pk;
-        pk.x = pack_bf16(p[0], p[1]);
-        pk.y = pack_bf16(p[2], p[3]);
-        pk.z = pack_bf16(p[4], p[5]);
-        pk.w = pack_bf16(p[6], p[7]);
-        const int panel = c >> 3, chunk = c & 7;
-        *reinterpret_cast<uint4*>(pb + panel * HB + r * 128 + ((chunk ^ (r & 7)) << 4)) = pk;
+        uint32_t pk[32];
+        if (valid == BK) {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const float p0 = ex2(fmaf(sv[2 * k], j.sl2, nm));
+            const float p1 = ex2(fmaf(sv[2 * k + 1], j.sl2, nm));
+            la += p0;
+            lb += p1;
+            pk[k] = pack_bf16(p0, p1);
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const int c0 = c * 64 + 2 * k;
+            const float p0 = c0 < valid ? ex2(fmaf(sv[2 * k], j.sl2, nm)) : 0.f;
+            const float p1 = c0 + 1 < valid ? ex2(fmaf(sv[2 * k + 1], j.sl2, nm)) : 0.f;
+            la += p0;
+            lb += p1;
+            pk[k] = pack_bf16(p0, p1);
+          }
+        }
+        tmem_st32(sc + c * 32, pk);
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      l += la + lb;
+      tmem_wait_st();
       fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_full + s);
+      if (lane == 0) mbar_arrive(p_full + g);
     }
-    // output row
-    const int qrow = q0 + r;
-    float o[128];
-    if (ok && nt > 0) {
-      ok = __all_sync(0xffffffffu, mbar_wait(pv_done, (nt - 1) & 1, abort_flag));
-      if (ok) {
-        fence_after_sync();
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(tmem + lane_off + O_COL + c * 32, v);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[c * 32 + i] = v[i];
-        }
-        tmem_wait_ld();
-      }
-    }
+    // ---- merge the two groups' partial softmax results
+    if (ok && ng > 0) ok = __all_sync(0xffffffffu, mbar_wait(pv_done + g, (ng - 1) & 1, abort_flag));
     if (!ok) {
       *abort_flag = 1;
       if (lane == 0) dev_fail(j.L, DEV_TIMEOUT, 402);
     }
-    const float inv = (ok && nt > 0 && l > 0.f) ? 1.0f / l : 0.f;
-    if (qrow < j.Nq) {
-      uint4* dst = reinterpret_cast<uint4*>(j.O + ((int64_t)h * j.Nq + qrow) * 128);
+    xst[(g * 2 + 0) * BQ + r] = ng > 0 && ok ? mrun : -INFINITY;
+    xst[(g * 2 + 1) * BQ + r] = ng > 0 && ok ? l : 0.f;
+    named_bar(1 + qd, 64);   // the two warps (one per group) of this TMEM lane quarter
+    const float m0 = xst[0 * BQ + r], l0 = xst[1 * BQ + r];
+    const float m1 = xst[2 * BQ + r], l1 = xst[3 * BQ + r];
+    const float mm = fmaxf(m0, m1);
+    const float a0 = m0 == -INFINITY ? 0.f : ex2(m0 - mm);
+    const float a1 = m1 == -INFINITY ? 0.f : ex2(m1 - mm);
+    const float den = fmaf(a1, l1, a0 * l0);
+    const float inv = den > 0.f ? 1.0f / den : 0.f;
+    const float c0 = a0 * inv, c1 = a1 * inv;
+    // the merge reads the other group's O too: observe its last PV completion as well
+    {
+      const int no = tiles_of(g ^ 1);
+      if (ok && no > 0) ok = __all_sync(0xffffffffu, mbar_wait(pv_done + (g ^ 1), (no - 1) & 1, abort_flag));
+    }
+    fence_after_sync();
+    // group g writes output columns [64 g, 64 g + 64) of this row from both O_0 and O_1
+    const int qrow = q0 + r;
+    const uint32_t o0 = tmem + lane_off + 128 + g * 64;
+    const uint32_t o1 = tmem + lane_off + 256 + 128 + g * 64;
+    const bool has0 = ok && tiles_of(0) > 0 && c0 != 0.f, has1 = ok && tiles_of(1) > 0 && c1 != 0.f;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        uint4 pk;
-        const float* x = o + c * 8;
-        const bool z = !(ok && nt > 0);
-        pk.x = pack_bf16(z ? 0.f : x[0] * inv, z ? 0.f : x[1] * inv);
-        pk.y = pack_bf16(z ? 0.f : x[2] * inv, z ? 0.f : x[3] * inv);
-        pk.z = pack_bf16(z ? 0.f : x[4] * inv, z ? 0.f : x[5] * inv);
-        pk.w = pack_bf16(z ? 0.f : x[6] * inv, z ? 0.f : x[7] * inv);
-        dst[c] = pk;
+    for (int c = 0; c < 2; ++c) {
+      float x0[32], x1[32];
+      tmem_ld32(o0 + c * 32, x0);
+      tmem_ld32(o1 + c * 32, x1);
+      tmem_wait_ld();
+      if (qrow < j.Nq) {
+        uint4* dst = reinterpret_cast<uint4*>(j.O + ((int64_t)h * j.Nq + qrow) * 128 + g * 64 + c * 32);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          float y[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float t0 = has0 ? x0[k * 8 + e] * c0 : 0.f;
+            y[e] = has1 ? fmaf(x1[k * 8 + e], c1, t0) : t0;
+          }
+          uint4 pk;
+          pk.x = pack_bf16(y[0], y[1]);
+          pk.y = pack_bf16(y[2], y[3]);
+          pk.z = pack_bf16(y[4], y[5]);
+          pk.w = pack_bf16(y[6], y[7]);
+          dst[k] = pk;
+        }
       }
     }
   }

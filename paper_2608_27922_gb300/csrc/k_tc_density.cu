@@ -63,7 +63,8 @@ constexpr int OFF_B = OFF_AX + EXT_BYTES;                 // [STAGES] tiles
 constexpr int OFF_BX = OFF_B + STAGES * TILE_BYTES;       // [STAGES] extension tiles
 constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [2][BN]
 constexpr int OFF_XCH = OFF_META + 2 * BN * 4;            // float [2][2][BM]
-constexpr int OFF_BAR = OFF_XCH + 2 * 2 * BM * 4;
+constexpr int OFF_FLAG = OFF_XCH + 2 * 2 * BM * 4;      // int: last-arrival flag of split tiles
+constexpr int OFF_BAR = OFF_FLAG + 16;
 constexpr size_t SMEM_BYTES = 1024 + OFF_BAR + 128;
 constexpr uint32_t LOAD_BYTES = TILE_BYTES + EXT_BYTES;
 
@@ -176,7 +177,13 @@ __global__ void __launch_bounds__(THREADS, 2)
   job_range(MODE, hd, L, nrows, c0, c1);
   const int row0 = blockIdx.x * BM;
   if (row0 >= nrows) return;                      // uniform: before any barrier or TMEM use
-  const int ntiles = c1 > c0 ? (c1 - c0 + BN - 1) / BN : 0;
+  // column tiles of this CTA: the row passes with plain row sums may split the column
+  // range over gridDim.z CTAs (their partial sums are combined below)
+  const int ntot = c1 > c0 ? (c1 - c0 + BN - 1) / BN : 0;
+  const int per = (ntot + (int)gridDim.z - 1) / (int)gridDim.z;
+  const int tbeg = min(ntot, (int)blockIdx.z * per);
+  const int ntiles = min(ntot, tbeg + per) - tbeg;
+  c0 += tbeg * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -391,11 +398,39 @@ __global__ void __launch_bounds__(THREADS, 2)
       *abort_flag = 1;
       if (lane == 0) dev_fail(j.w.L, DEV_TIMEOUT, 300 + MODE);
     }
+    bool finalize = true;
     if (MODE == TM_SCORE || MODE == TM_SUB || MODE == TM_NEWBASE) {
       // combine the two column halves of each row (no per-tile exchange in these passes)
       xch[half * BM + r_local] = acc;
       named_bar(1 + q, 64);
       acc = xch[r_local] + xch[BM + r_local];
+      if (gridDim.z > 1) {
+        // column-split row tile: publish this CTA's partial; the last CTA of the tile to
+        // arrive adds the partials in split order and finishes the rows
+        float* part = j.w.part + (int64_t)h * j.w.part_stride;
+        const int64_t zstride = (int64_t)gridDim.y * j.w.part_stride;
+        if (half == 0 && active) part[blockIdx.z * zstride + row] = acc;
+        __threadfence();
+        named_bar(6, 32 * EPI_WARPS);
+        int* flag = reinterpret_cast<int*>(smem + OFF_FLAG);
+        if (et == 0) {
+          int32_t* cnt = j.w.cnt + (int64_t)h * j.w.cnt_stride + blockIdx.x;
+          const int prev = atomicAdd(cnt, 1);
+          const int last = prev == (int)gridDim.z - 1;
+          if (last) atomicExch(cnt, 0);
+          *flag = last;
+        }
+        named_bar(6, 32 * EPI_WARPS);
+        finalize = *flag != 0;
+        if (finalize) {
+          __threadfence();
+          if (half == 0 && active) {
+            float sum = 0.f;
+            for (int z = 0; z < (int)gridDim.z; ++z) sum += __ldcg(part + z * zstride + row);
+            acc = sum;
+          }
+        }
+      }
     }
     if (MODE == TM_CROSS) {
       // each half saw only its own columns: the row's first crossing is the earlier one.
@@ -406,7 +441,7 @@ __global__ void __launch_bounds__(THREADS, 2)
       named_bar(1 + q, 64);
       cross = min(xi[r_local], xi[BM + r_local]);
     }
-    if (ok && active && half == 0) {
+    if (ok && finalize && active && half == 0) {
       if (MODE == TM_SCORE) {
         j.w.score[(int64_t)h * j.b.n_max + row] = (acc * c) / (float)hd.m_old;
       } else if (MODE == TM_CROSS) {
@@ -493,13 +528,13 @@ void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap
 template <int MODE>
 cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void* rk, const void* rx, int64_t rk_rows,
                       const void* ck, const void* cx, int64_t ck_rows, int max_rows, cudaStream_t s, Timer* t,
-                      const char* name) {
+                      const char* name, int split = 1) {
   CUtensorMap ma, max_, mb, mbx;
   if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_ext(&max_, rx, rk_rows, b.H, BM) ||
       !make_map_rows(&mb, ck, ck_rows, b.H, BN) || !make_map_ext(&mbx, cx, ck_rows, b.H, BN))
     return cudaErrorInvalidValue;
   TcJob job{b, w, kp};
-  dim3 grid((max_rows + BM - 1) / BM, b.H);
+  dim3 grid((max_rows + BM - 1) / BM, b.H, split);
   timer_begin(t, name, s);
   if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, job);
   else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, job);
@@ -535,7 +570,7 @@ cudaError_t tc_set_smem_limits() {
 
 cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
                             Timer* t) {
-  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc");
+  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", 2);
 }
 
 cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
@@ -550,12 +585,12 @@ cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cud
 
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   return launch_tc<TM_SUB>(b, w, kp, w.ksurv, w.ksurv_ext, b.M_max, w.kevict, w.kevict_ext, b.n_max, b.M_max, s,
-                           t, "subtract_tc");
+                           t, "subtract_tc", 2);
 }
 
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   return launch_tc<TM_NEWBASE>(b, w, kp, w.kperm, w.kperm_ext, b.n_max, b.k, w.bext, b.M_max, b.n_max, s, t,
-                               "newbase_tc");
+                               "newbase_tc", 2);
 }
 
 }  // namespace dkv
