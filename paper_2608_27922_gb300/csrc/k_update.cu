@@ -101,7 +101,47 @@ __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int ro
 }
 
 // Bitonic sort of (fkey(score) << 32 | source index) per head: ascending score,
-// equal scores in source order.
+// equal scores in source order (the keys are unique, so any correct sort is the
+// stable one).  Register-blocked: thread t holds keys [KPT t, KPT t + KPT); strides
+// below KPT are exchanged in registers, strides below 32 KPT with warp shuffles, and
+// only longer strides go through shared memory.
+template <int KPT, int J>
+__device__ __forceinline__ void cas_regs_c(unsigned long long (&x)[KPT], int t, int k) {
+#pragma unroll
+  for (int r = 0; r < KPT; ++r) {
+    if ((r ^ J) > r) {
+      const int i = t * KPT + r;
+      const bool up = (i & k) == 0;
+      const unsigned long long a = x[r], c = x[r ^ J];
+      if ((a > c) == up) { x[r] = c; x[r ^ J] = a; }
+    }
+  }
+}
+
+// in-register compare-exchange at stride j < KPT (strides as compile-time constants)
+template <int KPT>
+__device__ __forceinline__ void cas_regs(unsigned long long (&x)[KPT], int t, int k, int j) {
+  if (KPT > 8 && j == 8) cas_regs_c<KPT, (KPT > 8 ? 8 : 1)>(x, t, k);
+  else if (j == 4) cas_regs_c<KPT, 4>(x, t, k);
+  else if (j == 2) cas_regs_c<KPT, 2>(x, t, k);
+  else cas_regs_c<KPT, 1>(x, t, k);
+}
+
+template <int KPT>
+__device__ __forceinline__ void cas_shfl(unsigned long long (&x)[KPT], int t, int k, int j) {
+  const int ld = j / KPT;                       // lane distance of the partner
+  const bool lower = (threadIdx.x & ld) == 0;   // this thread holds the lower element
+#pragma unroll
+  for (int r = 0; r < KPT; ++r) {
+    const unsigned long long o = __shfl_xor_sync(0xffffffffu, x[r], ld);
+    const int i = t * KPT + r;
+    const bool up = (i & k) == 0;
+    const unsigned long long lo = x[r] < o ? x[r] : o, hi = x[r] < o ? o : x[r];
+    x[r] = (lower == up) ? lo : hi;
+  }
+}
+
+template <int KPT>
 __global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
   extern __shared__ unsigned long long keys[];
   const int h = blockIdx.x;
@@ -111,26 +151,56 @@ __global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
     for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = i;
     return;
   }
-  int n = 2;
+  int n = 32 * KPT;
   while (n < N) n <<= 1;
+  const int nthr = n / KPT;                       // <= blockDim.x
+  const int t = threadIdx.x;
+  const bool act = t < nthr;
   const float* sc = w.score + (int64_t)h * n_max;
-  for (int i = threadIdx.x; i < n; i += blockDim.x)
-    keys[i] = i < N ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
-  __syncthreads();
-  for (int k = 2; k <= n; k <<= 1) {
+  unsigned long long x[KPT];
+#pragma unroll
+  for (int r = 0; r < KPT; ++r) {
+    const int i = t * KPT + r;
+    x[r] = (act && i < N) ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
+  }
+  // sizes up to 32 KPT: registers and shuffles only
+  for (int k = 2; k <= 32 * KPT && k <= n; k <<= 1) {
     for (int j = k >> 1; j > 0; j >>= 1) {
+      if (j < KPT) cas_regs<KPT>(x, t, k, j);
+      else cas_shfl<KPT>(x, t, k, j);
+    }
+  }
+  // longer sizes: strides >= 32 KPT in shared memory, the rest in registers
+  for (int k = 64 * KPT; k <= n; k <<= 1) {
+    if (act)
+#pragma unroll
+      for (int r = 0; r < KPT; ++r) keys[t * KPT + r] = x[r];
+    __syncthreads();
+    for (int j = k >> 1; j >= 32 * KPT; j >>= 1) {
       for (int i = threadIdx.x; i < n; i += blockDim.x) {
         const int ix = i ^ j;
         if (ix > i) {
           const unsigned long long a = keys[i], c = keys[ix];
-          const bool up = (i & k) == 0;
-          if ((a > c) == up) { keys[i] = c; keys[ix] = a; }
+          if ((a > c) == ((i & k) == 0)) { keys[i] = c; keys[ix] = a; }
         }
       }
       __syncthreads();
     }
+    if (act)
+#pragma unroll
+      for (int r = 0; r < KPT; ++r) x[r] = keys[t * KPT + r];
+    __syncthreads();
+    for (int j = 16 * KPT; j > 0; j >>= 1) {
+      if (j < KPT) cas_regs<KPT>(x, t, k, j);
+      else cas_shfl<KPT>(x, t, k, j);
+    }
   }
-  for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = (int32_t)(keys[i] & 0xffffffffu);
+  if (act)
+#pragma unroll
+    for (int r = 0; r < KPT; ++r) {
+      const int i = t * KPT + r;
+      if (i < N) perm[i] = (int32_t)(x[r] & 0xffffffffu);
+    }
 }
 
 __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int esize) {
@@ -489,10 +559,11 @@ cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cud
 }
 
 cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
-  int n = 2;
+  int n = 256;
   while (n < b.n_max) n <<= 1;
   timer_begin(t, "sort", s);
-  k_sort<<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
+  if (n <= 8192) k_sort<8><<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
+  else k_sort<16><<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -539,7 +610,9 @@ cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cud
 }
 
 cudaError_t update_set_smem_limits() {
-  return cudaFuncSetAttribute(k_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8);
+  cudaError_t e = cudaFuncSetAttribute(k_sort<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 8192 * 8);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_sort<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8);
+  return e;
 }
 
 }  // namespace dkv
