@@ -63,6 +63,8 @@ def parse_args():
     ap.add_argument("--heads", type=int, default=0, help="override the head count (profiling runs)")
     ap.add_argument("--no-overlap", action="store_true",
                     help="run attention and the update on one stream instead of overlapping them")
+    ap.add_argument("--no-graphs", action="store_true",
+                    help="launch every step directly instead of replaying a captured CUDA graph")
     return ap.parse_args()
 
 
@@ -227,17 +229,18 @@ def run_ours(args):
             return
         # attention and admit both only read the bank (the update is atomic from the
         # reader's side), so they run concurrently; compress waits for attention
+        cur = torch.cuda.current_stream(dev)
         go = torch.cuda.Event()
-        go.record(stream)
+        go.record(cur)
         side.wait_event(go)
         bank.attend(Q, KW, VW, out=out, stream=side)
         done = torch.cuda.Event()
         done.record(side)
         if b is not None:
-            bank.admit(KC, VC, b, stream=stream)
-        stream.wait_event(done)
+            bank.admit(KC, VC, b, stream=cur)
+        cur.wait_event(done)
         if b is not None:
-            bank.compress(stream=stream)
+            bank.compress(stream=cur)
 
     def device_step(t):
         kw, vw = dblocks[wl.window_block(t)]
@@ -249,12 +252,31 @@ def run_ours(args):
         device_step(t)
     bank.sync()
 
+    # ---- optional CUDA graphs: one per timed step, captured before the timed region
+    # (each step reads its own input buffers; the bank state stays on the device, so the
+    # graphs replay the exact same work in order)
+    graphs = None
+    if not args.no_graphs:
+        bank.set_timing(True)   # the per-kernel timing events are captured into the graphs
+        graphs = []
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        with torch.cuda.stream(cap):
+            for i in range(K):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cap):
+                    device_step(W + i)
+                graphs.append(g)
+        stream.wait_stream(cap)
+        torch.cuda.synchronize()
+
     # ---- timed region: K steps, CUDA events on the launching stream, L2 flushed between steps
     clocks = ClockSampler(local, enabled=(not args.no_clocks) and rank == 0)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    bank.set_timing(True)
+    if graphs is None:
+        bank.set_timing(True)   # with graphs, the timing events were captured into them
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     keys = 0
     stats = []
@@ -264,7 +286,10 @@ def run_ours(args):
         if not args.no_flush:
             flush.fill_(float(i))
         ev[i][0].record(stream)
-        device_step(t)
+        if graphs is not None:
+            graphs[i].replay()
+        else:
+            device_step(t)
         ev[i][1].record(stream)
         ev[i][1].synchronize()
         L, hs = bank.stats()
@@ -382,6 +407,7 @@ def run_ours(args):
                                    f"N={wl.N}, M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
                        "score_mode": args.score_mode, "layers_per_gpu": 1,
                        "streams": "attention || admit, then compress" if not args.no_overlap else "one stream",
+                       "cuda_graphs": graphs is not None,
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                        "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
             "blocks_per_s": world * K / (total_ms_max / 1e3),

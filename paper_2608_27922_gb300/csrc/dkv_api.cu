@@ -60,17 +60,27 @@ struct Timer {
   }
 };
 
+// Inside a stream capture a plain event record only orders the graph; an external
+// record keeps the timestamp when the graph is replayed.
+static void record(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &st) == cudaSuccess && st == cudaStreamCaptureStatusActive)
+    cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+  else
+    cudaEventRecord(e, s);
+}
+
 void timer_begin(Timer* t, const char* name, cudaStream_t s) {
   if (!t || !t->on) return;
   t->cur = name;
   t->cur_a = t->get();
-  cudaEventRecord(t->cur_a, s);
+  record(t->cur_a, s);
 }
 
 void timer_end(Timer* t, cudaStream_t s) {
   if (!t || !t->on || !t->cur_a) return;
   cudaEvent_t b = t->get();
-  cudaEventRecord(b, s);
+  record(b, s);
   t->pending.push_back({t->cur, t->cur_a, b});
   t->cur_a = nullptr;
 }
