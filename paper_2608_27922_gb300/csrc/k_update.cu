@@ -30,6 +30,18 @@ __device__ __forceinline__ void warp_copy_row(void* dst, const void* src, int by
   for (int i = lane_id(); i < bytes / 16; i += 32) d[i] = s[i];
 }
 
+// Row copies as a flat loop over 16-byte chunks: a row of RB key bytes plus its 64-byte
+// extension row is RB/16 + 4 chunks; consecutive threads take consecutive chunks.
+template <typename RowMap>
+__device__ __forceinline__ void copy_rows(int nrows, int rb, RowMap map) {
+  const int per = rb / 16 + 4;
+  const int total = nrows * per;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
+    const int row = c / per, part = c - row * per;
+    map(row, part, per - 4);
+  }
+}
+
 __global__ void k_prepare(Bank b, Ws w, int N, int64_t step) {
   __shared__ int s_min_budget, s_live;
   if (threadIdx.x == 0) { s_min_budget = INT_MAX; s_live = 0; }
@@ -163,12 +175,49 @@ __global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
     const int i = t * KPT + r;
     x[r] = (act && i < N) ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
   }
-  // sizes up to 32 KPT: registers and shuffles only
+  // sizes up to 32 KPT: registers and shuffles only.  The bitonic direction bit (i & k)
+  // alternates between runs; when runs are merged below (KPT == 8) every run must come
+  // out ascending, so the last level uses a direction bit that is never set.
   for (int k = 2; k <= 32 * KPT && k <= n; k <<= 1) {
+    const int kd = (KPT == 8 && k == 32 * KPT) ? (1 << 30) : k;
     for (int j = k >> 1; j > 0; j >>= 1) {
-      if (j < KPT) cas_regs<KPT>(x, t, k, j);
-      else cas_shfl<KPT>(x, t, k, j);
+      if (j < KPT) cas_regs<KPT>(x, t, kd, j);
+      else cas_shfl<KPT>(x, t, kd, j);
     }
+  }
+  if (KPT == 8) {
+    // runs of 256 keys are sorted (warp-local bitonic above); merge runs pairwise in
+    // shared memory: a key's position in the merged run is its index in its own run
+    // plus its rank in the partner run (binary search)
+    unsigned long long* src = keys;
+    unsigned long long* dst = keys + n;
+    if (act)
+#pragma unroll
+      for (int r = 0; r < KPT; ++r) src[t * KPT + r] = x[r];
+    __syncthreads();
+    for (int len = 32 * KPT; len < n; len <<= 1) {
+      for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const unsigned long long key = src[i];
+        const int pair0 = i & ~(2 * len - 1);
+        const bool in_a = (i & len) == 0;
+        const int own = i - (in_a ? pair0 : pair0 + len);
+        const unsigned long long* other = src + (in_a ? pair0 + len : pair0);
+        // rank of key in the partner run: keys of the first run count the partner's
+        // strictly smaller keys, keys of the second run also count equal ones, so
+        // equal keys (the padding) keep distinct positions
+        int lo = 0, hi = len;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          const unsigned long long o = other[mid];
+          if (o < key || (!in_a && o == key)) lo = mid + 1; else hi = mid;
+        }
+        dst[pair0 + own + lo] = key;
+      }
+      __syncthreads();
+      unsigned long long* tmp = src; src = dst; dst = tmp;
+    }
+    for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = (int32_t)(src[i] & 0xffffffffu);
+    return;
   }
   // longer sizes: strides >= 32 KPT in shared memory, the rest in registers
   for (int k = 64 * KPT; k <= n; k <<= 1) {
@@ -205,14 +254,25 @@ __global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
 
 __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int esize) {
   const int h = blockIdx.y;
-  const int j = blockIdx.x * (blockDim.x / 32) + warp_id();
-  if (j >= N) return;
   const int rb = b.d * esize;
-  const int src = w.perm[(int64_t)h * b.n_max + j];
-  warp_copy_row((char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, Kc + ((int64_t)h * N + src) * rb, rb);
-  warp_copy_row((char*)w.kperm_ext + ((int64_t)h * b.n_max + j) * 64, (const char*)w.cext + ((int64_t)h * b.n_max + src) * 64,
-                64);
-  if (lane_id() == 0) w.kperm_norm[(int64_t)h * b.n_max + j] = w.cnorm[(int64_t)h * b.n_max + src];
+  const int64_t hn = (int64_t)h * b.n_max;
+  const int32_t* perm = w.perm + hn;
+  copy_rows(N, rb, [&](int j, int part, int kparts) {
+    const int src = perm[j];
+    if (src < 0 || src >= N) {   // pi must be a permutation of [0, N)
+      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 8000 + h);
+      return;
+    }
+    if (part < kparts) {
+      reinterpret_cast<uint4*>((char*)w.kperm + (hn + j) * rb)[part] =
+          reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb)[part];
+    } else {
+      const int e = part - kparts;
+      reinterpret_cast<uint4*>((char*)w.kperm_ext + (hn + j) * 64)[e] =
+          reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64)[e];
+      if (e == 0) w.kperm_norm[hn + j] = w.cnorm[hn + src];
+    }
+  });
 }
 
 // Per head: c_r = #{i : cross_i <= r} and feasibility c_r <= e_r for r in [0, rmax].
@@ -459,30 +519,31 @@ __global__ void k_gather(Bank b, Ws w, int esize) {
   const int h = blockIdx.y;
   const DevHead hd = w.hd[h];
   if (hd.empty || hd.e == 0) return;
-  const int row = blockIdx.x * (blockDim.x / 32) + warp_id();
   const int rb = b.d * esize;
   const int64_t bh = (int64_t)h * b.M_max;
+  const int64_t hn = (int64_t)h * b.n_max;
   const int ns = hd.m_old - hd.e;
-  if (row < ns) {
-    const int slot = w.surv_list[bh + row];
+  // rows [0, ns) survivors, [ns, ns + e) evicted
+  copy_rows(ns + hd.e, rb, [&](int row, int part, int kparts) {
+    const bool surv = row < ns;
+    const int slot = surv ? w.surv_list[bh + row] : w.evict_list[hn + row - ns];
     if (slot < 0 || slot >= hd.m_old) {
-      if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
+      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
       return;
     }
-    warp_copy_row((char*)w.ksurv + (bh + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
-    warp_copy_row((char*)w.ksurv_ext + (bh + row) * 64, (const char*)w.bext + (bh + slot) * 64, 64);
-    if (lane_id() == 0) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
-  }
-  if (row < hd.e) {
-    const int slot = w.evict_list[(int64_t)h * b.n_max + row];
-    if (slot < 0 || slot >= hd.m_old) {
-      if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 7500 + h);
-      return;
+    char* dk = surv ? (char*)w.ksurv + (bh + row) * rb : (char*)w.kevict + (hn + row - ns) * rb;
+    char* dx = surv ? (char*)w.ksurv_ext + (bh + row) * 64 : (char*)w.kevict_ext + (hn + row - ns) * 64;
+    if (part < kparts) {
+      reinterpret_cast<uint4*>(dk)[part] = reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb)[part];
+    } else {
+      const int e = part - kparts;
+      reinterpret_cast<uint4*>(dx)[e] = reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64)[e];
+      if (e == 0) {
+        if (surv) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
+        else w.kevict_norm[hn + row - ns] = b.knorm[bh + slot];
+      }
     }
-    warp_copy_row((char*)w.kevict + ((int64_t)h * b.n_max + row) * rb, (const char*)b.k + (bh + slot) * rb, rb);
-    warp_copy_row((char*)w.kevict_ext + ((int64_t)h * b.n_max + row) * 64, (const char*)w.bext + (bh + slot) * 64, 64);
-    if (lane_id() == 0) w.kevict_norm[(int64_t)h * b.n_max + row] = b.knorm[bh + slot];
-  }
+  });
 }
 
 // Eq. 12: the j-th admitted candidate (pi order) goes to the j-th evicted slot, the
@@ -490,30 +551,48 @@ __global__ void k_gather(Bank b, Ws w, int esize) {
 __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int esize) {
   const int h = blockIdx.y;
   const DevHead hd = w.hd[h];
-  const int j = blockIdx.x * (blockDim.x / 32) + warp_id();
   const int64_t bh = (int64_t)h * b.M_max;
+  const int64_t hn = (int64_t)h * b.n_max;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     const int m_new = hd.m_old - hd.e + hd.r;
     w.hd[h].m_new = m_new;
     b.occ[h] = m_new;
     if (m_new > hd.M) dev_fail(w.L, DEV_INCONSISTENT, 4000 + h);
   }
-  if (j >= hd.r) return;
-  const int slot = j < hd.e ? w.evict_list[(int64_t)h * b.n_max + j] : hd.m_old + (j - hd.e);
-  if (slot < 0 || slot >= hd.M) {
-    if (lane_id() == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
-    return;
-  }
   const int rb = b.d * esize;
-  const int src = w.perm[(int64_t)h * b.n_max + j];
-  warp_copy_row((char*)b.k + (bh + slot) * rb, (const char*)w.kperm + ((int64_t)h * b.n_max + j) * rb, rb);
-  warp_copy_row((char*)b.v + (bh + slot) * rb, Vc + ((int64_t)h * N + src) * rb, rb);
-  warp_copy_row((char*)w.bext + (bh + slot) * 64, (const char*)w.kperm_ext + ((int64_t)h * b.n_max + j) * 64, 64);
-  if (lane_id() == 0) {
-    b.knorm[bh + slot] = w.kperm_norm[(int64_t)h * b.n_max + j];
-    b.prov_step[bh + slot] = w.L->step;
-    b.prov_src[bh + slot] = src;
-    w.slot_new[(int64_t)h * b.n_max + j] = slot;
+  const int kp = rb / 16;
+  // per admitted row: key chunks, value chunks, then the 64-byte extension row
+  const int per = 2 * kp + 4;
+  const int total = hd.r * per;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
+    const int j = c / per, part = c - j * per;
+    const int slot = j < hd.e ? w.evict_list[hn + j] : hd.m_old + (j - hd.e);
+    if (slot < 0 || slot >= hd.M) {
+      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
+      continue;
+    }
+    const int src = w.perm[hn + j];
+    if (src < 0 || src >= N) {
+      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 8500 + h);
+      continue;
+    }
+    if (part < kp) {
+      reinterpret_cast<uint4*>((char*)b.k + (bh + slot) * rb)[part] =
+          reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb)[part];
+    } else if (part < 2 * kp) {
+      reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb)[part - kp] =
+          reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb)[part - kp];
+    } else {
+      const int e = part - 2 * kp;
+      reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64)[e] =
+          reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64)[e];
+      if (e == 0) {
+        b.knorm[bh + slot] = w.kperm_norm[hn + j];
+        b.prov_step[bh + slot] = w.L->step;
+        b.prov_src[bh + slot] = src;
+        w.slot_new[hn + j] = slot;
+      }
+    }
   }
 }
 
@@ -562,14 +641,14 @@ cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
   int n = 256;
   while (n < b.n_max) n <<= 1;
   timer_begin(t, "sort", s);
-  if (n <= 8192) k_sort<8><<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
+  if (n <= 8192) k_sort<8><<<b.H, BIG, (size_t)n * 16, s>>>(w, b.n_max);   // two merge buffers
   else k_sort<16><<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
   timer_end(t, s);
   return cudaGetLastError();
 }
 
 cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N + 7) / 8, b.H);
+  dim3 grid((N * (b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
   timer_begin(t, "permute", s);
   k_permute<<<grid, 256, 0, s>>>(b, w, (const char*)Kc, N, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -594,7 +673,7 @@ cudaError_t launch_select(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) 
 }
 
 cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
-  dim3 grid((b.M_max + 7) / 8, b.H);
+  dim3 grid((b.M_max * (b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
   timer_begin(t, "gather", s);
   k_gather<<<grid, 256, 0, s>>>(b, w, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -602,7 +681,7 @@ cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) 
 }
 
 cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N + 7) / 8, b.H);
+  dim3 grid((N * (2 * b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
   timer_begin(t, "commit", s);
   k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -610,7 +689,7 @@ cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cud
 }
 
 cudaError_t update_set_smem_limits() {
-  cudaError_t e = cudaFuncSetAttribute(k_sort<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 8192 * 8);
+  cudaError_t e = cudaFuncSetAttribute(k_sort<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 8192 * 16);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(k_sort<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8);
   return e;
 }
