@@ -126,12 +126,18 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* ba
   w.bext = take(Hh * Mm * 64);
   w.ksurv_ext = take(Hh * Mm * 64);
   w.kevict_ext = take(Hh * Nm * 64);
+  const int sort_stride = (n_max + 255) / 256 * 256;
+  w.sortbuf = (unsigned long long*)take(Hh * (size_t)sort_stride * 8);
+  const int invb_stride = (M_max + 3) & ~3;   // 16-byte rows for the bulk copies
+  w.invb = (float*)take((Hh * (size_t)invb_stride + 128) * 4);
   const int part_stride = (M_max > n_max ? M_max : n_max);
   const int cnt_stride = (part_stride + 127) / 128;
   w.part = (float*)take(2 * Hh * part_stride * 4);
   w.cnt = (int32_t*)take(Hh * cnt_stride * 4);
   w.part_stride = part_stride;
   w.cnt_stride = cnt_stride;
+  w.invb_stride = invb_stride;
+  w.sort_stride = sort_stride;
   w.hist_stride = hist_stride;
   w.snap_stride = snap_stride;
   w.feas_words = feas_words;
@@ -370,6 +376,7 @@ dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* st
   bank->last = s;
   cudaError_t e = cudaMemcpyAsync(bank->b.occ, occupancy, sizeof(int32_t) * bank->b.H, cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess) e = launch_bank_norms(bank->b, bank->w, bank->kp, s, &bank->timer);
+  if (e == cudaSuccess) e = launch_inv_base(bank->b, bank->w, s);
   return cuda_status(e);
 }
 

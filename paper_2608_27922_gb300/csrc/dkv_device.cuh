@@ -25,6 +25,7 @@ struct DevLayer {
   int64_t step;        // provenance step of the current update
   int32_t err;         // sticky error word (DEV_*)
   int32_t err_info;    // first failing site (kernel-specific code)
+  int32_t arrive;      // arrival counter of the r* kernel's head blocks (0 between launches)
 };
 
 // Per-head device state.

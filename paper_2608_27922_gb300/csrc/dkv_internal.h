@@ -51,9 +51,12 @@ struct Ws {
   void* bext;           // [H][M_max][32] bank (derived from the bank keys, kept in step)
   void* ksurv_ext;      // [H][M_max][32]
   void* kevict_ext;     // [H][n_max][32]
+  unsigned long long* sortbuf;   // [H][sort_stride] sorted runs of 256 sort keys
+  float* invb;          // [H][invb_stride] 1 / b of the bank states (derived from the
+                        //   baselines, kept in step; 128 floats of padding at the end)
   float* part;          // [2][H][part_stride] per-row partial sums of column-split passes
   int32_t* cnt;         // [H][cnt_stride] arrival counters of column-split row tiles (kept 0)
-  int hist_stride, snap_stride, feas_words, part_stride, cnt_stride;
+  int hist_stride, snap_stride, feas_words, part_stride, cnt_stride, invb_stride, sort_stride;
 };
 
 // Computes the sub-buffer offsets of the workspace; returns the total bytes.
@@ -89,6 +92,7 @@ cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cu
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // bank maintenance
 cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s);
 cudaError_t launch_set_occupancy(const Bank& b, const int32_t* occ_dev_src, int value, cudaStream_t s);
 // attention
 cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,

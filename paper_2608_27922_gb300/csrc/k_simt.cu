@@ -137,7 +137,9 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
     j.b.rho[bh + slot] = __fsub_rn(j.w.rho_t[bh + slot], acc);
   } else {
     j.b.rho[bh + self] = S;
-    j.b.base[bh + self] = fmaxf(S, j.kp.delta);
+    const float bnew = fmaxf(S, j.kp.delta);
+    j.b.base[bh + self] = bnew;
+    j.w.invb[(int64_t)h * j.w.invb_stride + self] = __frcp_rn(bnew);
   }
 }
 

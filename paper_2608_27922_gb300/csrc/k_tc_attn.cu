@@ -48,6 +48,13 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// max(a, b, c) in one instruction (three-input form, sm_100 and later).
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float y;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -238,7 +245,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_wait_ld();
           if (valid == BK) {
 #pragma unroll
-            for (int k = 0; k < 32; ++k) t[k & 7] = fmaxf(t[k & 7], v[k]);
+            for (int k = 0; k < 16; ++k) t[k & 7] = max3(t[k & 7], v[2 * k], v[2 * k + 1]);
           } else {
 #pragma unroll
             for (int k = 0; k < 32; ++k)
@@ -261,7 +268,11 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_wait_ld();
           uint32_t w32[32];
 #pragma unroll
-          for (int k = 0; k < 32; ++k) w32[k] = __float_as_uint(v[k] * alpha);
+          for (int k = 0; k < 16; ++k) {
+            const float2 y = __fmul2_rn(make_float2(v[2 * k], v[2 * k + 1]), make_float2(alpha, alpha));
+            w32[2 * k] = __float_as_uint(y.x);
+            w32[2 * k + 1] = __float_as_uint(y.y);
+          }
           tmem_st32(oc + c * 32, w32);
         }
       }
@@ -271,7 +282,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       // P_g = 2^(s log2(e)/sqrt(d) - m) as packed bf16 pairs over the first 64 columns of S_g
       const float nm = -mrun;
-      float la = 0.f, lb = 0.f;
+      const float2 sl2x2 = make_float2(j.sl2, j.sl2), nmx2 = make_float2(nm, nm);
+      float2 lab = make_float2(0.f, 0.f);     // running sums of the even and odd columns
       // pass 2: exponentials, 64 scores at a time
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
@@ -290,11 +302,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (valid == BK) {
 #pragma unroll
           for (int k = 0; k < 32; ++k) {
-            const float p0 = ex2(fmaf(sv[2 * k], j.sl2, nm));
-            const float p1 = ex2(fmaf(sv[2 * k + 1], j.sl2, nm));
-            la += p0;
-            lb += p1;
-            pk[k] = pack_bf16(p0, p1);
+            const float2 x = __ffma2_rn(make_float2(sv[2 * k], sv[2 * k + 1]), sl2x2, nmx2);
+            const float2 pp = make_float2(ex2(x.x), ex2(x.y));
+            lab = __fadd2_rn(lab, pp);
+            pk[k] = pack_bf16(pp.x, pp.y);
           }
         } else {
 #pragma unroll
@@ -302,14 +313,13 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int c0 = c * 64 + 2 * k;
             const float p0 = c0 < valid ? ex2(fmaf(sv[2 * k], j.sl2, nm)) : 0.f;
             const float p1 = c0 + 1 < valid ? ex2(fmaf(sv[2 * k + 1], j.sl2, nm)) : 0.f;
-            la += p0;
-            lb += p1;
+            lab = __fadd2_rn(lab, make_float2(p0, p1));
             pk[k] = pack_bf16(p0, p1);
           }
         }
         tmem_st32(sc + c * 32, pk);
       }
-      l += la + lb;
+      l += lab.x + lab.y;
       tmem_wait_st();
       fence_before_sync();
       __syncwarp();

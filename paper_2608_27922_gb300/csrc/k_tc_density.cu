@@ -93,44 +93,69 @@ __device__ __forceinline__ float term1(float a) {
   return P == 2 ? r2 : r2 * r2;
 }
 
-// |a|^-P + |b|^-P for a, b < 0 (one reciprocal).
+// Two interactions a, b < 0 under one reciprocal R = 1 / (a b):
+//   |a|^-P + |b|^-P          (term2x2)
+//   wa |a|^-P + wb |b|^-P    (term2wx2)
+// in packed fp32x2 arithmetic: lane l of X and Y holds one pair (a, b), and each lane
+// rounds exactly like the scalar expression.
 template <int P>
-__device__ __forceinline__ float term2(float a, float b) {
-  const float R = rcp_approx(a * b);
-  if (P == 1) return -(a + b) * R;
-  const float R2 = R * R;
-  if (P == 2) return R2 * fmaf(a, a, b * b);
-  const float a2 = a * a, b2 = b * b;
-  return (R2 * R2) * fmaf(a2, a2, b2 * b2);
+__device__ __forceinline__ float2 term2x2(float2 X, float2 Y) {
+  const float2 Pm = __fmul2_rn(X, Y);
+  const float2 R = make_float2(rcp_approx(Pm.x), rcp_approx(Pm.y));
+  if (P == 1) {
+    const float2 T = __fmul2_rn(__fadd2_rn(X, Y), R);
+    return make_float2(-T.x, -T.y);
+  }
+  const float2 R2 = __fmul2_rn(R, R);
+  if (P == 2) return __fmul2_rn(R2, __ffma2_rn(X, X, __fmul2_rn(Y, Y)));
+  const float2 X2 = __fmul2_rn(X, X), Y2 = __fmul2_rn(Y, Y);
+  return __fmul2_rn(__fmul2_rn(R2, R2), __ffma2_rn(X2, X2, __fmul2_rn(Y2, Y2)));
 }
 
-// wa |a|^-P + wb |b|^-P (one reciprocal).
 template <int P>
-__device__ __forceinline__ float term2w(float a, float b, float wa, float wb) {
-  const float R = rcp_approx(a * b);
-  if (P == 1) return -R * fmaf(wa, b, wb * a);
-  const float R2 = R * R;
-  if (P == 2) return R2 * fmaf(wa, b * b, wb * (a * a));
-  const float a2 = a * a, b2 = b * b;
-  return (R2 * R2) * fmaf(wa, b2 * b2, wb * (a2 * a2));
+__device__ __forceinline__ float2 term2wx2(float2 X, float2 Y, float2 WX, float2 WY) {
+  const float2 Pm = __fmul2_rn(X, Y);
+  const float2 R = make_float2(rcp_approx(Pm.x), rcp_approx(Pm.y));
+  if (P == 1) {
+    const float2 T = __fmul2_rn(R, __ffma2_rn(WX, Y, __fmul2_rn(WY, X)));
+    return make_float2(-T.x, -T.y);
+  }
+  const float2 R2 = __fmul2_rn(R, R);
+  if (P == 2) return __fmul2_rn(R2, __ffma2_rn(WX, __fmul2_rn(Y, Y), __fmul2_rn(WY, __fmul2_rn(X, X))));
+  const float2 X2 = __fmul2_rn(X, X), Y2 = __fmul2_rn(Y, Y);
+  return __fmul2_rn(__fmul2_rn(R2, R2), __ffma2_rn(WX, __fmul2_rn(Y2, Y2), __fmul2_rn(WY, __fmul2_rn(X2, X2))));
 }
 
-// Fixed-order binary tree over 16 values.
-__device__ __forceinline__ float tree16(float (&t)[16]) {
+// Fixed-order binary tree over 8 packed values, then the two lanes.
+__device__ __forceinline__ float tree8x2(float2 (&t)[8]) {
 #pragma unroll
-  for (int s = 8; s > 0; s >>= 1)
+  for (int s = 4; s > 0; s >>= 1)
 #pragma unroll
-    for (int k = 0; k < s; ++k) t[k] += t[k + s];
-  return t[0];
+    for (int k = 0; k < s; ++k) t[k] = __fadd2_rn(t[k], t[k + s]);
+  return t[0].x + t[0].y;
 }
 
-// Sum of |v_j|^-P over a full 32-column chunk.
+// Sum of |v_j|^-P over a full 32-column chunk: column j shares a reciprocal with
+// column j + 16.
 template <int P>
 __device__ __forceinline__ float chunk_sum(const float (&v)[32]) {
-  float t[16];
+  float2 t[8];
 #pragma unroll
-  for (int k = 0; k < 16; ++k) t[k] = term2<P>(v[2 * k], v[2 * k + 1]);
-  return tree16(t);
+  for (int k = 0; k < 8; ++k)
+    t[k] = term2x2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]));
+  return tree8x2(t);
+}
+
+// Sum of wb_j |v_j|^-P over a full 32-column chunk (wb in shared memory, 8-byte aligned).
+template <int P>
+__device__ __forceinline__ float chunk_sum_w(const float (&v)[32], const float* wb) {
+  const float2* w2 = reinterpret_cast<const float2*>(wb);
+  float2 t[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    t[k] = term2wx2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]), w2[k],
+                       w2[k + 8]);
+  return tree8x2(t);
 }
 
 // Same over the first `lim` columns (lim < 32), term by term.
@@ -169,6 +194,7 @@ __global__ void __launch_bounds__(THREADS, 2)
   uint64_t* bar_acce = bars + 7;    // [2]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  uint64_t* bar_meta = bars + 10;   // [2] SCORE: 1 / b of the columns of accumulator b
 
   const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
@@ -189,7 +215,11 @@ __global__ void __launch_bounds__(THREADS, 2)
   if (threadIdx.x == 0) {
     mbar_init(bar_a, 1);
     for (int s = 0; s < STAGES; ++s) { mbar_init(bar_full + s, 1); mbar_init(bar_empty + s, 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(bar_accf + b, 1); mbar_init(bar_acce + b, EPI_WARPS); }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_accf + b, 1);
+      mbar_init(bar_acce + b, EPI_WARPS);
+      mbar_init(bar_meta + b, 1);
+    }
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -243,6 +273,12 @@ __global__ void __launch_bounds__(THREADS, 2)
         if (!(ok = mbar_wait(bar_full + s, (t / STAGES) & 1, abort_flag))) break;
         if (!(ok = mbar_wait(bar_acce + b, ((t >> 1) & 1) ^ 1, abort_flag))) break;
         fence_after_sync();
+        if (MODE == TM_SCORE) {
+          // the epilogue of tile t - 2 has released meta[b]: fetch 1 / b_j of tile t
+          // (a whole 128-float row; the values past the last column are not used)
+          mbar_arrive_expect_tx(bar_meta + b, BN * 4);
+          bulk_load(meta + b * BN, j.w.invb + (int64_t)h * j.w.invb_stride + c0 + t * BN, BN * 4, bar_meta + b);
+        }
         const uint32_t b_base = smem_u32(smem + OFF_B + s * TILE_BYTES);
         const uint32_t bx_base = smem_u32(smem + OFF_BX + s * EXT_BYTES);
 #pragma unroll
@@ -259,10 +295,13 @@ __global__ void __launch_bounds__(THREADS, 2)
         *abort_flag = 1;
         dev_fail(j.w.L, DEV_TIMEOUT, 200 + MODE);
       }
-      // all issued MMAs must be complete before TMEM is freed
+      // all issued MMAs must be complete before TMEM is freed, and no copy may be in flight
       if (done > 0) {
         volatile int no_abort = 0;
         mbar_wait(bar_accf + ((done - 1) & 1), ((done - 1) >> 1) & 1, &no_abort);
+        if (MODE == TM_SCORE)
+          for (int t = done > 2 ? done - 2 : 0; t < done; ++t)
+            mbar_wait(bar_meta + (t & 1), (t >> 1) & 1, &no_abort);
       }
     }
   } else {
@@ -304,11 +343,8 @@ __global__ void __launch_bounds__(THREADS, 2)
       const int b = t & 1;
       const int col0 = c0 + t * BN;
       const int nc = min(BN, c1 - col0);
-      if (MODE == TM_SCORE) {   // 1 / b_j of this tile's columns
-        if (et < BN) meta[b * BN + et] = et < nc ? 1.0f / j.b.base[bh + col0 + et] : 0.f;
-        named_bar(5, 32 * EPI_WARPS);
-      }
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_accf + b, (t >> 1) & 1, abort_flag));
+      if (MODE == TM_SCORE && ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_meta + b, (t >> 1) & 1, abort_flag));
       float tot[2] = {0.f, 0.f};
       if (ok) {
         fence_after_sync();
@@ -323,10 +359,7 @@ __global__ void __launch_bounds__(THREADS, 2)
           if (MODE == TM_SCORE) {
             const float* ib = meta + b * BN + cs;
             if (lim == 32) {
-              float tt[16];
-#pragma unroll
-              for (int k = 0; k < 16; ++k) tt[k] = term2w<P>(v[2 * k], v[2 * k + 1], ib[2 * k], ib[2 * k + 1]);
-              tot[ch] = tree16(tt);
+              tot[ch] = chunk_sum_w<P>(v, ib);
             } else {
               float s = 0.f;
 #pragma unroll
@@ -458,7 +491,9 @@ __global__ void __launch_bounds__(THREADS, 2)
         if (self >= 0 && self < hd.M) {
           const float rho = c * acc;
           j.b.rho[bh + self] = rho;
-          j.b.base[bh + self] = fmaxf(rho, kp.delta);
+          const float bnew = fmaxf(rho, kp.delta);
+          j.b.base[bh + self] = bnew;
+          j.w.invb[(int64_t)h * j.w.invb_stride + self] = __frcp_rn(bnew);
         } else {
           dev_fail(j.w.L, DEV_INCONSISTENT, 6004);
         }
@@ -585,7 +620,7 @@ cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cud
 
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   return launch_tc<TM_SUB>(b, w, kp, w.ksurv, w.ksurv_ext, b.M_max, w.kevict, w.kevict_ext, b.n_max, b.M_max, s,
-                           t, "subtract_tc", 2);
+                           t, "subtract_tc");
 }
 
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {

@@ -23,13 +23,6 @@ constexpr int BIG = 1024;   // threads of the one-block-per-head kernels
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 
-// Copies one row of `bytes` bytes (a multiple of 16) with one warp.
-__device__ __forceinline__ void warp_copy_row(void* dst, const void* src, int bytes) {
-  const uint4* s = reinterpret_cast<const uint4*>(src);
-  uint4* d = reinterpret_cast<uint4*>(dst);
-  for (int i = lane_id(); i < bytes / 16; i += 32) d[i] = s[i];
-}
-
 // Row copies as a flat loop over 16-byte chunks: a row of RB key bytes plus its 64-byte
 // extension row is RB/16 + 4 chunks; consecutive threads take consecutive chunks.
 template <typename RowMap>
@@ -112,17 +105,22 @@ __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int ro
   }
 }
 
-// Bitonic sort of (fkey(score) << 32 | source index) per head: ascending score,
-// equal scores in source order (the keys are unique, so any correct sort is the
-// stable one).  Register-blocked: thread t holds keys [KPT t, KPT t + KPT); strides
-// below KPT are exchanged in registers, strides below 32 KPT with warp shuffles, and
-// only longer strides go through shared memory.
-template <int KPT, int J>
-__device__ __forceinline__ void cas_regs_c(unsigned long long (&x)[KPT], int t, int k) {
+// Sort of the keys (fkey(score) << 32 | source index) per head: ascending score, equal
+// scores in source order (the keys are unique, so any correct sort is the stable one).
+// Phase 1 sorts runs of RUN = 256 keys, one warp each, with a bitonic network kept in
+// registers (thread = SKPT consecutive keys; strides below SKPT) and warp shuffles
+// (longer strides).  Phase 2 places every key at its index in its own run plus its
+// rank in each other run, so no merge levels are needed and every run is placed by
+// its own block.
+constexpr int SKPT = 8;
+constexpr int RUN = 32 * SKPT;
+
+template <int J>
+__device__ __forceinline__ void cas_regs_c(unsigned long long (&x)[SKPT], int t, int k) {
 #pragma unroll
-  for (int r = 0; r < KPT; ++r) {
+  for (int r = 0; r < SKPT; ++r) {
     if ((r ^ J) > r) {
-      const int i = t * KPT + r;
+      const int i = t * SKPT + r;
       const bool up = (i & k) == 0;
       const unsigned long long a = x[r], c = x[r ^ J];
       if ((a > c) == up) { x[r] = c; x[r ^ J] = a; }
@@ -130,126 +128,101 @@ __device__ __forceinline__ void cas_regs_c(unsigned long long (&x)[KPT], int t, 
   }
 }
 
-// in-register compare-exchange at stride j < KPT (strides as compile-time constants)
-template <int KPT>
-__device__ __forceinline__ void cas_regs(unsigned long long (&x)[KPT], int t, int k, int j) {
-  if (KPT > 8 && j == 8) cas_regs_c<KPT, (KPT > 8 ? 8 : 1)>(x, t, k);
-  else if (j == 4) cas_regs_c<KPT, 4>(x, t, k);
-  else if (j == 2) cas_regs_c<KPT, 2>(x, t, k);
-  else cas_regs_c<KPT, 1>(x, t, k);
+// in-register compare-exchange at stride j < SKPT (strides as compile-time constants)
+__device__ __forceinline__ void cas_regs(unsigned long long (&x)[SKPT], int t, int k, int j) {
+  if (j == 4) cas_regs_c<4>(x, t, k);
+  else if (j == 2) cas_regs_c<2>(x, t, k);
+  else cas_regs_c<1>(x, t, k);
 }
 
-template <int KPT>
-__device__ __forceinline__ void cas_shfl(unsigned long long (&x)[KPT], int t, int k, int j) {
-  const int ld = j / KPT;                       // lane distance of the partner
-  const bool lower = (threadIdx.x & ld) == 0;   // this thread holds the lower element
+// compare-exchange with the lane at distance j / SKPT
+__device__ __forceinline__ void cas_shfl(unsigned long long (&x)[SKPT], int t, int k, int j) {
+  const int ld = j / SKPT;
+  const bool lower = (t & ld) == 0;   // this lane holds the lower element of each pair
 #pragma unroll
-  for (int r = 0; r < KPT; ++r) {
+  for (int r = 0; r < SKPT; ++r) {
     const unsigned long long o = __shfl_xor_sync(0xffffffffu, x[r], ld);
-    const int i = t * KPT + r;
+    const int i = t * SKPT + r;
     const bool up = (i & k) == 0;
     const unsigned long long lo = x[r] < o ? x[r] : o, hi = x[r] < o ? o : x[r];
     x[r] = (lower == up) ? lo : hi;
   }
 }
 
-template <int KPT>
-__global__ void __launch_bounds__(BIG) k_sort(Ws w, int n_max) {
-  extern __shared__ unsigned long long keys[];
-  const int h = blockIdx.x;
+// Phase 1: warp w of block x sorts run a = 8 x + w (source indices [256 a, 256 a + 256),
+// padded with ~0) ascending; the direction bit is taken from the run-local index, so
+// every run comes out ascending.
+__global__ void __launch_bounds__(256) k_sort_runs(Ws w, int n_max) {
+  const int h = blockIdx.y;
   const int N = w.L->N;
-  int32_t* perm = w.perm + (int64_t)h * n_max;
   if (w.hd[h].empty) {   // empty bank: source order (Alg. 1, m = 0 branch)
-    for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = i;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x)
+      w.perm[(int64_t)h * n_max + i] = i;
     return;
   }
-  int n = 32 * KPT;
-  while (n < N) n <<= 1;
-  const int nthr = n / KPT;                       // <= blockDim.x
-  const int t = threadIdx.x;
-  const bool act = t < nthr;
+  const int a = blockIdx.x * 8 + warp_id();
+  if (a * RUN >= N) return;                       // warp-uniform
+  const int t = lane_id();
   const float* sc = w.score + (int64_t)h * n_max;
-  unsigned long long x[KPT];
+  unsigned long long x[SKPT];
 #pragma unroll
-  for (int r = 0; r < KPT; ++r) {
-    const int i = t * KPT + r;
-    x[r] = (act && i < N) ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
+  for (int r = 0; r < SKPT; ++r) {
+    const int i = a * RUN + t * SKPT + r;
+    x[r] = i < N ? ((unsigned long long)fkey(sc[i]) << 32) | (unsigned)i : ~0ull;
   }
-  // sizes up to 32 KPT: registers and shuffles only.  The bitonic direction bit (i & k)
-  // alternates between runs; when runs are merged below (KPT == 8) every run must come
-  // out ascending, so the last level uses a direction bit that is never set.
-  for (int k = 2; k <= 32 * KPT && k <= n; k <<= 1) {
-    const int kd = (KPT == 8 && k == 32 * KPT) ? (1 << 30) : k;
+  for (int k = 2; k <= RUN; k <<= 1)
     for (int j = k >> 1; j > 0; j >>= 1) {
-      if (j < KPT) cas_regs<KPT>(x, t, kd, j);
-      else cas_shfl<KPT>(x, t, kd, j);
+      if (j < SKPT) cas_regs(x, t, k, j);
+      else cas_shfl(x, t, k, j);
     }
-  }
-  if (KPT == 8) {
-    // runs of 256 keys are sorted (warp-local bitonic above); merge runs pairwise in
-    // shared memory: a key's position in the merged run is its index in its own run
-    // plus its rank in the partner run (binary search)
-    unsigned long long* src = keys;
-    unsigned long long* dst = keys + n;
-    if (act)
+  unsigned long long* out = w.sortbuf + (int64_t)h * w.sort_stride + a * RUN + t * SKPT;
 #pragma unroll
-      for (int r = 0; r < KPT; ++r) src[t * KPT + r] = x[r];
-    __syncthreads();
-    for (int len = 32 * KPT; len < n; len <<= 1) {
-      for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const unsigned long long key = src[i];
-        const int pair0 = i & ~(2 * len - 1);
-        const bool in_a = (i & len) == 0;
-        const int own = i - (in_a ? pair0 : pair0 + len);
-        const unsigned long long* other = src + (in_a ? pair0 + len : pair0);
-        // rank of key in the partner run: keys of the first run count the partner's
-        // strictly smaller keys, keys of the second run also count equal ones, so
-        // equal keys (the padding) keep distinct positions
-        int lo = 0, hi = len;
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          const unsigned long long o = other[mid];
-          if (o < key || (!in_a && o == key)) lo = mid + 1; else hi = mid;
-        }
-        dst[pair0 + own + lo] = key;
-      }
-      __syncthreads();
-      unsigned long long* tmp = src; src = dst; dst = tmp;
-    }
-    for (int i = threadIdx.x; i < N; i += blockDim.x) perm[i] = (int32_t)(src[i] & 0xffffffffu);
+  for (int r = 0; r < SKPT; r += 2)
+    *reinterpret_cast<ulonglong2*>(out + r) = make_ulonglong2(x[r], x[r + 1]);
+}
+
+// Number of keys of the sorted run r[0..RUN) below x (branchless, 9 probes).
+__device__ __forceinline__ int run_rank(const unsigned long long* r, unsigned long long x) {
+  int pos = 0;
+#pragma unroll
+  for (int s = RUN / 2; s > 0; s >>= 1)
+    if (r[pos + s - 1] < x) pos += s;
+  return pos + (r[pos] < x ? 1 : 0);
+}
+
+// Phase 2: block (a, h) places the keys of run a: final position = index in run a plus
+// the number of smaller keys in every other run (keys are unique, so positions are
+// distinct and cover [0, N)).
+__global__ void __launch_bounds__(RUN) k_sort_rank(Ws w, int n_max) {
+  extern __shared__ unsigned long long runs[];
+  const int h = blockIdx.y;
+  const int N = w.L->N;
+  if (w.hd[h].empty) return;
+  const int nruns = (N + RUN - 1) / RUN;
+  const int a = blockIdx.x;
+  if (a >= nruns) return;                         // block-uniform
+  const unsigned long long* src = w.sortbuf + (int64_t)h * w.sort_stride;
+  for (int i = threadIdx.x; i < nruns * RUN / 2; i += RUN)
+    reinterpret_cast<ulonglong2*>(runs)[i] = reinterpret_cast<const ulonglong2*>(src)[i];
+  __syncthreads();
+  const int t = threadIdx.x;
+  const unsigned long long x = runs[a * RUN + t];
+  if (x == ~0ull) return;                         // padding of the last run
+  int pos = t;
+  int b = 0;
+  for (; b + 4 <= nruns; b += 4) {
+    int c[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) c[u] = b + u == a ? 0 : run_rank(runs + (b + u) * RUN, x);
+    pos += (c[0] + c[1]) + (c[2] + c[3]);
+  }
+  for (; b < nruns; ++b)
+    if (b != a) pos += run_rank(runs + b * RUN, x);
+  if (pos >= N) {
+    dev_fail(w.L, DEV_INCONSISTENT, 8800 + h);
     return;
   }
-  // longer sizes: strides >= 32 KPT in shared memory, the rest in registers
-  for (int k = 64 * KPT; k <= n; k <<= 1) {
-    if (act)
-#pragma unroll
-      for (int r = 0; r < KPT; ++r) keys[t * KPT + r] = x[r];
-    __syncthreads();
-    for (int j = k >> 1; j >= 32 * KPT; j >>= 1) {
-      for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const int ix = i ^ j;
-        if (ix > i) {
-          const unsigned long long a = keys[i], c = keys[ix];
-          if ((a > c) == ((i & k) == 0)) { keys[i] = c; keys[ix] = a; }
-        }
-      }
-      __syncthreads();
-    }
-    if (act)
-#pragma unroll
-      for (int r = 0; r < KPT; ++r) x[r] = keys[t * KPT + r];
-    __syncthreads();
-    for (int j = 16 * KPT; j > 0; j >>= 1) {
-      if (j < KPT) cas_regs<KPT>(x, t, k, j);
-      else cas_shfl<KPT>(x, t, k, j);
-    }
-  }
-  if (act)
-#pragma unroll
-    for (int r = 0; r < KPT; ++r) {
-      const int i = t * KPT + r;
-      if (i < N) perm[i] = (int32_t)(x[r] & 0xffffffffu);
-    }
+  w.perm[(int64_t)h * n_max + pos] = (int32_t)(x & 0xffffffffu);
 }
 
 __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int esize) {
@@ -276,61 +249,77 @@ __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int 
 }
 
 // Per head: c_r = #{i : cross_i <= r} and feasibility c_r <= e_r for r in [0, rmax].
-__global__ void __launch_bounds__(BIG) k_rstar_head(Ws w) {
+// Reads a DevHead written by another block of the same launch (bypassing L1).
+__device__ __forceinline__ DevHead ld_head_cg(const DevHead* p) {
+  DevHead hd;
+  const int4 a = __ldcg(reinterpret_cast<const int4*>(p));
+  const int4 c = __ldcg(reinterpret_cast<const int4*>(p) + 1);
+  hd.m_old = a.x; hd.M = a.y; hd.r = a.z; hd.e = a.w;
+  hd.n_mand = c.x; hd.n_pre = c.y; hd.m_new = c.z; hd.empty = c.w;
+  return hd;
+}
+
+// One block per head: violator counts c_r (prefix sums of the crossing histogram),
+// budgets e_r (Eq. 10) and the feasibility bit of every prefix r; the last block to
+// finish combines the heads (Eq. 11) and sets r, e of every head.
+__global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   __shared__ int s_tot[BIG];
-  __shared__ int s_best;
+  __shared__ int s_best, s_last;
   const int h = blockIdx.x;
   const DevHead hd = w.hd[h];
   const int rmax = w.L->rmax;
+  const int N = w.L->N;
   uint32_t* feas = w.feas + (int64_t)h * w.feas_words;
   const int nw = (rmax + 1 + 31) / 32;
+  if (threadIdx.x == 0) s_best = 0;
   if (hd.empty) {   // an empty head does not constrain the shared prefix
     for (int i = threadIdx.x; i < nw; i += blockDim.x) feas[i] = 0xffffffffu;
-    return;
-  }
-  for (int i = threadIdx.x; i < nw; i += blockDim.x) feas[i] = 0u;
-  if (threadIdx.x == 0) s_best = 0;
-  const int n = rmax + 1;
-  const int chunk = (n + blockDim.x - 1) / blockDim.x;
-  const int lo = threadIdx.x * chunk, hi = min(n, lo + chunk);
-  const int32_t* hist = w.hist + (int64_t)h * w.hist_stride;
-  int tot = 0;
-  for (int r = lo; r < hi; ++r) tot += hist[r];
-  s_tot[threadIdx.x] = tot;
-  __syncthreads();
-  for (int o = 1; o < (int)blockDim.x; o <<= 1) {   // inclusive Hillis-Steele scan
-    const int v = threadIdx.x >= o ? s_tot[threadIdx.x - o] : 0;
+  } else {
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) feas[i] = 0u;
+    const int n = rmax + 1;
+    const int chunk = (n + blockDim.x - 1) / blockDim.x;
+    const int lo = threadIdx.x * chunk, hi = min(n, lo + chunk);
+    const int32_t* hist = w.hist + (int64_t)h * w.hist_stride;
+    int tot = 0;
+    for (int r = lo; r < hi; ++r) tot += hist[r];
+    s_tot[threadIdx.x] = tot;
     __syncthreads();
-    s_tot[threadIdx.x] += v;
-    __syncthreads();
-  }
-  int c = s_tot[threadIdx.x] - tot;   // exclusive prefix
-  int best = 0;
-  for (int r = lo; r < hi; ++r) {
-    c += hist[r];
-    const int e = max(0, hd.m_old + r - hd.M);
-    const bool ok = (r == 0) || (c <= e);   // r = 0 is always feasible (Sec. 3.4 Step 2)
-    if (ok) {
-      atomicOr(&feas[r >> 5], 1u << (r & 31));
-      best = r;
+    for (int o = 1; o < (int)blockDim.x; o <<= 1) {   // inclusive Hillis-Steele scan
+      const int v = threadIdx.x >= o ? s_tot[threadIdx.x - o] : 0;
+      __syncthreads();
+      s_tot[threadIdx.x] += v;
+      __syncthreads();
     }
+    int c = s_tot[threadIdx.x] - tot;   // exclusive prefix
+    int best = 0;
+    for (int r = lo; r < hi; ++r) {
+      c += hist[r];
+      const int e = max(0, hd.m_old + r - hd.M);
+      const bool ok = (r == 0) || (c <= e);   // r = 0 is always feasible (Sec. 3.4 Step 2)
+      if (ok) {
+        atomicOr(&feas[r >> 5], 1u << (r & 31));
+        best = r;
+      }
+    }
+    atomicMax(&s_best, best);
   }
-  atomicMax(&s_best, best);
+  __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) w.hd[h].r = s_best;   // largest feasible prefix of this head alone
-}
-
-__global__ void __launch_bounds__(BIG) k_rstar_layer(Bank b, Ws w, int sync_heads) {
-  __shared__ int s_best;
-  const int rmax = w.L->rmax;
-  const int N = w.L->N;
-  const int nw = (rmax + 1 + 31) / 32;
+  if (threadIdx.x == 0) {
+    if (!hd.empty) w.hd[h].r = s_best;   // largest feasible prefix of this head alone
+    __threadfence();
+    s_last = atomicAdd(&w.L->arrive, 1) == (int)gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  // ---- last block: the layer's shared prefix
+  __threadfence();
   if (threadIdx.x == 0) s_best = 0;
   __syncthreads();
   if (sync_heads) {
     for (int i = threadIdx.x; i < nw; i += blockDim.x) {
       uint32_t a = 0xffffffffu;
-      for (int h = 0; h < b.H; ++h) a &= w.feas[(int64_t)h * w.feas_words + i];
+      for (int hh = 0; hh < b.H; ++hh) a &= __ldcg(w.feas + (int64_t)hh * w.feas_words + i);
       if (i == nw - 1 && ((rmax + 1) & 31)) a &= (1u << ((rmax + 1) & 31)) - 1u;
       if (i == 0) a |= 1u;
       if (a) atomicMax(&s_best, i * 32 + 31 - __clz(a));
@@ -341,22 +330,24 @@ __global__ void __launch_bounds__(BIG) k_rstar_layer(Bank b, Ws w, int sync_head
   __shared__ int s_rmax_used, s_rmin_used;
   if (threadIdx.x == 0) { s_rmax_used = 0; s_rmin_used = INT_MAX; }
   __syncthreads();
-  for (int h = threadIdx.x; h < b.H; h += blockDim.x) {
-    DevHead hd = w.hd[h];
+  for (int hh = threadIdx.x; hh < b.H; hh += blockDim.x) {
+    DevHead d = ld_head_cg(w.hd + hh);
     int r;
-    if (hd.empty) r = min(N, hd.M);
-    else r = sync_heads ? rstar : hd.r;
-    hd.r = r;
-    hd.e = hd.empty ? 0 : max(0, hd.m_old + r - hd.M);
-    w.hd[h] = hd;
+    if (d.empty) r = min(N, d.M);
+    else r = sync_heads ? rstar : d.r;
+    d.r = r;
+    d.e = d.empty ? 0 : max(0, d.m_old + r - d.M);
+    w.hd[hh] = d;
     atomicMax(&s_rmax_used, r);
     atomicMin(&s_rmin_used, r);
   }
   __syncthreads();
   // reported r*: Alg. 1's min(N, M) when every head starts empty (min over per-head budgets),
   // the shared prefix when synchronised, else the largest per-head prefix
-  if (threadIdx.x == 0)
+  if (threadIdx.x == 0) {
     w.L->r_star = w.L->empty_all ? s_rmin_used : (sync_heads ? rstar : s_rmax_used);
+    w.L->arrive = 0;
+  }
 }
 
 // Block-wide exclusive scan of one flag per thread; returns this thread's offset and
@@ -376,6 +367,53 @@ __device__ int block_scan_flag(int flag, int* s_warp, int* total) {
   *total = s_warp[32];
   __syncthreads();
   return off;
+}
+
+// Adds one to s_hist[bin] for every lane with valid set, one shared-memory atomic per
+// distinct bin of the warp (all 32 lanes must call it).
+__device__ __forceinline__ void hist_add(int* s_hist, bool valid, unsigned bin) {
+  const unsigned key = valid ? bin : 0xffffffffu;
+  const unsigned peers = __match_any_sync(0xffffffffu, key);
+  if (valid && lane_id() == __ffs(peers) - 1) atomicAdd(&s_hist[bin], __popc(peers));
+}
+
+// Warp 0: the bin of a 256-bin histogram where the running count, taken from the top
+// bin down (from_top) or from bin 0 up, first reaches kk (>= 1).  Returns the bin and
+// kk minus the count before it through *bin and *rest; false if the total is below kk.
+__device__ bool find_bin(const int* s_hist, unsigned kk, bool from_top, unsigned* bin, unsigned* rest) {
+  const int l = lane_id();
+  unsigned c[8], cnt = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int bj = from_top ? 255 - (8 * l + j) : 8 * l + j;
+    c[j] = (unsigned)s_hist[bj];
+    cnt += c[j];
+  }
+  unsigned incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (l >= o) incl += v;
+  }
+  const unsigned hit = __ballot_sync(0xffffffffu, incl >= kk);
+  if (hit == 0u) return false;
+  const int src = __ffs(hit) - 1;
+  unsigned my_bin = 0, my_rest = 0;
+  if (l == src) {
+    unsigned cum = incl - cnt;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (cum + c[j] >= kk) {
+        my_bin = from_top ? 255 - (8 * l + j) : 8 * l + j;
+        my_rest = kk - cum;
+        break;
+      }
+      cum += c[j];
+    }
+  }
+  *bin = __shfl_sync(0xffffffffu, my_bin, src);
+  *rest = __shfl_sync(0xffffffffu, my_rest, src);
+  return true;
 }
 
 __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
@@ -402,8 +440,12 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     npre += (c == 0);
     nm += (r > 0 && c <= r);
   }
-  atomicAdd(&s_cnt[0], nm);
-  atomicAdd(&s_cnt[1], npre);
+  nm = __reduce_add_sync(0xffffffffu, nm);
+  npre = __reduce_add_sync(0xffffffffu, npre);
+  if (lane_id() == 0) {
+    atomicAdd(&s_cnt[0], nm);
+    atomicAdd(&s_cnt[1], npre);
+  }
   __syncthreads();
   int n_mand = s_cnt[0];
   if (threadIdx.x == 0) { w.hd[h].n_mand = n_mand; w.hd[h].n_pre = s_cnt[1]; }
@@ -421,18 +463,23 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int i = threadIdx.x; i < 256; i += blockDim.x) s_hist[i] = 0;
       __syncthreads();
-      for (int i = threadIdx.x; i < m; i += blockDim.x) {
-        if (r > 0 && cross[i] <= r) continue;
-        const unsigned key = fkey(rt[i]);
-        if ((key & mask) == prefix) atomicAdd(&s_hist[(key >> shift) & 255u], 1);
+      for (int base = 0; base < m; base += blockDim.x) {
+        const int i = base + threadIdx.x;
+        bool v = false;
+        unsigned key = 0;
+        if (i < m && !(r > 0 && cross[i] <= r)) {
+          key = fkey(rt[i]);
+          v = (key & mask) == prefix;
+        }
+        hist_add(s_hist, v, (key >> shift) & 255u);
       }
       __syncthreads();
-      if (threadIdx.x == 0) {
-        unsigned kk = s_kk, cum = 0;
-        for (int bin = 255; bin >= 0; --bin) {
-          const unsigned c = (unsigned)s_hist[bin];
-          if (cum + c >= kk) { s_kk = kk - cum; s_prefix = prefix | ((unsigned)bin << shift); break; }
-          cum += c;
+      if (warp_id() == 0) {
+        unsigned bin, rest;
+        if (find_bin(s_hist, s_kk, true, &bin, &rest)) {
+          if (lane_id() == 0) { s_kk = rest; s_prefix = prefix | (bin << shift); }
+        } else if (lane_id() == 0) {
+          dev_fail(w.L, DEV_INCONSISTENT, 2100 + h);
         }
       }
       __syncthreads();
@@ -450,7 +497,8 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
   __syncthreads();
   if (threadIdx.x == 0) s_cnt[0] = 0;
   __syncthreads();
-  atomicAdd(&s_cnt[0], n_eq_local);
+  n_eq_local = __reduce_add_sync(0xffffffffu, n_eq_local);
+  if (lane_id() == 0) atomicAdd(&s_cnt[0], n_eq_local);
   __syncthreads();
   const unsigned n_eq = (unsigned)s_cnt[0];
   unsigned long long tprefix = 0, tmask = 0;
@@ -461,19 +509,23 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     for (int shift = 56; shift >= 0; shift -= 8) {
       for (int i = threadIdx.x; i < 256; i += blockDim.x) s_hist[i] = 0;
       __syncthreads();
-      for (int i = threadIdx.x; i < m; i += blockDim.x) {
-        if ((r > 0 && cross[i] <= r) || fkey(rt[i]) != T) continue;
-        const unsigned long long tk = ((unsigned long long)(uint32_t)b.prov_step[bh + i] << 32) |
-                                      (uint32_t)b.prov_src[bh + i];
-        if ((tk & tmask) == tprefix) atomicAdd(&s_hist[(tk >> shift) & 255ull], 1);
+      for (int base = 0; base < m; base += blockDim.x) {
+        const int i = base + threadIdx.x;
+        bool v = false;
+        unsigned long long tk = 0;
+        if (i < m && !(r > 0 && cross[i] <= r) && fkey(rt[i]) == T) {
+          tk = ((unsigned long long)(uint32_t)b.prov_step[bh + i] << 32) | (uint32_t)b.prov_src[bh + i];
+          v = (tk & tmask) == tprefix;
+        }
+        hist_add(s_hist, v, (unsigned)((tk >> shift) & 255ull));
       }
       __syncthreads();
-      if (threadIdx.x == 0) {   // smallest first
-        unsigned kk = s_kk, cum = 0;
-        for (int bin = 0; bin < 256; ++bin) {
-          const unsigned c = (unsigned)s_hist[bin];
-          if (cum + c >= kk) { s_kk = kk - cum; s_tprefix = tprefix | ((unsigned long long)bin << shift); break; }
-          cum += c;
+      if (warp_id() == 0) {   // smallest first
+        unsigned bin, rest;
+        if (find_bin(s_hist, s_kk, false, &bin, &rest)) {
+          if (lane_id() == 0) { s_kk = rest; s_tprefix = tprefix | ((unsigned long long)bin << shift); }
+        } else if (lane_id() == 0) {
+          dev_fail(w.L, DEV_INCONSISTENT, 2200 + h);
         }
       }
       __syncthreads();
@@ -511,6 +563,14 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     n_sv += min((int)blockDim.x, m - base) - tot;
   }
   if (threadIdx.x == 0 && n_ev != e) dev_fail(w.L, DEV_INCONSISTENT, 3000 + h);
+}
+
+// 1 / b of every occupied bank slot (after an import; the update keeps it in step).
+__global__ void k_inv_base(Bank b, Ws w) {
+  const int h = blockIdx.y;
+  const int m = min(max(b.occ[h], 0), b.M_max);
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < m; i += gridDim.x * blockDim.x)
+    w.invb[(int64_t)h * w.invb_stride + i] = __frcp_rn(b.base[(int64_t)h * b.M_max + i]);
 }
 
 // Keys of the surviving states (rows of Eq. C.4's subtraction) and of the evicted
@@ -637,12 +697,17 @@ cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cud
   return cudaGetLastError();
 }
 
+cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s) {
+  dim3 grid((b.M_max + 255) / 256, b.H);
+  k_inv_base<<<grid, 256, 0, s>>>(b, w);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
-  int n = 256;
-  while (n < b.n_max) n <<= 1;
+  const int max_runs = (b.n_max + RUN - 1) / RUN;
   timer_begin(t, "sort", s);
-  if (n <= 8192) k_sort<8><<<b.H, BIG, (size_t)n * 16, s>>>(w, b.n_max);   // two merge buffers
-  else k_sort<16><<<b.H, BIG, (size_t)n * 8, s>>>(w, b.n_max);
+  k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max);
+  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(w, b.n_max);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -656,11 +721,8 @@ cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cu
 }
 
 cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  timer_begin(t, "rstar_head", s);
-  k_rstar_head<<<b.H, BIG, 0, s>>>(w);
-  timer_end(t, s);
-  timer_begin(t, "rstar_layer", s);
-  k_rstar_layer<<<1, BIG, 0, s>>>(b, w, kp.sync_heads);
+  timer_begin(t, "rstar", s);
+  k_rstar<<<b.H, BIG, 0, s>>>(b, w, kp.sync_heads);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -689,9 +751,8 @@ cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cud
 }
 
 cudaError_t update_set_smem_limits() {
-  cudaError_t e = cudaFuncSetAttribute(k_sort<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 8192 * 16);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_sort<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8);
-  return e;
+  // phase 2 of the sort holds every run of a head: up to 64 runs of 2 KiB
+  return cudaFuncSetAttribute(k_sort_rank, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * RUN * 8);
 }
 
 }  // namespace dkv
