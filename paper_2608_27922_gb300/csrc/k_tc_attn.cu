@@ -60,6 +60,36 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Row maximum accumulation over 32 scores (t: eight partial maxima).
+__device__ __forceinline__ void max_acc(float (&t)[8], const float (&v)[32]) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k) t[k & 7] = max3(t[k & 7], v[2 * k], v[2 * k + 1]);
+}
+
+// Scores of the columns at or past `lim` (keys past the end of the range) become -inf:
+// they do not raise the maximum and their exponentials are exactly 0.
+__device__ __forceinline__ void mask_tail(float (&v)[32], int lim) {
+#pragma unroll
+  for (int k = 0; k < 32; ++k)
+    if (k >= lim) v[k] = -INFINITY;
+}
+
+// P = 2^(s sl2 - m) over 64 scores (a: the first 32, b: the next 32) as 32 packed bf16
+// pairs; lab accumulates the even and the odd columns.
+__device__ __forceinline__ void exp_pack(const float (&a)[32], const float (&b)[32], float sl2, float nm,
+                                         float2& lab, uint32_t (&pk)[32]) {
+  const float2 sl2x2 = make_float2(sl2, sl2), nmx2 = make_float2(nm, nm);
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    const float s0 = k < 16 ? a[2 * k] : b[2 * k - 32];
+    const float s1 = k < 16 ? a[2 * k + 1] : b[2 * k - 31];
+    const float2 x = __ffma2_rn(make_float2(s0, s1), sl2x2, nmx2);
+    const float2 pp = make_float2(ex2(x.x), ex2(x.y));
+    lab = __fadd2_rn(lab, pp);
+    pk[k] = pack_bf16(pp.x, pp.y);
+  }
+}
+
 struct AttnJob {
   Bank b;
   DevLayer* L;   // sticky error word
@@ -232,26 +262,23 @@ __global__ void __launch_bounds__(THREADS, 1)
       ok = ok && __all_sync(0xffffffffu, mbar_wait(s_full + g, i & 1, abort_flag));
       if (!ok) break;
       fence_after_sync();
-      // pass 1: row maximum of the raw scores (masking only on a partial last tile)
+      // the whole row of S_g (128 scores) in registers: four loads, one wait
+      float s0[32], s1[32], s2[32], s3[32];
+      tmem_ld32(sc, s0);
+      tmem_ld32(sc + 32, s1);
+      tmem_ld32(sc + 64, s2);
+      tmem_ld32(sc + 96, s3);
+      tmem_wait_ld();
+      if (valid < BK) {   // partial last tile of the bank or of the window
+        mask_tail(s0, valid); mask_tail(s1, valid - 32); mask_tail(s2, valid - 64); mask_tail(s3, valid - 96);
+      }
+      // row maximum of the raw scores
       float tmax;
       {
         float t[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) t[k] = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sc + c * 32, v);
-          tmem_wait_ld();
-          if (valid == BK) {
-#pragma unroll
-            for (int k = 0; k < 16; ++k) t[k & 7] = max3(t[k & 7], v[2 * k], v[2 * k + 1]);
-          } else {
-#pragma unroll
-            for (int k = 0; k < 32; ++k)
-              if (c * 32 + k < valid) t[k & 7] = fmaxf(t[k & 7], v[k]);
-          }
-        }
+        max_acc(t, s0); max_acc(t, s1); max_acc(t, s2); max_acc(t, s3);
         tmax = fmaxf(fmaxf(fmaxf(t[0], t[1]), fmaxf(t[2], t[3])), fmaxf(fmaxf(t[4], t[5]), fmaxf(t[6], t[7])));
       }
       tmax *= j.sl2;
@@ -259,8 +286,24 @@ __global__ void __launch_bounds__(THREADS, 1)
       // (one thread issues both, in order), so O_g is idle here.
       const bool raise = tmax > mrun + RESCALE_LOG2;
       const float mnew = raise ? tmax : mrun;
+      const float mprev = mrun;
+      if (raise) {
+        l *= (i > 0) ? ex2(mrun - mnew) : 0.f;
+        mrun = mnew;
+      }
+      // P_g = 2^(s log2(e)/sqrt(d) - m) as packed bf16 pairs over the first 64 columns of S_g
+      const float nm = -mrun;
+      float2 lab = make_float2(0.f, 0.f);     // running sums of the even and odd columns
+      {
+        uint32_t pk[32];
+        exp_pack(s0, s1, j.sl2, nm, lab, pk);
+        tmem_st32(sc, pk);
+        exp_pack(s2, s3, j.sl2, nm, lab, pk);
+        tmem_st32(sc + 32, pk);
+      }
+      // O_g rescale: after the P stores (S is dead), before PV(i) is released
       if (__any_sync(0xffffffffu, raise && i > 0)) {
-        const float alpha = raise ? ex2(mrun - mnew) : 1.0f;
+        const float alpha = raise ? ex2(mprev - mnew) : 1.0f;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           float v[32];
@@ -275,49 +318,6 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tmem_st32(oc + c * 32, w32);
         }
-      }
-      if (raise) {
-        l *= (i > 0) ? ex2(mrun - mnew) : 0.f;
-        mrun = mnew;
-      }
-      // P_g = 2^(s log2(e)/sqrt(d) - m) as packed bf16 pairs over the first 64 columns of S_g
-      const float nm = -mrun;
-      const float2 sl2x2 = make_float2(j.sl2, j.sl2), nmx2 = make_float2(nm, nm);
-      float2 lab = make_float2(0.f, 0.f);     // running sums of the even and odd columns
-      // pass 2: exponentials, 64 scores at a time
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        float sv[64];
-        {
-          float v[32];
-          tmem_ld32(sc + c * 64, v);
-#pragma unroll
-          for (int k = 0; k < 32; ++k) sv[k] = v[k];
-          tmem_ld32(sc + c * 64 + 32, v);
-#pragma unroll
-          for (int k = 0; k < 32; ++k) sv[32 + k] = v[k];
-          tmem_wait_ld();
-        }
-        uint32_t pk[32];
-        if (valid == BK) {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const float2 x = __ffma2_rn(make_float2(sv[2 * k], sv[2 * k + 1]), sl2x2, nmx2);
-            const float2 pp = make_float2(ex2(x.x), ex2(x.y));
-            lab = __fadd2_rn(lab, pp);
-            pk[k] = pack_bf16(pp.x, pp.y);
-          }
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const int c0 = c * 64 + 2 * k;
-            const float p0 = c0 < valid ? ex2(fmaf(sv[2 * k], j.sl2, nm)) : 0.f;
-            const float p1 = c0 + 1 < valid ? ex2(fmaf(sv[2 * k + 1], j.sl2, nm)) : 0.f;
-            lab = __fadd2_rn(lab, make_float2(p0, p1));
-            pk[k] = pack_bf16(p0, p1);
-          }
-        }
-        tmem_st32(sc + c * 32, pk);
       }
       l += lab.x + lab.y;
       tmem_wait_st();
