@@ -23,15 +23,29 @@ constexpr int BIG = 1024;   // threads of the one-block-per-head kernels
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 
-// Row copies as a flat loop over 16-byte chunks: a row of RB key bytes plus its 64-byte
-// extension row is RB/16 + 4 chunks; consecutive threads take consecutive chunks.
-template <typename RowMap>
-__device__ __forceinline__ void copy_rows(int nrows, int rb, RowMap map) {
-  const int per = rb / 16 + 4;
-  const int total = nrows * per;
+// Row copies as a flat loop over groups of four 16-byte chunks (64 bytes) of a row.
+// Every row is a whole number of groups and no group spans two sources, so a thread
+// resolves its row once and has four independent loads in flight before its stores.
+// map(row, group) returns the group's source and destination (src == nullptr: nothing
+// to copy) and performs the row's scalar updates for one of its groups.
+struct Group4 {
+  const uint4* src;
+  uint4* dst;
+};
+
+template <typename Map>
+__device__ __forceinline__ void copy_groups(int nrows, int per_row, Map map) {
+  const int total = nrows * per_row;
   for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
-    const int row = c / per, part = c - row * per;
-    map(row, part, per - 4);
+    const int row = c / per_row, grp = c - row * per_row;
+    const Group4 g = map(row, grp);
+    if (g.src) {
+      uint4 v[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) v[k] = g.src[k];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) g.dst[k] = v[k];
+    }
   }
 }
 
@@ -70,38 +84,74 @@ __device__ __forceinline__ void split3(float x, __nv_bfloat16& hi, __nv_bfloat16
   lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
 }
 
+// Sum of squares of the pl (2 or 4) consecutive elements at p, one vector load.
+template <typename T>
+__device__ __forceinline__ float sq_sum(const T* p, int pl) {
+  float x[4];
+  if constexpr (sizeof(T) == 2) {
+    if (pl == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(p);
+      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+      const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+      x[0] = __low2float(a); x[1] = __high2float(a); x[2] = __low2float(c); x[3] = __high2float(c);
+    } else {
+      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(p);
+      x[0] = __low2float(a); x[1] = __high2float(a); x[2] = 0.f; x[3] = 0.f;
+    }
+  } else {
+    if (pl == 4) {
+      const float4 f = *reinterpret_cast<const float4*>(p);
+      x[0] = f.x; x[1] = f.y; x[2] = f.z; x[3] = f.w;
+    } else {
+      const float2 f = *reinterpret_cast<const float2*>(p);
+      x[0] = f.x; x[1] = f.y; x[2] = 0.f; x[3] = 0.f;
+    }
+  }
+  return fmaf(x[3], x[3], fmaf(x[2], x[2], fmaf(x[1], x[1], x[0] * x[0])));
+}
+
 // ||k||^2 per row and, if ext != nullptr, the row's 32 extension values used by the
 // tensor-core passes: row form [-g_hi, -g_mid, -g_lo, 1, 1, 1, 0 x 10] and column form
 // [1, 1, 1, -h_hi, -h_mid, -h_lo, 0 x 10], g = |k|^2 / 2 + goff, h = |k|^2 / 2.
+// A warp takes NR_ROWS rows (lane = d / 32 consecutive elements of each, one vector load),
+// with all loads issued before the reductions.
+constexpr int NR_ROWS = 4;
+
 template <typename T>
 __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
                             int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d,
                             __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
   const int h = blockIdx.y;
-  const int row = blockIdx.x * (blockDim.x / 32) + warp_id();
-  const int n = count_is_occ ? count[h] : N;
-  if (row < 0 || row >= n || row >= rows_cap) return;
-  const T* r = K + (int64_t)h * head_stride + (int64_t)row * d;
-  float a = 0.f;
-  for (int k = lane_id(); k < d; k += 32) {
-    const float x = to_f<T>(r[k]);
-    a = fmaf(x, x, a);
-  }
+  const int row0 = (blockIdx.x * (blockDim.x / 32) + warp_id()) * NR_ROWS;
+  const int n = min(count_is_occ ? count[h] : N, rows_cap);
+  if (row0 >= n) return;
+  const int pl = d / 32;
+  const int l = lane_id();
+  float a[NR_ROWS];
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-  if (lane_id() == 0) out[(int64_t)h * out_hs + row] = a;
-  if (ext) {
-    __nv_bfloat16 g[3], hh[3];
-    split3(-(0.5f * a + goff), g[0], g[1], g[2]);
-    split3(-(0.5f * a), hh[0], hh[1], hh[2]);
-    const int l = lane_id();
-    const __nv_bfloat16 one = __float2bfloat16_rn(1.0f), zero = __float2bfloat16_rn(0.0f);
-    __nv_bfloat16 v = zero;
-    if (l < 3) v = g[l];
-    else if (l < 6) v = one;
-    else if (l >= 16 && l < 19) v = one;
-    else if (l >= 19 && l < 22) v = hh[l - 19];
-    ext[(int64_t)h * ext_hs + (int64_t)row * 32 + l] = v;
+  for (int q = 0; q < NR_ROWS; ++q)
+    a[q] = row0 + q < n ? sq_sum<T>(K + (int64_t)h * head_stride + (int64_t)(row0 + q) * d + l * pl, pl) : 0.f;
+#pragma unroll
+  for (int q = 0; q < NR_ROWS; ++q)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a[q] += __shfl_xor_sync(0xffffffffu, a[q], o);
+#pragma unroll
+  for (int q = 0; q < NR_ROWS; ++q) {
+    const int row = row0 + q;
+    if (row >= n) break;
+    if (l == 0) out[(int64_t)h * out_hs + row] = a[q];
+    if (ext) {
+      __nv_bfloat16 g[3], hh[3];
+      split3(-(0.5f * a[q] + goff), g[0], g[1], g[2]);
+      split3(-(0.5f * a[q]), hh[0], hh[1], hh[2]);
+      const __nv_bfloat16 one = __float2bfloat16_rn(1.0f), zero = __float2bfloat16_rn(0.0f);
+      __nv_bfloat16 v = zero;
+      if (l < 3) v = g[l];
+      else if (l < 6) v = one;
+      else if (l >= 16 && l < 19) v = one;
+      else if (l >= 19 && l < 22) v = hh[l - 19];
+      ext[(int64_t)h * ext_hs + (int64_t)row * 32 + l] = v;
+    }
   }
 }
 
@@ -230,21 +280,19 @@ __global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int 
   const int rb = b.d * esize;
   const int64_t hn = (int64_t)h * b.n_max;
   const int32_t* perm = w.perm + hn;
-  copy_rows(N, rb, [&](int j, int part, int kparts) {
+  const int kg = rb / 64;                      // key groups; then one extension group
+  copy_groups(N, kg + 1, [&](int j, int grp) -> Group4 {
     const int src = perm[j];
     if (src < 0 || src >= N) {   // pi must be a permutation of [0, N)
-      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 8000 + h);
-      return;
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 8000 + h);
+      return {nullptr, nullptr};
     }
-    if (part < kparts) {
-      reinterpret_cast<uint4*>((char*)w.kperm + (hn + j) * rb)[part] =
-          reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb)[part];
-    } else {
-      const int e = part - kparts;
-      reinterpret_cast<uint4*>((char*)w.kperm_ext + (hn + j) * 64)[e] =
-          reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64)[e];
-      if (e == 0) w.kperm_norm[hn + j] = w.cnorm[hn + src];
-    }
+    if (grp < kg)
+      return {reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb) + 4 * grp,
+              reinterpret_cast<uint4*>((char*)w.kperm + (hn + j) * rb) + 4 * grp};
+    w.kperm_norm[hn + j] = w.cnorm[hn + src];
+    return {reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64),
+            reinterpret_cast<uint4*>((char*)w.kperm_ext + (hn + j) * 64)};
   });
 }
 
@@ -357,10 +405,17 @@ __device__ int block_scan_flag(int flag, int* s_warp, int* total) {
   const int within = __popc(bal & ((1u << lane_id()) - 1u));
   if (lane_id() == 0) s_warp[warp_id()] = __popc(bal);
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int run = 0;
-    for (int i = 0; i < (int)(blockDim.x / 32); ++i) { const int v = s_warp[i]; s_warp[i] = run; run += v; }
-    s_warp[32] = run;
+  if (warp_id() == 0) {   // exclusive scan of the warp counts by one warp
+    const int nw = (int)(blockDim.x / 32);
+    const int v = lane_id() < nw ? s_warp[lane_id()] : 0;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int x = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane_id() >= o) incl += x;
+    }
+    if (lane_id() < nw) s_warp[lane_id()] = incl - v;
+    if (lane_id() == 31) s_warp[32] = incl;
   }
   __syncthreads();
   const int off = s_warp[warp_id()] + within;
@@ -416,7 +471,16 @@ __device__ bool find_bin(const int* s_hist, unsigned kk, bool from_top, unsigned
   return true;
 }
 
+// Banks up to SEL_STAGE states are staged in shared memory for the select passes (sort
+// key of rho~ and a mandatory bit per state); larger ones are re-read from global memory.
+constexpr int SEL_STAGE = 40960;
+
+__host__ __device__ constexpr size_t sel_smem_bytes(int m_cap) {
+  return m_cap > SEL_STAGE ? 0 : (size_t)m_cap * 4 + ((size_t)m_cap + 31) / 32 * 4;
+}
+
 __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
+  extern __shared__ uint32_t s_stage[];   // [m] sort keys, then [(m + 31) / 32] mandatory bits
   __shared__ int s_hist[256];
   __shared__ int s_warp[33];
   __shared__ int s_cnt[2];
@@ -433,12 +497,23 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
   if (hd.empty) return;
   if (threadIdx.x == 0) { s_cnt[0] = 0; s_cnt[1] = 0; }
   __syncthreads();
-  // mandatory set and pre-violators
+  // mandatory set and pre-violators (and the shared-memory stage of keys and flags)
+  const bool staged = b.M_max <= SEL_STAGE;
+  uint32_t* skey = s_stage;
+  uint32_t* smand = s_stage + (staged ? b.M_max : 0);
   int nm = 0, npre = 0;
-  for (int i = threadIdx.x; i < m; i += blockDim.x) {
-    const int c = cross[i];
-    npre += (c == 0);
-    nm += (r > 0 && c <= r);
+  for (int base = 0; base < m; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    bool mand = false;
+    if (i < m) {
+      const int c = cross[i];
+      npre += (c == 0);
+      mand = r > 0 && c <= r;
+      nm += mand;
+      if (staged) skey[i] = fkey(rt[i]);
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, mand);
+    if (staged && lane_id() == 0 && i < m) smand[i >> 5] = bal;
   }
   nm = __reduce_add_sync(0xffffffffu, nm);
   npre = __reduce_add_sync(0xffffffffu, npre);
@@ -455,6 +530,10 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     return;
   }
   const int k = e - n_mand;   // states to evict by decreasing rho~(r)
+  auto is_mand = [&](int i) -> bool {
+    return staged ? ((smand[i >> 5] >> (i & 31)) & 1u) != 0u : (r > 0 && cross[i] <= r);
+  };
+  auto key_of = [&](int i) -> unsigned { return staged ? skey[i] : fkey(rt[i]); };
   // radix select of the k-th largest key among non-mandatory states
   unsigned prefix = 0, mask = 0;
   if (threadIdx.x == 0) { s_prefix = 0; s_kk = (unsigned)k; }
@@ -467,8 +546,8 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
         const int i = base + threadIdx.x;
         bool v = false;
         unsigned key = 0;
-        if (i < m && !(r > 0 && cross[i] <= r)) {
-          key = fkey(rt[i]);
+        if (i < m && !is_mand(i)) {
+          key = key_of(i);
           v = (key & mask) == prefix;
         }
         hist_add(s_hist, v, (key >> shift) & 255u);
@@ -493,7 +572,7 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
   int n_eq_local = 0;
   if (k > 0)
     for (int i = threadIdx.x; i < m; i += blockDim.x)
-      if (!(r > 0 && cross[i] <= r) && fkey(rt[i]) == T) ++n_eq_local;
+      if (!is_mand(i) && key_of(i) == T) ++n_eq_local;
   __syncthreads();
   if (threadIdx.x == 0) s_cnt[0] = 0;
   __syncthreads();
@@ -513,7 +592,7 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
         const int i = base + threadIdx.x;
         bool v = false;
         unsigned long long tk = 0;
-        if (i < m && !(r > 0 && cross[i] <= r) && fkey(rt[i]) == T) {
+        if (i < m && !is_mand(i) && key_of(i) == T) {
           tk = ((unsigned long long)(uint32_t)b.prov_step[bh + i] << 32) | (uint32_t)b.prov_src[bh + i];
           v = (tk & tmask) == tprefix;
         }
@@ -539,10 +618,10 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     const int i = base + threadIdx.x;
     int ev = 0;
     if (i < m) {
-      const bool mand = r > 0 && cross[i] <= r;
+      const bool mand = is_mand(i);
       if (mand) ev = 1;
       else if (k > 0) {
-        const unsigned key = fkey(rt[i]);
+        const unsigned key = key_of(i);
         if (key > T) ev = 1;
         else if (key == T) {
           if (!need_tie) ev = 1;
@@ -584,25 +663,23 @@ __global__ void k_gather(Bank b, Ws w, int esize) {
   const int64_t hn = (int64_t)h * b.n_max;
   const int ns = hd.m_old - hd.e;
   // rows [0, ns) survivors, [ns, ns + e) evicted
-  copy_rows(ns + hd.e, rb, [&](int row, int part, int kparts) {
+  const int kg = rb / 64;
+  copy_groups(ns + hd.e, kg + 1, [&](int row, int grp) -> Group4 {
     const bool surv = row < ns;
     const int slot = surv ? w.surv_list[bh + row] : w.evict_list[hn + row - ns];
     if (slot < 0 || slot >= hd.m_old) {
-      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
-      return;
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
+      return {nullptr, nullptr};
     }
-    char* dk = surv ? (char*)w.ksurv + (bh + row) * rb : (char*)w.kevict + (hn + row - ns) * rb;
+    if (grp < kg) {
+      char* dk = surv ? (char*)w.ksurv + (bh + row) * rb : (char*)w.kevict + (hn + row - ns) * rb;
+      return {reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb) + 4 * grp,
+              reinterpret_cast<uint4*>(dk) + 4 * grp};
+    }
+    if (surv) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
+    else w.kevict_norm[hn + row - ns] = b.knorm[bh + slot];
     char* dx = surv ? (char*)w.ksurv_ext + (bh + row) * 64 : (char*)w.kevict_ext + (hn + row - ns) * 64;
-    if (part < kparts) {
-      reinterpret_cast<uint4*>(dk)[part] = reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb)[part];
-    } else {
-      const int e = part - kparts;
-      reinterpret_cast<uint4*>(dx)[e] = reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64)[e];
-      if (e == 0) {
-        if (surv) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
-        else w.kevict_norm[hn + row - ns] = b.knorm[bh + slot];
-      }
-    }
+    return {reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64), reinterpret_cast<uint4*>(dx)};
   });
 }
 
@@ -620,40 +697,31 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
     if (m_new > hd.M) dev_fail(w.L, DEV_INCONSISTENT, 4000 + h);
   }
   const int rb = b.d * esize;
-  const int kp = rb / 16;
-  // per admitted row: key chunks, value chunks, then the 64-byte extension row
-  const int per = 2 * kp + 4;
-  const int total = hd.r * per;
-  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
-    const int j = c / per, part = c - j * per;
+  const int kg = rb / 64;   // per admitted row: key groups, value groups, one extension group
+  copy_groups(hd.r, 2 * kg + 1, [&](int j, int grp) -> Group4 {
     const int slot = j < hd.e ? w.evict_list[hn + j] : hd.m_old + (j - hd.e);
     if (slot < 0 || slot >= hd.M) {
-      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
-      continue;
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
+      return {nullptr, nullptr};
     }
     const int src = w.perm[hn + j];
     if (src < 0 || src >= N) {
-      if (part == 0) dev_fail(w.L, DEV_INCONSISTENT, 8500 + h);
-      continue;
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 8500 + h);
+      return {nullptr, nullptr};
     }
-    if (part < kp) {
-      reinterpret_cast<uint4*>((char*)b.k + (bh + slot) * rb)[part] =
-          reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb)[part];
-    } else if (part < 2 * kp) {
-      reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb)[part - kp] =
-          reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb)[part - kp];
-    } else {
-      const int e = part - 2 * kp;
-      reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64)[e] =
-          reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64)[e];
-      if (e == 0) {
-        b.knorm[bh + slot] = w.kperm_norm[hn + j];
-        b.prov_step[bh + slot] = w.L->step;
-        b.prov_src[bh + slot] = src;
-        w.slot_new[hn + j] = slot;
-      }
-    }
-  }
+    if (grp < kg)
+      return {reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb) + 4 * grp,
+              reinterpret_cast<uint4*>((char*)b.k + (bh + slot) * rb) + 4 * grp};
+    if (grp < 2 * kg)
+      return {reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg),
+              reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb) + 4 * (grp - kg)};
+    b.knorm[bh + slot] = w.kperm_norm[hn + j];
+    b.prov_step[bh + slot] = w.L->step;
+    b.prov_src[bh + slot] = src;
+    w.slot_new[hn + j] = slot;
+    return {reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64),
+            reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64)};
+  });
 }
 
 }  // namespace
@@ -669,7 +737,7 @@ static float ext_goff(const KParams& kp) { return kp.eps * 0.5f / kp.inv_s2; }  
 
 cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
                               Timer* t) {
-  dim3 grid((N + 7) / 8, b.H);
+  dim3 grid((N + 8 * NR_ROWS - 1) / (8 * NR_ROWS), b.H);
   __nv_bfloat16* ext = (__nv_bfloat16*)w.cext;
   timer_begin(t, "cand_norms", s);
   if (b.bf16)
@@ -683,7 +751,7 @@ cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N,
 }
 
 cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  dim3 grid((b.M_max + 7) / 8, b.H);
+  dim3 grid((b.M_max + 8 * NR_ROWS - 1) / (8 * NR_ROWS), b.H);
   __nv_bfloat16* ext = (__nv_bfloat16*)w.bext;
   timer_begin(t, "bank_norms", s);
   if (b.bf16)
@@ -713,7 +781,7 @@ cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
 }
 
 cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N * (b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
+  dim3 grid((N * (b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
   timer_begin(t, "permute", s);
   k_permute<<<grid, 256, 0, s>>>(b, w, (const char*)Kc, N, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -729,13 +797,13 @@ cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStre
 
 cudaError_t launch_select(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
   timer_begin(t, "select", s);
-  k_select<<<b.H, BIG, 0, s>>>(b, w);
+  k_select<<<b.H, BIG, sel_smem_bytes(b.M_max), s>>>(b, w);
   timer_end(t, s);
   return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
-  dim3 grid((b.M_max * (b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
+  dim3 grid((b.M_max * (b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
   timer_begin(t, "gather", s);
   k_gather<<<grid, 256, 0, s>>>(b, w, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -743,7 +811,7 @@ cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) 
 }
 
 cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N * (2 * b.d * (b.bf16 ? 2 : 4) / 16 + 4) + 255) / 256, b.H);
+  dim3 grid((N * (2 * b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
   timer_begin(t, "commit", s);
   k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4);
   timer_end(t, s);
@@ -752,7 +820,10 @@ cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cud
 
 cudaError_t update_set_smem_limits() {
   // phase 2 of the sort holds every run of a head: up to 64 runs of 2 KiB
-  return cudaFuncSetAttribute(k_sort_rank, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * RUN * 8);
+  cudaError_t e = cudaFuncSetAttribute(k_sort_rank, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * RUN * 8);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sel_smem_bytes(SEL_STAGE));
+  return e;
 }
 
 }  // namespace dkv
