@@ -48,6 +48,16 @@ the design notes of the repository):
   order) and does not take part in the shared prefix search.
 * sync_heads=False gives the "independent per-head prefix" ablation
   (App. E "Cross-head synchronization").
+* The other policy ablations of Table 2(b) / App. E, all on the same steps:
+  order="source" takes candidates in source order (pi = identity) instead of
+  ascending Eq. 6 scores; evict="densest" evicts the e_{r*} states of largest
+  rho~(r*) with no mandatory-first step; evict="mandatory_source" evicts the
+  threshold crossers first and fills the remaining slots in source order of
+  the bank, read as provenance order (oldest (step, src) first);
+  refresh_baselines=True sets b = max(rho, delta) for every retained state
+  after each update instead of keeping the insertion-time baseline.  In every
+  variant r* is still the largest prefix feasible under Eqs. 9-11 for the
+  candidates in the variant's order.
 """
 from __future__ import annotations
 
@@ -76,6 +86,9 @@ class Params:
     eps: float = 1.0          # regulariser
     delta: float = 1e-6       # baseline floor
     sync_heads: bool = True   # shared cross-head prefix (default policy)
+    order: str = "score"      # "score" (Eq. 6 ascending, default) or "source"
+    evict: str = "mandatory_densest"   # or "densest", "mandatory_source"
+    refresh_baselines: bool = False    # default: baselines frozen at insertion (Eq. 5)
 
     def sigma_for(self, d: int) -> float:
         return math.sqrt(d / 2.0) if self.sigma is None else float(self.sigma)
@@ -246,6 +259,8 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
     in source order.  ``step`` is recorded as the provenance of admitted states.
     ``literal=True`` recomputes every prefix sum from scratch (tiny inputs).
     """
+    assert prm.order in ("score", "source")
+    assert prm.evict in ("mandatory_densest", "densest", "mandatory_source")
     H = len(bank.heads)
     Kc = np.asarray(Kc, dtype=np.float64)
     Vc = np.asarray(Vc, dtype=np.float64)
@@ -271,8 +286,8 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
         # Eq. 6 / C.1: s_h(x) = (1/m) sum_i w(kbar_i, k_x) / b_i
         Wxb = soft_riesz(sq_dist(Kc[h], hb.K), prm, hb.d)              # [N, m]
         s = (Wxb / hb.base.astype(np.float64)[None, :]).sum(axis=1) / m
-        # stable ascending sort, ties broken by source order
-        pi = np.argsort(s, kind="stable")
+        # stable ascending sort, ties broken by source order (or source order itself)
+        pi = np.argsort(s, kind="stable") if prm.order == "score" else np.arange(N)
         Kc_pi = Kc[h][pi]
         if literal:
             rt = _prefix_rho_tilde_literal(hb, Kc_pi, prm, rmax)
@@ -310,11 +325,20 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
         mand = (g_r >= prm.tau) if r > 0 else np.zeros(m, bool)
         mand_idx = np.nonzero(mand)[0]
         assert mand_idx.shape[0] <= e_r, "feasibility violated"
-        rest = np.nonzero(~mand)[0]
-        # decreasing rho~(r*); ties: older provenance (smaller step, then src) first
-        order = np.lexsort((hb.src[rest], hb.step[rest], -rho_t[rest]))
-        fill = rest[order[:e_r - mand_idx.shape[0]]]
-        R = np.concatenate([mand_idx, fill]).astype(np.int64)
+        if prm.evict == "densest":
+            # the e_r largest rho~(r*) over the whole bank; ties: older provenance first
+            order = np.lexsort((hb.src, hb.step, -rho_t))
+            R = order[:e_r].astype(np.int64)
+        else:
+            rest = np.nonzero(~mand)[0]
+            if prm.evict == "mandatory_source":
+                # fill in source (provenance) order: oldest (step, src) first
+                order = np.lexsort((hb.src[rest], hb.step[rest]))
+            else:
+                # decreasing rho~(r*); ties: older provenance (smaller step, then src) first
+                order = np.lexsort((hb.src[rest], hb.step[rest], -rho_t[rest]))
+            fill = rest[order[:e_r - mand_idx.shape[0]]]
+            R = np.concatenate([mand_idx, fill]).astype(np.int64)
         keep = np.ones(m, bool)
         keep[R] = False
         adm = pi[:r]
@@ -339,7 +363,11 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
             rho_new = np.zeros(0)
         hb.K, hb.V = K_new, V_new
         hb.rho = np.concatenate([rho_surv, rho_new]).astype(hb.store)
-        hb.base = np.concatenate([hb.base[keep], np.maximum(rho_new, prm.delta)]).astype(hb.store)
+        if prm.refresh_baselines:
+            # every retained state's baseline follows its current (stored) density
+            hb.base = np.maximum(hb.rho.astype(np.float64), prm.delta).astype(hb.store)
+        else:
+            hb.base = np.concatenate([hb.base[keep], np.maximum(rho_new, prm.delta)]).astype(hb.store)
         hb.step = np.concatenate([hb.step[keep], np.full(r, step, np.int64)])
         hb.src = np.concatenate([hb.src[keep], adm.astype(np.int64)])
         recs[h] = HeadRecord(empty_init=False, s=s, pi=pi, counts=counts, e=e, cross=cross,

@@ -230,8 +230,11 @@ def _brute_update_decision(O, before, K, prm):
         hb = before.heads[h]
         s = prm.sigma_for(hb.d)
         w = lambda a, b: (prm.eps + float(np.sum((a - b) ** 2)) / (s * s)) ** (-prm.p)
-        score = [sum(w(hb.K[i], K[h][x]) / float(hb.base[i]) for i in range(hb.m)) / hb.m for x in range(N)]
-        pi = sorted(range(N), key=lambda x: (score[x], x))
+        if getattr(prm, "order", "score") == "source":
+            pi = list(range(N))
+        else:
+            score = [sum(w(hb.K[i], K[h][x]) / float(hb.base[i]) for i in range(hb.m)) / hb.m for x in range(N)]
+            pi = sorted(range(N), key=lambda x: (score[x], x))
         for r in range(rmax + 1):
             c = 0
             for i in range(hb.m):
@@ -437,6 +440,78 @@ def check_attention_textbook(O):
     assert np.allclose(O.attend(eb, Q, Kw, Vw), ref2, atol=1e-12)
 
 
+# --------------------------------------------------------------------------- P9: policy ablations
+def _expected_eviction(hr, hb0, e, evict):
+    """R re-derived with explicit sorts from rho~, the mandatory flags and provenance."""
+    idx = list(range(hb0.m))
+    prov = lambda i: (int(hb0.step[i]), int(hb0.src[i]))
+    if evict == "densest":
+        return sorted(idx, key=lambda i: (-float(hr.rho_tilde[i]), prov(i)))[:e]
+    mand = [i for i in idx if hr.mandatory[i]]
+    rest = [i for i in idx if not hr.mandatory[i]]
+    if evict == "mandatory_source":
+        rest = sorted(rest, key=prov)
+    else:
+        rest = sorted(rest, key=lambda i: (-float(hr.rho_tilde[i]), prov(i)))
+    return mand + rest[:e - len(mand)]
+
+
+def check_policy_variants(O):
+    """Table 2(b) / App. E ablations: source-order candidates, densest-only and
+    mandatory + source eviction, refreshed baselines (each alone and combined)."""
+    variants = [dict(order="source"), dict(evict="densest"), dict(evict="mandatory_source"),
+                dict(refresh_baselines=True), dict(order="source", evict="densest", refresh_baselines=True)]
+    for vi, kw in enumerate(variants):
+        for seed in range(3):
+            prm = _prm(O, sigma=1.0, p=2.0, tau=1.5, **kw)
+            for t, (before, K, V, rec, after) in enumerate(
+                    _random_bank_rollout(O, 500 + 10 * vi + seed, prm=prm, steps=5, M=10, N=7)):
+                r_bf = _brute_update_decision(O, before, K, prm)
+                if r_bf is not None:
+                    assert rec.r_star == r_bf, (kw, seed, t, rec.r_star, r_bf)
+                for h, (hb0, hb1, hr) in enumerate(zip(before.heads, after.heads, rec.heads)):
+                    assert hb1.m <= hb1.M
+                    if hb0.m == 0:
+                        continue
+                    if prm.order == "source":
+                        assert np.array_equal(hr.pi, np.arange(K.shape[1]))
+                    assert hr.admitted.tolist() == hr.pi[:rec.r_star].tolist()
+                    e = max(0, hb0.m + rec.r_star - hb0.M)
+                    assert sorted(hr.evicted.tolist()) == sorted(_expected_eviction(hr, hb0, e, prm.evict))
+                    phi = O.density(hb1.K, prm)
+                    assert np.allclose(hb1.rho, phi, rtol=1e-9, atol=1e-12)
+                    prov0 = {(int(a), int(b)): float(x) for a, b, x in zip(hb0.step, hb0.src, hb0.base)}
+                    for i, (a, b) in enumerate(zip(hb1.step, hb1.src)):
+                        if prm.refresh_baselines:
+                            assert float(hb1.base[i]) == max(float(hb1.rho[i]), prm.delta)
+                        elif (int(a), int(b)) in prov0:
+                            assert float(hb1.base[i]) == prov0[(int(a), int(b))]
+
+    # Densest-only eviction can keep a threshold crosser that the default evicts: an isolated
+    # state with a tiny baseline (g >= tau) next to a dense pair, one candidate far away.
+    d = 2
+    Kb = np.array([[10.0, 0.0], [0.0, 0.0], [0.1, 0.0]])
+    prm0 = _prm(O, sigma=1.0, p=2.0, tau=2.0)
+    rho = O.density(Kb, prm0)
+    base = rho.copy()
+    base[0] = rho[0] / 4.0                         # g_0(0) = 4 >= tau
+    Kc = np.array([[[-50.0, 0.0]]])
+    Vc = np.zeros((1, 1, d))
+    outs = {}
+    for ev in ("mandatory_densest", "densest"):
+        prm = _prm(O, sigma=1.0, p=2.0, tau=2.0, evict=ev)
+        bank = O.LayerBank.empty([3], d, store=np.float64)
+        hb = bank.heads[0]
+        hb.K, hb.V = Kb.copy(), np.zeros((3, d))
+        hb.rho, hb.base = rho.copy(), base.copy()
+        hb.step, hb.src = np.zeros(3, np.int64), np.arange(3, dtype=np.int64)
+        rec = O.update_layer(bank, Kc, Vc, step=1, prm=prm)
+        assert rec.r_star == 1
+        outs[ev] = sorted(rec.heads[0].evicted.tolist())
+    assert outs["mandatory_densest"] == [0]        # the crosser goes first
+    assert outs["densest"] in ([1], [2])           # the densest of the pair instead
+
+
 ALL_CHECKS = [
     check_kernel_closed_forms,
     check_distance_identities,
@@ -449,4 +524,5 @@ ALL_CHECKS = [
     check_shared_prefix_across_heads,
     check_storage_accounting,
     check_attention_textbook,
+    check_policy_variants,
 ]

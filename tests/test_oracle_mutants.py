@@ -63,6 +63,13 @@ MUTANTS = [
     ("attn_drops_window", "Kall = np.concatenate([hb.K, np.asarray(Kw, dtype=np.float64)], axis=0)",
      "Kall = np.concatenate([hb.K, 0.0 * np.asarray(Kw, dtype=np.float64)], axis=0)"),
     ("storage_meta", "meta_bytes: int = 4 + 4 + 8 + 4", "meta_bytes: int = 4 + 4 + 4 + 4"),
+    ("densest_ascending", "order = np.lexsort((hb.src, hb.step, -rho_t))",
+     "order = np.lexsort((hb.src, hb.step, rho_t))"),
+    ("source_fill_newest_first", "order = np.lexsort((hb.src[rest], hb.step[rest]))\n",
+     "order = np.lexsort((-hb.src[rest], -hb.step[rest]))\n"),
+    ("refresh_ignored", "if prm.refresh_baselines:\n", "if False:\n"),
+    ("source_order_ignored", 'if prm.order == "score" else np.arange(N)', 'if True else np.arange(N)'),
+    ("densest_keeps_mandatory_first", 'if prm.evict == "densest":', 'if prm.evict == "never":'),
 ]
 
 
