@@ -56,6 +56,11 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="wan13b_layer_h12")
     ap.add_argument("--score-mode", choices=["tensor", "fp32"], default="tensor")
+    ap.add_argument("--order", choices=["score", "source"], default="score",
+                    help="candidate order (policy ablation of Table 2(b); default: the method's)")
+    ap.add_argument("--eviction", choices=["mandatory_densest", "densest", "mandatory_source"],
+                    default="mandatory_densest", help="eviction rule (policy ablation)")
+    ap.add_argument("--refresh-baselines", action="store_true", help="refresh b after every update (ablation)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -211,7 +216,12 @@ def run_ours(args):
     dblocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
     dq = [torch.from_numpy(q).to(dev, bf) for q in inp.queries[:W + K]]
     mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
-    bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(layer), wl.N, bf, score_mode=mode, device=dev)
+    policy = dict(order={"score": dkv.DKV_ORDER_SCORE, "source": dkv.DKV_ORDER_SOURCE}[args.order],
+                  eviction={"mandatory_densest": dkv.DKV_EVICT_MANDATORY_DENSEST, "densest": dkv.DKV_EVICT_DENSEST,
+                            "mandatory_source": dkv.DKV_EVICT_MANDATORY_SOURCE}[args.eviction],
+                  refresh_baselines=int(args.refresh_baselines))
+    bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(layer), wl.N, bf, score_mode=mode, device=dev,
+                         **policy)
     bank.reset()
     out = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
@@ -469,6 +479,8 @@ def run_ours(args):
             "config": {"workload": f"{wl.name}: {wl.L if world > 1 else 1} layer(s) x {wl.H} heads, d={wl.d}, "
                                    f"N={wl.N}, M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
                        "score_mode": args.score_mode, "layers_per_gpu": 1,
+                       "policy": {"order": args.order, "eviction": args.eviction,
+                                  "refresh_baselines": bool(args.refresh_baselines)},
                        "streams": "attention || admit, then compress" if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",

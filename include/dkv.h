@@ -80,6 +80,20 @@ typedef enum { DKV_DTYPE_BF16 = 0, DKV_DTYPE_FP32 = 1 } dkv_dtype_t;
  *                   (the exactness mode; required for fp32 banks).           */
 typedef enum { DKV_SCORE_TENSOR = 0, DKV_SCORE_FP32 = 1 } dkv_score_mode_t;
 
+/* Update policy (Table 2(b) and App. E "Policy ablations"; the defaults are the
+ * paper's method).  Candidate order: ascending Eq. 6 score (default) or source
+ * order of the block (pi = identity; no score pass).  Eviction (Sec. 3.4 Step 3):
+ * threshold crossers first, then decreasing rho~(r*) (default); only decreasing
+ * rho~(r*) ("densest-only"); or threshold crossers first, then source order of the
+ * bank, read as provenance order, oldest (step, src) first.  In every policy r* is
+ * the largest prefix feasible under Eqs. 9-11 for the candidates in that order.    */
+typedef enum { DKV_ORDER_SCORE = 0, DKV_ORDER_SOURCE = 1 } dkv_order_t;
+typedef enum {
+  DKV_EVICT_MANDATORY_DENSEST = 0,
+  DKV_EVICT_DENSEST = 1,
+  DKV_EVICT_MANDATORY_SOURCE = 2
+} dkv_evict_t;
+
 /* Method parameters.  Defaults (dkv_params_default): tau = 2, sigma = sqrt(d/2),
  * p = 2, eps = 1, delta = 1e-6, shared cross-head prefix (Sec. 4.1; App. B
  * "Parameterization"; App. D "Default DensityKV configuration").           */
@@ -92,6 +106,11 @@ typedef struct {
   int32_t sync_heads;   /* 1: one prefix length r* for all heads (Eq. 11);
                            0: each head its own largest feasible prefix (App. E)      */
   int32_t score_mode;   /* dkv_score_mode_t                                            */
+  int32_t order;        /* dkv_order_t                                                 */
+  int32_t eviction;     /* dkv_evict_t                                                 */
+  int32_t refresh_baselines; /* 0: baselines frozen at insertion (Eq. 5, default);
+                           1: b = max(rho, delta) for every retained state after each
+                           update (App. E "Density baseline" ablation)              */
   int32_t reserved;     /* must be 0                                                   */
 } dkv_params_t;
 

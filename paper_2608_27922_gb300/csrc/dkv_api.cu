@@ -198,7 +198,7 @@ const char* dkv_status_str(dkv_status_t s) {
   return "unknown status";
 }
 
-int32_t dkv_version(void) { return 100; }
+int32_t dkv_version(void) { return 110; }
 
 dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   if (!out || d <= 0) return DKV_ERR_ARG;
@@ -209,6 +209,9 @@ dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   out->delta = 1e-6f;
   out->sync_heads = 1;
   out->score_mode = DKV_SCORE_TENSOR;
+  out->order = DKV_ORDER_SCORE;
+  out->eviction = DKV_EVICT_MANDATORY_DENSEST;
+  out->refresh_baselines = 0;
   out->reserved = 0;
   return DKV_OK;
 }
@@ -234,6 +237,10 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   if (!(p.tau > 1.0f) || !(p.eps > 0.0f) || !(p.delta > 0.0f) || !(p.sigma >= 0.0f) ||
       !(p.p == 1.0f || p.p == 2.0f || p.p == 4.0f) || (p.sync_heads != 0 && p.sync_heads != 1) ||
       (p.score_mode != DKV_SCORE_TENSOR && p.score_mode != DKV_SCORE_FP32) || p.reserved != 0 ||
+      (p.order != DKV_ORDER_SCORE && p.order != DKV_ORDER_SOURCE) ||
+      (p.eviction != DKV_EVICT_MANDATORY_DENSEST && p.eviction != DKV_EVICT_DENSEST &&
+       p.eviction != DKV_EVICT_MANDATORY_SOURCE) ||
+      (p.refresh_baselines != 0 && p.refresh_baselines != 1) ||
       !std::isfinite(p.tau) || !std::isfinite(p.sigma) || !std::isfinite(p.eps) || !std::isfinite(p.delta))
     return DKV_ERR_ARG;
   int M_max = 0;
@@ -282,6 +289,9 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   bk->kp.delta = p.delta;
   bk->kp.p = (int)p.p;
   bk->kp.sync_heads = p.sync_heads;
+  bk->kp.order = p.order;
+  bk->kp.eviction = p.eviction;
+  bk->kp.refresh = p.refresh_baselines;
   // workspace header: zeroed layer state and the per-head budgets (one-time, synchronous)
   cudaError_t e = cudaMemset(bk->w.L, 0, sizeof(DevLayer));
   if (e == cudaSuccess) e = cudaMemset(bk->w.hd, 0, sizeof(DevHead) * H);
@@ -321,8 +331,9 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   if (e == cudaSuccess) e = launch_prepare(b, w, N, step, s, t);
   if (e == cudaSuccess) e = launch_cand_norms(b, w, Kc, N, bank->kp, s, t);
   if (e == cudaSuccess)
-    e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
-  if (e == cudaSuccess) e = launch_sort(b, w, s, t);
+    if (bank->kp.order == DKV_ORDER_SCORE)   // source order needs no scores (App. E)
+      e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
+  if (e == cudaSuccess) e = launch_sort(b, w, bank->kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = launch_permute(b, w, Kc, N, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_cross_tc(b, w, bank->kp, s, t) : launch_cross_fp32(b, w, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_rstar(b, w, bank->kp, s, t);
@@ -346,7 +357,7 @@ dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream) {
   bank->last = s;
   bank->state = 0;
   cudaError_t e = bank->tc ? launch_project_tc(b, w, kp, s, t) : launch_project_fp32(b, w, kp, s, t);
-  if (e == cudaSuccess) e = launch_select(b, w, s, t);
+  if (e == cudaSuccess) e = launch_select(b, w, kp.eviction, s, t);
   if (e == cudaSuccess) e = launch_gather(b, w, s, t);
   if (e == cudaSuccess) e = launch_commit(b, w, bank->Vc, bank->N, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_subtract_tc(b, w, kp, s, t) : launch_subtract_fp32(b, w, kp, s, t);

@@ -48,6 +48,9 @@ struct KParams {
   float delta;
   int32_t p;         // 1, 2 or 4
   int32_t sync_heads;
+  int32_t order;     // dkv_order_t
+  int32_t eviction;  // dkv_evict_t
+  int32_t refresh;   // 1: b = max(rho, delta) for every retained state after each update
 };
 
 // Snapshots of the running prefix sum of Eq. C.2 are kept every SNAP columns.

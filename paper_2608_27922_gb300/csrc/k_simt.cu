@@ -134,7 +134,13 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
   } else if (MODE == PM_PROJECT) {
     j.w.rho_t[bh + row] = S;
   } else if (MODE == PM_SUB) {
-    j.b.rho[bh + slot] = __fsub_rn(j.w.rho_t[bh + slot], acc);
+    const float rho = __fsub_rn(j.w.rho_t[bh + slot], acc);
+    j.b.rho[bh + slot] = rho;
+    if (j.kp.refresh) {   // refreshed-baseline policy: b follows the current density
+      const float bnew = fmaxf(rho, j.kp.delta);
+      j.b.base[bh + slot] = bnew;
+      j.w.invb[(int64_t)h * j.w.invb_stride + slot] = __frcp_rn(bnew);
+    }
   } else {
     j.b.rho[bh + self] = S;
     const float bnew = fmaxf(S, j.kp.delta);

@@ -485,8 +485,17 @@ __global__ void __launch_bounds__(THREADS, 2)
         j.w.rho_t[bh + row] = fmaf(c, S, j.b.rho[bh + row]);
       } else if (MODE == TM_SUB) {
         const int slot = hd.e == 0 ? row : j.w.surv_list[bh + row];
-        if (slot >= 0 && slot < hd.m_old) j.b.rho[bh + slot] = fmaf(-c, acc, j.w.rho_t[bh + slot]);
-        else dev_fail(j.w.L, DEV_INCONSISTENT, 6003);
+        if (slot >= 0 && slot < hd.m_old) {
+          const float rho = fmaf(-c, acc, j.w.rho_t[bh + slot]);
+          j.b.rho[bh + slot] = rho;
+          if (kp.refresh) {   // refreshed-baseline policy: b follows the current density
+            const float bnew = fmaxf(rho, kp.delta);
+            j.b.base[bh + slot] = bnew;
+            j.w.invb[(int64_t)h * j.w.invb_stride + slot] = __frcp_rn(bnew);
+          }
+        } else {
+          dev_fail(j.w.L, DEV_INCONSISTENT, 6003);
+        }
       } else {
         if (self >= 0 && self < hd.M) {
           const float rho = c * acc;

@@ -10,6 +10,7 @@
 //                radix select on the fp32 bit patterns; ties evict the older state
 //   gather       keys of the surviving and of the evicted states (operands of Eq. C.4)
 //   commit       Eq. 12: admitted keys/values into the evicted slots, the rest appended
+#include "dkv.h"
 #include "dkv_internal.h"
 
 #include <climits>
@@ -202,10 +203,11 @@ __device__ __forceinline__ void cas_shfl(unsigned long long (&x)[SKPT], int t, i
 // Phase 1: warp w of block x sorts run a = 8 x + w (source indices [256 a, 256 a + 256),
 // padded with ~0) ascending; the direction bit is taken from the run-local index, so
 // every run comes out ascending.
-__global__ void __launch_bounds__(256) k_sort_runs(Ws w, int n_max) {
+__global__ void __launch_bounds__(256) k_sort_runs(Ws w, int n_max, int identity) {
   const int h = blockIdx.y;
   const int N = w.L->N;
-  if (w.hd[h].empty) {   // empty bank: source order (Alg. 1, m = 0 branch)
+  // empty bank: source order (Alg. 1, m = 0 branch); source-order policy: the same
+  if (w.hd[h].empty || identity) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x)
       w.perm[(int64_t)h * n_max + i] = i;
     return;
@@ -243,11 +245,11 @@ __device__ __forceinline__ int run_rank(const unsigned long long* r, unsigned lo
 // Phase 2: block (a, h) places the keys of run a: final position = index in run a plus
 // the number of smaller keys in every other run (keys are unique, so positions are
 // distinct and cover [0, N)).
-__global__ void __launch_bounds__(RUN) k_sort_rank(Ws w, int n_max) {
+__global__ void __launch_bounds__(RUN) k_sort_rank(Ws w, int n_max, int identity) {
   extern __shared__ unsigned long long runs[];
   const int h = blockIdx.y;
   const int N = w.L->N;
-  if (w.hd[h].empty) return;
+  if (w.hd[h].empty || identity) return;
   const int nruns = (N + RUN - 1) / RUN;
   const int a = blockIdx.x;
   if (a >= nruns) return;                         // block-uniform
@@ -479,7 +481,7 @@ __host__ __device__ constexpr size_t sel_smem_bytes(int m_cap) {
   return m_cap > SEL_STAGE ? 0 : (size_t)m_cap * 4 + ((size_t)m_cap + 31) / 32 * 4;
 }
 
-__global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
+__global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w, int eviction) {
   extern __shared__ uint32_t s_stage[];   // [m] sort keys, then [(m + 31) / 32] mandatory bits
   __shared__ int s_hist[256];
   __shared__ int s_warp[33];
@@ -529,11 +531,18 @@ __global__ void __launch_bounds__(BIG) k_select(Bank b, Ws w) {
     if (threadIdx.x == 0) dev_fail(w.L, DEV_INCONSISTENT, 2000 + h);
     return;
   }
-  const int k = e - n_mand;   // states to evict by decreasing rho~(r)
+  // Eviction policy: threshold crossers first (default and mandatory + source), or none
+  // (densest-only); the rest by decreasing rho~(r) or, for mandatory + source, in
+  // provenance order: every key ties, so the provenance selection below takes the oldest.
+  const bool mand_first = eviction != DKV_EVICT_DENSEST;
+  const bool by_source = eviction == DKV_EVICT_MANDATORY_SOURCE;
+  if (!mand_first) n_mand = 0;
+  const int k = e - n_mand;   // states to evict after the mandatory ones
   auto is_mand = [&](int i) -> bool {
+    if (!mand_first) return false;
     return staged ? ((smand[i >> 5] >> (i & 31)) & 1u) != 0u : (r > 0 && cross[i] <= r);
   };
-  auto key_of = [&](int i) -> unsigned { return staged ? skey[i] : fkey(rt[i]); };
+  auto key_of = [&](int i) -> unsigned { return by_source ? 0u : (staged ? skey[i] : fkey(rt[i])); };
   // radix select of the k-th largest key among non-mandatory states
   unsigned prefix = 0, mask = 0;
   if (threadIdx.x == 0) { s_prefix = 0; s_kk = (unsigned)k; }
@@ -771,11 +780,11 @@ cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_sort(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
+cudaError_t launch_sort(const Bank& b, const Ws& w, int identity, cudaStream_t s, Timer* t) {
   const int max_runs = (b.n_max + RUN - 1) / RUN;
   timer_begin(t, "sort", s);
-  k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max);
-  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(w, b.n_max);
+  k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max, identity);
+  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(w, b.n_max, identity);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -795,9 +804,9 @@ cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStre
   return cudaGetLastError();
 }
 
-cudaError_t launch_select(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
+cudaError_t launch_select(const Bank& b, const Ws& w, int eviction, cudaStream_t s, Timer* t) {
   timer_begin(t, "select", s);
-  k_select<<<b.H, BIG, sel_smem_bytes(b.M_max), s>>>(b, w);
+  k_select<<<b.H, BIG, sel_smem_bytes(b.M_max), s>>>(b, w, eviction);
   timer_end(t, s);
   return cudaGetLastError();
 }

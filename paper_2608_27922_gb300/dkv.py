@@ -22,6 +22,8 @@ LIB_PATH = os.path.join(_PKG, "lib", "libdkv.so")
 DKV_OK = 0
 DKV_DTYPE_BF16, DKV_DTYPE_FP32 = 0, 1
 DKV_SCORE_TENSOR, DKV_SCORE_FP32 = 0, 1
+DKV_ORDER_SCORE, DKV_ORDER_SOURCE = 0, 1
+DKV_EVICT_MANDATORY_DENSEST, DKV_EVICT_DENSEST, DKV_EVICT_MANDATORY_SOURCE = 0, 1, 2
 STATUS = {0: "DKV_OK", 1: "DKV_ERR_ARG", 2: "DKV_ERR_SHAPE", 3: "DKV_ERR_STATE", 4: "DKV_ERR_CUDA",
           5: "DKV_ERR_NOMEM", 6: "DKV_ERR_TIMEOUT", 7: "DKV_ERR_UNSUPPORTED", 8: "DKV_ERR_DEVICE"}
 
@@ -29,7 +31,8 @@ STATUS = {0: "DKV_OK", 1: "DKV_ERR_ARG", 2: "DKV_ERR_SHAPE", 3: "DKV_ERR_STATE",
 class dkv_params_t(ctypes.Structure):
     _fields_ = [("tau", ctypes.c_float), ("sigma", ctypes.c_float), ("p", ctypes.c_float),
                 ("eps", ctypes.c_float), ("delta", ctypes.c_float), ("sync_heads", ctypes.c_int32),
-                ("score_mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("score_mode", ctypes.c_int32), ("order", ctypes.c_int32), ("eviction", ctypes.c_int32),
+                ("refresh_baselines", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class dkv_buffers_t(ctypes.Structure):

@@ -23,10 +23,17 @@ def to_dev(x: np.ndarray, dtype: torch.dtype) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to("cuda", dtype)
 
 
+ORDER_NAMES = {dkv.DKV_ORDER_SCORE: "score", dkv.DKV_ORDER_SOURCE: "source"}
+EVICT_NAMES = {dkv.DKV_EVICT_MANDATORY_DENSEST: "mandatory_densest", dkv.DKV_EVICT_DENSEST: "densest",
+               dkv.DKV_EVICT_MANDATORY_SOURCE: "mandatory_source"}
+
+
 def oracle_params(bank: dkv.BankLayer) -> oracle.Params:
     p = bank.params
     return oracle.Params(tau=float(p.tau), sigma=float(p.sigma), p=float(p.p), eps=float(p.eps),
-                         delta=float(np.float32(p.delta)), sync_heads=bool(p.sync_heads))
+                         delta=float(np.float32(p.delta)), sync_heads=bool(p.sync_heads),
+                         order=ORDER_NAMES[p.order], evict=EVICT_NAMES[p.eviction],
+                         refresh_baselines=bool(p.refresh_baselines))
 
 
 def load_state(bank: dkv.BankLayer, ob: oracle.LayerBank) -> None:
@@ -125,9 +132,10 @@ def update_and_compare(bank: dkv.BankLayer, ob: oracle.LayerBank, K: np.ndarray,
     for h, (hb, hr) in enumerate(zip(before.heads, rec.heads)):
         if hr.empty_init:
             continue
-        s_g = inter["score"][h, :N]
-        rel = np.abs(s_g - hr.s) / np.maximum(np.abs(hr.s), 1e-30)
-        rep.score_max_rel = max(rep.score_max_rel, float(rel.max()))
+        if prm.order == "score":   # the source-order policy computes no scores
+            s_g = inter["score"][h, :N]
+            rel = np.abs(s_g - hr.s) / np.maximum(np.abs(hr.s), 1e-30)
+            rep.score_max_rel = max(rep.score_max_rel, float(rel.max()))
         pg = inter["perm"][h, :N]
         diff = np.nonzero(pg != hr.pi)[0]
         rep.perm_mismatch += len(diff)

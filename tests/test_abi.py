@@ -62,8 +62,10 @@ def test_struct_layouts_match_c():
 #include <stddef.h>
 #include "dkv.h"
 int main(void) {
-  printf("%zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t), sizeof(dkv_layer_stats_t),
-         sizeof(dkv_head_stats_t), sizeof(dkv_intermediates_t), offsetof(dkv_buffers_t, workspace_bytes));
+  printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t),
+         sizeof(dkv_layer_stats_t), sizeof(dkv_head_stats_t), sizeof(dkv_intermediates_t),
+         offsetof(dkv_buffers_t, workspace_bytes), offsetof(dkv_params_t, order), offsetof(dkv_params_t, eviction),
+         offsetof(dkv_params_t, refresh_baselines), offsetof(dkv_params_t, reserved));
   return 0;
 }
 """
@@ -80,7 +82,9 @@ int main(void) {
     sizes = [int(x) for x in out]
     assert sizes == [ctypes.sizeof(dkv.dkv_params_t), ctypes.sizeof(dkv.dkv_buffers_t),
                      ctypes.sizeof(dkv.dkv_layer_stats_t), ctypes.sizeof(dkv.dkv_head_stats_t),
-                     ctypes.sizeof(dkv.dkv_intermediates_t), dkv.dkv_buffers_t.workspace_bytes.offset]
+                     ctypes.sizeof(dkv.dkv_intermediates_t), dkv.dkv_buffers_t.workspace_bytes.offset,
+                     dkv.dkv_params_t.order.offset, dkv.dkv_params_t.eviction.offset,
+                     dkv.dkv_params_t.refresh_baselines.offset, dkv.dkv_params_t.reserved.offset]
 
 
 def test_host_only_entry_points():

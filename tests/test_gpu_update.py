@@ -95,6 +95,31 @@ def test_ragged_bf16_rollout(dkv, mode):
     _rollout(dkv, wl, mode)
 
 
+# Table 2(b) / App. E policy ablations (each alone, and three combined)
+POLICIES = {
+    "source_order": dict(order=1),
+    "densest_only": dict(eviction=1),
+    "mandatory_source": dict(eviction=2),
+    "refresh_baselines": dict(refresh_baselines=1),
+    "combined": dict(order=1, eviction=1, refresh_baselines=1),
+}
+
+
+@pytest.mark.parametrize("policy", sorted(POLICIES))
+def test_policy_variants_fp32(dkv, policy):
+    """Every policy on the tiny fp32 rollout (exactness mode): identical retained sets."""
+    wl = synth.get_workload("tiny_fp32_l1h2_d64")
+    reps = _rollout(dkv, wl, "fp32", check_attn=False, **POLICIES[policy])
+    assert sum(r.set_mismatch for r in reps) == 0
+
+
+@pytest.mark.parametrize("policy", sorted(POLICIES))
+def test_policy_variants_tc(dkv, policy):
+    """Every policy on the ragged bf16 rollout in the tensor-core mode."""
+    wl = synth.get_workload("wan13b_layer_h12", H=3, N=300, W=200, Nq=130, budgets=700, steps=7)
+    _rollout(dkv, wl, "tc", check_attn=False, **POLICIES[policy])
+
+
 @pytest.mark.parametrize("mode", ["fp32", "tc"])
 def test_frozen_regime_literal_kappa(dkv, mode):
     """Literal kappa (near-isotropic keys): the bank saturates and r* drops to 0 (no change)."""
