@@ -61,6 +61,11 @@ def parse_args():
     ap.add_argument("--eviction", choices=["mandatory_densest", "densest", "mandatory_source"],
                     default="mandatory_densest", help="eviction rule (policy ablation)")
     ap.add_argument("--refresh-baselines", action="store_true", help="refresh b after every update (ablation)")
+    ap.add_argument("--layers", type=int, default=1,
+                    help="layers updated per step on this GPU (whole-stack throughput; > 1 selects the stack run)")
+    ap.add_argument("--streams", type=int, default=4, help="stream pairs the layers of a stack step spread over")
+    ap.add_argument("--distinct-layers", type=int, default=2,
+                    help="stack run: layers with their own synthetic input stream (the rest reuse them)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -580,12 +585,136 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_stack(args):
+    """Whole-stack throughput on one GPU: every step updates `--layers` independent layer
+    banks (attention || admit, then compress, per layer), the layers spread over
+    `--streams` stream pairs and the whole step captured as one CUDA graph.  Inputs of
+    `--distinct-layers` synthetic layer streams are reused round-robin by the others
+    (each layer still has its own bank)."""
+    import torch
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_27922_gb300 import dkv
+
+    wl = make_workload(args.workload, 1, args.heads)
+    L, S = args.layers, max(1, args.streams)
+    D = max(1, min(args.distinct_layers, L))
+    W, K = args.warmup, args.steps
+    bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    inputs = []
+    for l in range(D):
+        inp = Inputs(wl, l, W + K)
+        inputs.append(({b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf))
+                        for b, (k, v) in inp.blocks.items()},
+                       [torch.from_numpy(q).to(dev, bf) for q in inp.queries]))
+    mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
+    banks = [dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(l), wl.N, bf, score_mode=mode, device=dev)
+             for l in range(L)]
+    for bk in banks:
+        bk.reset()
+    outs = [torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev) for _ in range(L)]
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    mains = [torch.cuda.Stream(dev) for _ in range(S)]
+    sides = [torch.cuda.Stream(dev) for _ in range(S)]
+
+    def stack_step(t):
+        cur = torch.cuda.current_stream(dev)
+        fork = torch.cuda.Event()
+        fork.record(cur)
+        joins = []
+        for l in range(L):
+            ms, ss = mains[l % S], sides[l % S]
+            blocks, queries = inputs[l % D]
+            kw, vw = blocks[wl.window_block(t)]
+            b = wl.admitted_block(t)
+            ms.wait_event(fork)
+            go = torch.cuda.Event()
+            go.record(ms)
+            ss.wait_event(go)
+            banks[l].attend(queries[t], kw, vw, out=outs[l], stream=ss)
+            done = torch.cuda.Event()
+            done.record(ss)
+            if b is not None:
+                kc, vc = blocks[b]
+                banks[l].admit(kc, vc, b, stream=ms)
+            ms.wait_event(done)
+            if b is not None:
+                banks[l].compress(stream=ms)
+            j = torch.cuda.Event()
+            j.record(ms)
+            joins.append(j)
+        for j in joins:
+            cur.wait_event(j)
+
+    stream = torch.cuda.current_stream(dev)
+    for t in range(W):
+        stack_step(t)
+    torch.cuda.synchronize()
+    graphs = []
+    cap = torch.cuda.Stream(dev)
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        for i in range(K):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=cap):
+                stack_step(W + i)
+            graphs.append(g)
+    stream.wait_stream(cap)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0, enabled=not args.no_clocks)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    keys = 0
+    total_ms = 0.0
+    rstars = []
+    for i in range(K):
+        t = W + i
+        if not args.no_flush:
+            flush.fill_(float(i))
+        ev[i][0].record(stream)
+        graphs[i].replay()
+        ev[i][1].record(stream)
+        ev[i][1].synchronize()
+        total_ms += ev[i][0].elapsed_time(ev[i][1])
+        if wl.admitted_block(t) is not None:
+            per_layer = []
+            for bk in banks:
+                Ls, hs = bk.stats()
+                keys += sum(h.occupancy_before + wl.N for h in hs)
+                per_layer.append((Ls.r_star, sum(h.evicted for h in hs)))
+            rstars.append(per_layer)
+    clk = clocks.stop()
+    for bk in banks:
+        bk.sync()
+    line = {
+        "metric": METRIC, "value": keys / (total_ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": K, "warmup": W,
+        "ms_per_step": total_ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": f"{wl.name}: {L} layer(s) x {wl.H} heads per step, d={wl.d}, N={wl.N}, "
+                               f"M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
+                   "score_mode": args.score_mode, "layers_per_gpu": L, "streams": f"{S} stream pairs",
+                   "cuda_graphs": True, "inputs": f"{D} distinct synthetic layer streams, reused round-robin",
+                   "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
+                   "parallelism": "layers of one GPU on concurrent streams"},
+        "blocks_per_s": K / (total_ms / 1e3),
+        "e2e": None, "gpu_launches": None, "roofline": None, "cpu_baseline": None, "clocks": clk,
+        "update": {"last_step_r_star_per_layer": [r for r, _ in rstars[-1]] if rstars else [],
+                   "last_step_evicted_per_layer": [e for _, e in rstars[-1]] if rstars else [],
+                   "layers_admitting_per_step": [sum(1 for r, _ in st if r > 0) for st in rstars]},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     if args.warmup < 3:
         print("warning: --warmup < 3 does not reach the steady state of the bank", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args)
+    elif args.layers > 1:
+        run_stack(args)
     else:
         run_ours(args)
 
