@@ -61,6 +61,8 @@ def parse_args():
     ap.add_argument("--eviction", choices=["mandatory_densest", "densest", "mandatory_source"],
                     default="mandatory_densest", help="eviction rule (policy ablation)")
     ap.add_argument("--refresh-baselines", action="store_true", help="refresh b after every update (ablation)")
+    ap.add_argument("--attn-passes", type=int, default=1,
+                    help="bank-reading attention passes per update (denoising passes; the update runs once)")
     ap.add_argument("--layers", type=int, default=1,
                     help="layers updated per step on this GPU (whole-stack throughput; > 1 selects the stack run)")
     ap.add_argument("--streams", type=int, default=4, help="stream pairs the layers of a stack step spread over")
@@ -186,12 +188,25 @@ class Inputs:
         ro = synth.LayerRollout(wl, layer)
         need = set()
         for t in range(n_steps):
-            need.add(wl.window_block(t))
+            for blk, _, _ in wl.window_parts(t):
+                need.add(blk)
             b = wl.admitted_block(t)
             if b is not None:
                 need.add(b)
         self.blocks = {b: ro.block(b) for b in sorted(need)}
         self.queries = [ro.queries(t) for t in range(n_steps)]
+
+    def window(self, t, blocks, cat):
+        """Window K/V of step t from the given block tensors (whole block: no copy)."""
+        parts = self.wl.window_parts(t)
+        if len(parts) == 1 and parts[0][1] == 0 and parts[0][2] == self.wl.N:
+            return blocks[parts[0][0]]
+        return (cat([blocks[b][0][:, s0:e0] for b, s0, e0 in parts]),
+                cat([blocks[b][1][:, s0:e0] for b, s0, e0 in parts]))
+
+    def window_is_block(self, t, b):
+        parts = self.wl.window_parts(t)
+        return len(parts) == 1 and parts[0] == (b, 0, self.wl.N)
 
 
 # --------------------------------------------------------------------------- our arm
@@ -220,6 +235,9 @@ def run_ours(args):
     bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     dblocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
     dq = [torch.from_numpy(q).to(dev, bf) for q in inp.queries[:W + K]]
+    cat1 = lambda xs: torch.cat(xs, dim=1).contiguous()
+    dwin = [inp.window(t, dblocks, cat1) for t in range(W + K)]
+    P = max(1, args.attn_passes)
     mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
     policy = dict(order={"score": dkv.DKV_ORDER_SCORE, "source": dkv.DKV_ORDER_SOURCE}[args.order],
                   eviction={"mandatory_densest": dkv.DKV_EVICT_MANDATORY_DENSEST, "densest": dkv.DKV_EVICT_DENSEST,
@@ -237,7 +255,8 @@ def run_ours(args):
     def step(t, Q, KW, VW, KC, VC):
         b = wl.admitted_block(t)
         if args.no_overlap:
-            bank.attend(Q, KW, VW, out=out)
+            for _ in range(P):
+                bank.attend(Q, KW, VW, out=out)
             if b is not None:
                 bank.admit(KC, VC, b)
                 bank.compress()
@@ -248,7 +267,8 @@ def run_ours(args):
         go = torch.cuda.Event()
         go.record(cur)
         side.wait_event(go)
-        bank.attend(Q, KW, VW, out=out, stream=side)
+        for _ in range(P):   # every denoising pass reads the bank; the update runs once
+            bank.attend(Q, KW, VW, out=out, stream=side)
         done = torch.cuda.Event()
         done.record(side)
         if b is not None:
@@ -258,7 +278,7 @@ def run_ours(args):
             bank.compress(stream=cur)
 
     def device_step(t):
-        kw, vw = dblocks[wl.window_block(t)]
+        kw, vw = dwin[t]
         b = wl.admitted_block(t)
         kc, vc = dblocks[b] if b is not None else (None, None)
         step(t, dq[t], kw, vw, kc, vc)
@@ -341,18 +361,21 @@ def run_ours(args):
         host_blocks = {b: (torch.from_numpy(k).to(bf).pin_memory(), torch.from_numpy(v).to(bf).pin_memory())
                        for b, (k, v) in inp.blocks.items()}
         host_q = [torch.from_numpy(q).to(bf).pin_memory() for q in inp.queries[W + K:]]
+        cat_pin = lambda xs: torch.cat(xs, dim=1).contiguous().pin_memory()
+        host_win = [inp.window(W + K + i, host_blocks, cat_pin) for i in range(K)]
         host_out = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf).pin_memory()
         kbuf = torch.empty(wl.H, wl.N, wl.d, dtype=bf, device=dev)
         vbuf = torch.empty_like(kbuf)
-        kw_buf = torch.empty(wl.H, wl.W, wl.d, dtype=bf, device=dev)
-        vw_buf = torch.empty_like(kw_buf)
+        # one contiguous device buffer pair per distinct window length (allocated before any capture)
+        win_bufs = {n: (torch.empty(wl.H, n, wl.d, dtype=bf, device=dev), torch.empty(wl.H, n, wl.d, dtype=bf, device=dev))
+                    for n in sorted({hw[0].shape[1] for hw in host_win})}
         qbuf = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
         copy_s = torch.cuda.Stream(dev)
         bank.set_timing(False)
 
         def e2e_step(i):
             t = W + K + i
-            wb, ab = wl.window_block(t), wl.admitted_block(t)
+            ab = wl.admitted_block(t)
             cur = torch.cuda.current_stream(dev)
             start = torch.cuda.Event()
             start.record(cur)
@@ -361,19 +384,22 @@ def run_ours(args):
                 qbuf.copy_(host_q[i], non_blocking=True)
             q_ready = torch.cuda.Event()
             q_ready.record(copy_s)
-            kw_buf.copy_(host_blocks[wb][0], non_blocking=True)
-            vw_buf.copy_(host_blocks[wb][1], non_blocking=True)
-            nbytes = qbuf.numel() * qbuf.element_size() + 2 * kw_buf.numel() * kw_buf.element_size()
-            if ab is not None and ab != wb:
+            kw_h, vw_h = host_win[i]
+            kw, vw = win_bufs[kw_h.shape[1]]
+            kw.copy_(kw_h, non_blocking=True)
+            vw.copy_(vw_h, non_blocking=True)
+            nbytes = qbuf.numel() * qbuf.element_size() + 2 * kw_h.numel() * kw_h.element_size()
+            if ab is not None and not inp.window_is_block(t, ab):
                 kbuf.copy_(host_blocks[ab][0], non_blocking=True)
                 vbuf.copy_(host_blocks[ab][1], non_blocking=True)
                 kc, vc = kbuf, vbuf
                 nbytes += 2 * kbuf.numel() * kbuf.element_size()
             else:
-                kc, vc = kw_buf, vw_buf   # the block leaving the window is the window block
+                kc, vc = kw, vw   # the block leaving the window is the window block
             if args.no_overlap:
                 cur.wait_event(q_ready)
-                bank.attend(qbuf, kw_buf, vw_buf, out=out)
+                for _ in range(P):
+                    bank.attend(qbuf, kw, vw, out=out)
                 host_out.copy_(out, non_blocking=True)
                 if ab is not None:
                     bank.admit(kc, vc, ab)
@@ -383,7 +409,8 @@ def run_ours(args):
             kv_ready.record(cur)
             side.wait_event(kv_ready)
             side.wait_event(q_ready)
-            bank.attend(qbuf, kw_buf, vw_buf, out=out, stream=side)
+            for _ in range(P):
+                bank.attend(qbuf, kw, vw, out=out, stream=side)
             att_done = torch.cuda.Event()
             att_done.record(side)
             if ab is not None:
@@ -484,6 +511,7 @@ def run_ours(args):
             "config": {"workload": f"{wl.name}: {wl.L if world > 1 else 1} layer(s) x {wl.H} heads, d={wl.d}, "
                                    f"N={wl.N}, M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
                        "score_mode": args.score_mode, "layers_per_gpu": 1,
+                       "attn_passes_per_update": max(1, args.attn_passes),
                        "policy": {"order": args.order, "eviction": args.eviction,
                                   "refresh_baselines": bool(args.refresh_baselines)},
                        "streams": "attention || admit, then compress" if not args.no_overlap else "one stream",
@@ -605,11 +633,13 @@ def run_stack(args):
     W, K = args.warmup, args.steps
     bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     inputs = []
+    cat1 = lambda xs: torch.cat(xs, dim=1).contiguous()
     for l in range(D):
         inp = Inputs(wl, l, W + K)
-        inputs.append(({b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf))
-                        for b, (k, v) in inp.blocks.items()},
-                       [torch.from_numpy(q).to(dev, bf) for q in inp.queries]))
+        blocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
+        inputs.append((blocks, [torch.from_numpy(q).to(dev, bf) for q in inp.queries],
+                       [inp.window(t, blocks, cat1) for t in range(W + K)]))
+    P = max(1, args.attn_passes)
     mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
     banks = [dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(l), wl.N, bf, score_mode=mode, device=dev)
              for l in range(L)]
@@ -627,14 +657,15 @@ def run_stack(args):
         joins = []
         for l in range(L):
             ms, ss = mains[l % S], sides[l % S]
-            blocks, queries = inputs[l % D]
-            kw, vw = blocks[wl.window_block(t)]
+            blocks, queries, windows = inputs[l % D]
+            kw, vw = windows[t]
             b = wl.admitted_block(t)
             ms.wait_event(fork)
             go = torch.cuda.Event()
             go.record(ms)
             ss.wait_event(go)
-            banks[l].attend(queries[t], kw, vw, out=outs[l], stream=ss)
+            for _ in range(P):
+                banks[l].attend(queries[t], kw, vw, out=outs[l], stream=ss)
             done = torch.cuda.Event()
             done.record(ss)
             if b is not None:

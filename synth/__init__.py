@@ -126,7 +126,8 @@ class Workload:
     Nq: int                     # queries per step (per head)
     steps: int                  # rollout length
     dtype: str                  # "fp32" or "bf16"
-    window: str                 # "own": window = block t; "prev": window = block t-1
+    window: str                 # "own": window = block t; "prev": window = block t-1;
+                                # "sink5": first frame of block 0 + the 5 most recent frames
     budgets: Tuple[int, ...]    # M_h per (layer, head)
     clusters: Tuple[int, ...]
     kappa: Tuple[float, ...]
@@ -135,6 +136,7 @@ class Workload:
     key_scale: Optional[float] = None  # None -> sqrt(d)
     kappa_per_dim: bool = True  # vMF concentration used = kappa * d (see module docstring)
     seed: int = 0
+    frames_per_block: int = 3   # a block is this many latent frames of N / frames_per_block tokens
 
     def kappa_vmf(self, idx: int) -> float:
         return self.kappa[idx] * (self.d if self.kappa_per_dim else 1)
@@ -150,13 +152,41 @@ class Workload:
         """Index of the block that leaves the window (is offered to the bank) at step t."""
         if self.window == "own":
             return t
+        if self.window == "sink5":
+            # after step t the 5-frame window starts at frame 3t - 2: block t - 2 has left it
+            return t - 2 if t >= 2 else None
         return t - 1 if t >= 1 else None
 
     def window_block(self, t: int) -> int:
-        """Index of the block whose K/V form the local window read at step t."""
+        """Index of the block whose K/V form the local window read at step t (whole-block
+        windows only; see window_parts)."""
+        if self.window == "sink5":
+            raise ValueError("the sink5 window is not one block; use window_parts")
         if self.window == "own":
             return t
         return t - 1 if t >= 1 else 0
+
+    def window_parts(self, t: int) -> List[Tuple[int, int, int]]:
+        """The local window read at step t as (block, first token, end token) pieces, in order.
+        sink5: the first frame of block 0 (the first-frame sink) followed by the five most
+        recent finalized frames (Sec. 4.1 / App. D); at t = 0 nothing is finalized and the
+        block attends to itself."""
+        if self.window != "sink5":
+            return [(self.window_block(t), 0, self.N)]
+        F = self.N // self.frames_per_block
+        if t == 0:
+            return [(0, 0, self.N)]
+        parts = [(0, 0, F)]
+        for f in range(max(1, self.frames_per_block * t - 5), self.frames_per_block * t):
+            b, o = divmod(f, self.frames_per_block)
+            if parts[-1][0] == b and parts[-1][2] == o * F and len(parts) > 1:
+                parts[-1] = (b, parts[-1][1], (o + 1) * F)
+            else:
+                parts.append((b, o * F, (o + 1) * F))
+        return parts
+
+    def window_len(self, t: int) -> int:
+        return sum(e - s for _, s, e in self.window_parts(t))
 
 
 def _per_head(rng: np.random.Generator, n: int, choices=None, lo=None, hi=None, const=None):
@@ -204,6 +234,12 @@ _SPECS: Dict[str, dict] = {
     "wan13b_layer_h12": dict(L=1, H=12, d=128, N=4680, W=4680, Nq=4680, steps=20, dtype="bf16",
                              window="prev", budgets=9360, clusters=64, kappa=20.0,
                              recurrence=0.6, seed=0),
+    # The Wan-1.3B layer with the paper's visible context: a first-frame sink plus a 5-frame
+    # local window (9,360 window tokens) next to the bank; the block offered at step t is the
+    # one that has left the 5-frame window (t - 2).
+    "wan13b_layer_h12_sink5": dict(L=1, H=12, d=128, N=4680, W=9360, Nq=4680, steps=20, dtype="bf16",
+                                   window="sink5", budgets=9360, clusters=64, kappa=20.0,
+                                   recurrence=0.6, seed=0),
     # Full Wan-1.3B-shaped stack: 30 x 12 heads; 64-256 clusters and 40-80% recurrence per head.
     "wan13b_stack_l30h12": dict(L=30, H=12, d=128, N=4680, W=4680, Nq=4680, steps=40, dtype="bf16",
                                 window="prev", budgets=9360,
@@ -321,5 +357,13 @@ class LayerRollout:
         return Q
 
     def window(self, t: int) -> Tuple[np.ndarray, np.ndarray]:
-        """Local-window K/V read at step t (a whole block)."""
-        return self.block(self.wl.window_block(t))
+        """Local-window K/V read at step t, float32 [len(heads)][window_len(t)][d]."""
+        parts = self.wl.window_parts(t)
+        if len(parts) == 1 and parts[0][1] == 0 and parts[0][2] == self.wl.N:
+            return self.block(parts[0][0])
+        ks, vs = [], []
+        for b, s0, e0 in parts:
+            K, V = self.block(b)
+            ks.append(K[:, s0:e0])
+            vs.append(V[:, s0:e0])
+        return np.concatenate(ks, axis=1), np.concatenate(vs, axis=1)

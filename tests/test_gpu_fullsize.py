@@ -227,6 +227,14 @@ def test_fullsize_large_bank(dkv):
     assert min(occ) > 2 * wl.N
 
 
+def test_fullsize_sink5_context(dkv):
+    """The paper's visible context: first-frame sink + 5-frame window (9,360 window tokens)
+    next to the bank; the block offered at step t is the one that left the window."""
+    wl = synth.get_workload("wan13b_layer_h12_sink5")
+    evicted, _ = _run(dkv, wl, steps=6)
+    assert evicted > 0
+
+
 @pytest.mark.parametrize("sync", [1, 0])
 def test_fullsize_headwise_budgets(dkv, sync):
     """Wan-14B-shaped layer: 40 heads with budgets drawn from {2340, 4680, 9360, 18720}."""

@@ -42,3 +42,29 @@ def test_workload_shapes():
     wl0 = synth.get_workload("tiny_fp32_l1h2_d64")
     assert (wl0.L, wl0.H, wl0.d, wl0.N, wl0.budgets, wl0.dtype) == (1, 2, 64, 256, (512, 512), "fp32")
     assert wl0.admitted_block(0) == 0 and synth.get_workload("wan13b_layer_h12").admitted_block(0) is None
+
+
+def test_sink5_window_parts_and_contents():
+    """First-frame sink + five most recent frames (Sec. 4.1, App. D): 9,360 window tokens
+    from step 2 on, the sink first; the block offered at step t is t - 2."""
+    wl = synth.get_workload("wan13b_layer_h12_sink5", H=2, N=12, W=24, Nq=4)
+    F = wl.N // wl.frames_per_block
+    assert wl.window_len(0) == wl.N and wl.window_len(1) == wl.N
+    for t in range(2, 6):
+        parts = wl.window_parts(t)
+        assert parts[0] == (0, 0, F)                                   # the sink
+        frames = []
+        for b, s0, e0 in parts[1:]:
+            assert s0 % F == 0 and e0 % F == 0
+            frames += [b * wl.frames_per_block + f for f in range(s0 // F, e0 // F)]
+        assert frames == list(range(3 * t - 5, 3 * t))                # the 5 most recent frames
+        assert wl.window_len(t) == 6 * F
+        assert wl.admitted_block(t) == t - 2
+    assert wl.admitted_block(0) is None and wl.admitted_block(1) is None
+    ro = synth.LayerRollout(wl, 0)
+    Kw, Vw = ro.window(3)
+    K0, _ = ro.block(0)
+    K1, V1 = ro.block(1)
+    K2, V2 = ro.block(2)
+    assert np.array_equal(Kw[:, :F], K0[:, :F])
+    assert np.array_equal(Kw[:, F:3 * F], K1[:, F:]) and np.array_equal(Vw[:, 3 * F:], V2)
