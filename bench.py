@@ -84,6 +84,31 @@ def dist_env():
     return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("LOCAL_RANK", "0"))
 
 
+def layer_of_rank(rank: int) -> int:
+    """Weak scaling: each rank updates its own layer (layers are independent: separate
+    banks, r* per layer), so ranks exchange nothing on the data path."""
+    return rank
+
+
+def reduce_over_ranks(total_ms: float, keys: float, world: int, device=None):
+    """Whole-job figures: the slowest rank's time and the keys of all ranks."""
+    if world <= 1:
+        return total_ms, float(keys)
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([total_ms, keys], dtype=torch.float64, device=device)
+    mx = tt.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    sm = tt.clone()
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(sm[1])
+
+
+def reference_runs_on(rank: int) -> bool:
+    """The reference arm (the oracle on the host) runs and prints on rank 0 only."""
+    return rank == 0
+
+
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
     """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
@@ -228,7 +253,7 @@ def run_ours(args):
     from paper_2608_27922_gb300 import dkv
 
     wl = make_workload(args.workload, world, args.heads)
-    layer = rank
+    layer = layer_of_rank(rank)
     W, K = args.warmup, args.steps
     n_total = W + K + (0 if args.no_e2e else K)
     inp = Inputs(wl, layer, n_total)
@@ -341,15 +366,7 @@ def run_ours(args):
     clk = clocks.stop()
     bank.sync()
     total_ms = sum(step_ms)
-    if world > 1:
-        tt = torch.tensor([total_ms, keys], dtype=torch.float64, device=dev)
-        mx = tt.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = tt.clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        total_ms_max, keys_all = float(mx[0]), float(sm[1])
-    else:
-        total_ms_max, keys_all = total_ms, float(keys)
+    total_ms_max, keys_all = reduce_over_ranks(total_ms, keys, world, dev)
     value = keys_all / (total_ms_max / 1e3)
 
     # ---- end to end through the C ABI with host buffers: H2D inputs, compute, D2H output.
@@ -465,13 +482,7 @@ def run_ours(args):
                 e2e_keys += sum(h.occupancy_before + wl.N for h in hs)
             h2d += h2d_i
             d2h += host_out.numel() * host_out.element_size()
-        if world > 1:
-            tt = torch.tensor([e2e_ms, e2e_keys], dtype=torch.float64, device=dev)
-            mx = tt.clone()
-            dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-            sm = tt.clone()
-            dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-            e2e_ms, e2e_keys = float(mx[0]), float(sm[1])
+        e2e_ms, e2e_keys = reduce_over_ranks(e2e_ms, e2e_keys, world, dev)
         e2e = {"value": e2e_keys / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d // K,
                "d2h_bytes_per_step": d2h // K, "ms_per_step": e2e_ms / K,
                "copies": "pinned host buffers; Q and O on a copy stream, window K/V on the launching stream",
@@ -587,7 +598,7 @@ def cpu_baseline_sample(wl, layer):
 
 def run_reference(args):
     rank, world, _ = dist_env()
-    if rank != 0:
+    if not reference_runs_on(rank):
         return
     wl = make_workload(args.workload, 1)
     ro, ob, t = _oracle_head_setup(wl, 0, 0)
