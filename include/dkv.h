@@ -254,6 +254,15 @@ dkv_status_t dkv_bank_set_timing(dkv_bank_t bank, int32_t enable);
 dkv_status_t dkv_bank_kernel_times(dkv_bank_t bank, int32_t max_kernels, char* names /* [max][48] */,
                                    int32_t* launches, double* total_ms, int32_t* n_kernels);
 
+/* Self-test of the bounded device-side waits (no paper counterpart; a diagnostic).
+ * Launches one CTA that waits, through the library's own bounded-wait helper, on a
+ * barrier nothing arrives on; after limit_us microseconds (1 .. 1e6) the wait gives
+ * up, the kernel records the timeout and returns.  Returns DKV_ERR_TIMEOUT when the
+ * wait gave up as designed (the expected result), and writes the measured wait
+ * duration to *elapsed_ns (host).  Synchronises the device; allocates 16 bytes of
+ * device memory for the duration of the call.  The context stays usable.          */
+dkv_status_t dkv_selftest_wait_timeout(int32_t limit_us, int64_t* elapsed_ns);
+
 /* Largest candidate count accepted by dkv_candidate_order_noalloc. */
 #define DKV_NOALLOC_MAX_N 16384
 

@@ -83,6 +83,7 @@ SIGNATURES = [
     ("dkv_bank_kernel_times", _I, [_P, _I, ctypes.c_char_p, ctypes.POINTER(ctypes.c_int32),
                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int32)]),
     ("dkv_candidate_order_noalloc", _I, [_P, _P, _I, _P, _I, _I, _I, ctypes.POINTER(dkv_params_t), _P, _P, _P]),
+    ("dkv_selftest_wait_timeout", _I, [_I, ctypes.POINTER(ctypes.c_int64)]),
 ]
 
 DKV_NOALLOC_MAX_N = 16384
@@ -235,6 +236,14 @@ def dkv_candidate_order_noalloc(K_bank, base, m: int, Kc, N: int, d: int, dtype:
     _check(lib().dkv_candidate_order_noalloc(_ptr(K_bank) if m > 0 else 0, _ptr(base) if m > 0 else 0, m,
                                              _ptr(Kc), N, d, dtype, ctypes.byref(params), _ptr(scores_out),
                                              _ptr(perm_out), _stream(stream)), "dkv_candidate_order_noalloc")
+
+
+def dkv_selftest_wait_timeout(limit_us: int):
+    """Runs the bounded-wait self-test; returns (status, elapsed_ns).  DKV_ERR_TIMEOUT (6)
+    is the expected status: the wait gave up after limit_us as designed."""
+    el = ctypes.c_int64(0)
+    st = lib().dkv_selftest_wait_timeout(int(limit_us), ctypes.byref(el))
+    return int(st), int(el.value)
 
 
 # ----------------------------------------------------------------- buffer owner

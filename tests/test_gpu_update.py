@@ -220,3 +220,16 @@ def test_device_error_word_reports_inconsistent_bank(dkv):
     bank.update(K, K, 1)
     bank.sync()
     bank.close()
+
+
+def test_bounded_wait_gives_up_and_context_stays_usable(dkv):
+    """A device-side wait on a barrier nothing arrives on gives up after its limit (1 ms
+    here) through the same helper every tensor-core kernel uses; the host reads the
+    timeout status, and the context still runs a parity-checked update afterwards."""
+    st, el = dkv.dkv_selftest_wait_timeout(1000)
+    assert st == 6, st                      # DKV_ERR_TIMEOUT: the wait gave up as designed
+    assert 1_000_000 <= el < 100_000_000, el
+    st2, _ = dkv.dkv_selftest_wait_timeout(1000)
+    assert st2 == 6
+    wl = synth.get_workload("tiny_fp32_l1h2_d64", steps=3)
+    _rollout(dkv, wl, "fp32", check_attn=False)
