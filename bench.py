@@ -286,8 +286,8 @@ def run_ours(args):
                 bank.admit(KC, VC, b)
                 bank.compress()
             return
-        # attention and admit both only read the bank (the update is atomic from the
-        # reader's side), so they run concurrently; compress waits for attention
+        # attention, admit and evict only read the bank (the update is atomic from the
+        # reader's side), so they run concurrently; only the commit waits for attention
         cur = torch.cuda.current_stream(dev)
         go = torch.cuda.Event()
         go.record(cur)
@@ -298,9 +298,10 @@ def run_ours(args):
         done.record(side)
         if b is not None:
             bank.admit(KC, VC, b, stream=cur)
+            bank.evict(stream=cur)
         cur.wait_event(done)
         if b is not None:
-            bank.compress(stream=cur)
+            bank.commit(stream=cur)
 
     def device_step(t):
         kw, vw = dwin[t]
@@ -372,7 +373,7 @@ def run_ours(args):
     # ---- end to end through the C ABI with host buffers: H2D inputs, compute, D2H output.
     # Every step uploads its queries and window K/V from pinned host memory and downloads
     # the attention output; the uploads gate the kernels that read them (admit needs only
-    # the window K/V, attention also Q), and O is downloaded while compress runs.
+    # the window K/V, attention also Q), and O is downloaded while the commit runs.
     e2e = None
     if not args.no_e2e:
         host_blocks = {b: (torch.from_numpy(k).to(bf).pin_memory(), torch.from_numpy(v).to(bf).pin_memory())
@@ -432,6 +433,7 @@ def run_ours(args):
             att_done.record(side)
             if ab is not None:
                 bank.admit(kc, vc, ab, stream=cur)
+                bank.evict(stream=cur)
             copy_s.wait_event(att_done)
             with torch.cuda.stream(copy_s):
                 host_out.copy_(out, non_blocking=True)
@@ -439,7 +441,7 @@ def run_ours(args):
             o_done.record(copy_s)
             cur.wait_event(att_done)
             if ab is not None:
-                bank.compress(stream=cur)
+                bank.commit(stream=cur)
             cur.wait_event(o_done)
             return nbytes
 
@@ -525,7 +527,7 @@ def run_ours(args):
                        "attn_passes_per_update": max(1, args.attn_passes),
                        "policy": {"order": args.order, "eviction": args.eviction,
                                   "refresh_baselines": bool(args.refresh_baselines)},
-                       "streams": "attention || admit, then compress" if not args.no_overlap else "one stream",
+                       "streams": "attention || admit + evict, then commit" if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                        "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
@@ -626,7 +628,7 @@ def run_reference(args):
 
 def run_stack(args):
     """Whole-stack throughput on one GPU: every step updates `--layers` independent layer
-    banks (attention || admit, then compress, per layer), the layers spread over
+    banks (attention || admit + evict, then commit, per layer), the layers spread over
     `--streams` stream pairs and the whole step captured as one CUDA graph.  Inputs of
     `--distinct-layers` synthetic layer streams are reused round-robin by the others
     (each layer still has its own bank)."""
@@ -682,9 +684,10 @@ def run_stack(args):
             if b is not None:
                 kc, vc = blocks[b]
                 banks[l].admit(kc, vc, b, stream=ms)
+                banks[l].evict(stream=ms)
             ms.wait_event(done)
             if b is not None:
-                banks[l].compress(stream=ms)
+                banks[l].commit(stream=ms)
             j = torch.cuda.Event()
             j.record(ms)
             joins.append(j)

@@ -196,8 +196,23 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
 
 /* Step 3 + commit for the block given to the preceding admit (Sec. 3.4;
  * Alg. 1; Eq. 12; Eq. C.4).  After it completes on `stream`, occupancy,
- * k, v, rho, base, knorm and provenance describe the committed banks.         */
+ * k, v, rho, base, knorm and provenance describe the committed banks.
+ * Equivalent to dkv_bank_evict followed by dkv_bank_commit on one stream.    */
 dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream);
+
+/* First half of compress: rho~ at the shared prefix r* (Eq. C.2), the mandatory
+ * and densest eviction sets (Sec. 3.4) and the workspace copies of survivors and
+ * evicted keys.  Reads the bank but does not modify k, v, occupancy or provenance,
+ * so bank-reading attention of the current step may still run concurrently on
+ * another stream.  Valid only right after admit (else DKV_ERR_STATE).          */
+dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream);
+
+/* Second half of compress: the commit of Eq. 12 (admitted candidates into the
+ * evicted slots, then appended), density maintenance of the survivors (Eq. C.4)
+ * and the frozen baselines of the admitted states (Eq. 5).  Overwrites k, v and
+ * occupancy: every reader of the pre-update bank (attention on another stream)
+ * must be ordered before it.  Valid only right after evict (else DKV_ERR_STATE). */
+dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream);
 
 /* Bank-reading attention (Sec. 3.2, Fig. 2):
  *   O[h] = softmax(Q[h] [Kbank_h ; Kw[h]]^T / sqrt(d)) [Vbank_h ; Vw[h]]
@@ -237,7 +252,7 @@ typedef struct {
   const int32_t* perm;       /* [H][n_max]  pi_h: candidate index at sorted position   */
   const int32_t* cross;      /* [H][M_max]  min{r : g_i(r) >= tau} over r <= rmax,
                                             INT32_MAX when no such r                 */
-  const float* rho_tilde;    /* [H][M_max]  rho~_i(r_h) (Eq. C.2), set by compress     */
+  const float* rho_tilde;    /* [H][M_max]  rho~_i(r_h) (Eq. C.2), set by evict        */
   const int32_t* slot_new;   /* [H][n_max]  bank slot of the j-th admitted candidate   */
   int64_t n_max;
   int64_t M_max;

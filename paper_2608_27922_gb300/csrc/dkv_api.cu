@@ -156,7 +156,7 @@ struct dkv_bank_s {
   dkv_params_t params{};
   std::vector<int32_t> budgets;
   bool tc = false;
-  int state = 0;   // 0: idle, 1: admitted
+  int state = 0;   // 0: idle, 1: admitted, 2: evicted
   const void* Kc = nullptr;
   const void* Vc = nullptr;
   int N = 0;
@@ -327,14 +327,11 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   const Ws& w = bank->w;
   Timer* t = &bank->timer;
   bank->last = s;
-  cudaError_t e = cudaMemsetAsync(w.hist, 0, sizeof(int32_t) * (size_t)b.H * w.hist_stride, s);
-  if (e == cudaSuccess) e = launch_prepare(b, w, N, step, s, t);
-  if (e == cudaSuccess) e = launch_cand_norms(b, w, Kc, N, bank->kp, s, t);
+  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, bank->kp, s, t);
   if (e == cudaSuccess)
     if (bank->kp.order == DKV_ORDER_SCORE)   // source order needs no scores (App. E)
       e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
-  if (e == cudaSuccess) e = launch_sort(b, w, bank->kp.order == DKV_ORDER_SOURCE, s, t);
-  if (e == cudaSuccess) e = launch_permute(b, w, Kc, N, s, t);
+  if (e == cudaSuccess) e = launch_sort(b, w, Kc, bank->kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_cross_tc(b, w, bank->kp, s, t) : launch_cross_fp32(b, w, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_rstar(b, w, bank->kp, s, t);
   if (e != cudaSuccess) return DKV_ERR_CUDA;
@@ -346,7 +343,7 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   return DKV_OK;
 }
 
-dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream) {
+dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream) {
   if (!bank) return DKV_ERR_ARG;
   if (bank->state != 1) return DKV_ERR_STATE;
   cudaStream_t s = (cudaStream_t)stream;
@@ -355,14 +352,33 @@ dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream) {
   Timer* t = &bank->timer;
   const KParams& kp = bank->kp;
   bank->last = s;
-  bank->state = 0;
+  bank->state = 2;
   cudaError_t e = bank->tc ? launch_project_tc(b, w, kp, s, t) : launch_project_fp32(b, w, kp, s, t);
   if (e == cudaSuccess) e = launch_select(b, w, kp.eviction, s, t);
-  if (e == cudaSuccess) e = launch_gather(b, w, s, t);
-  if (e == cudaSuccess) e = launch_commit(b, w, bank->Vc, bank->N, s, t);
+  return cuda_status(e);
+}
+
+dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream) {
+  if (!bank) return DKV_ERR_ARG;
+  if (bank->state != 2) return DKV_ERR_STATE;
+  cudaStream_t s = (cudaStream_t)stream;
+  const Bank& b = bank->b;
+  const Ws& w = bank->w;
+  Timer* t = &bank->timer;
+  const KParams& kp = bank->kp;
+  bank->last = s;
+  bank->state = 0;
+  cudaError_t e = launch_commit(b, w, bank->Vc, bank->N, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_subtract_tc(b, w, kp, s, t) : launch_subtract_fp32(b, w, kp, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_newbase_tc(b, w, kp, s, t) : launch_newbase_fp32(b, w, kp, s, t);
   return cuda_status(e);
+}
+
+dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream) {
+  if (!bank) return DKV_ERR_ARG;
+  if (bank->state != 1) return DKV_ERR_STATE;
+  const dkv_status_t st = dkv_bank_evict(bank, stream);
+  return st != DKV_OK ? st : dkv_bank_commit(bank, stream);
 }
 
 dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const void* Kw, const void* Vw,

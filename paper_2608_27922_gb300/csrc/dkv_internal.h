@@ -69,18 +69,16 @@ void timer_end(Timer* t, cudaStream_t s);
 
 // ---- launches (each returns cudaGetLastError() of its launch) ----
 // update front half (admit)
-cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cudaStream_t s, Timer* t);
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
-                              Timer* t);
+// candidates' norms and extension rows, zeroed crossing histogram, update snapshot
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
+                              cudaStream_t s, Timer* t);
 cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
-cudaError_t launch_sort(const Bank& b, const Ws& w, int identity, cudaStream_t s, Timer* t);
-cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t);
 cudaError_t launch_cross_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // update back half (compress)
 cudaError_t launch_project_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_select(const Bank& b, const Ws& w, int eviction, cudaStream_t s, Timer* t);
-cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t);
 cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t);
 cudaError_t launch_subtract_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_newbase_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);

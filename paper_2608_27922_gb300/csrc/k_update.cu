@@ -1,15 +1,16 @@
 // Selection, ordering and compaction kernels of the bank update (no pair math).
 //
-//   prepare      snapshot of occupancy, budgets and the prefix range of this update
-//   cand_norms   ||k_x||^2 of the candidates (fp32)
-//   sort         stable ascending order of the Eq. 6 scores, ties by source index (Alg. 1)
-//   permute      candidate keys copied into pi order (operand of the prefix passes)
+//   cand_norms   ||k_x||^2 of the candidates (fp32) and their extension rows, plus (one
+//                extra block) the snapshot of occupancy, budgets and prefix range
+//   sort         stable ascending order of the Eq. 6 scores, ties by source index (Alg. 1),
+//                and the candidate keys copied into that order (operand of the prefix passes)
 //   rstar_*      violator counts c_r = #{cross <= r}, budgets e_r (Eq. 10), feasibility,
 //                and the largest prefix feasible for every head (Eq. 11)
 //   select       mandatory set {g(r*) >= tau} plus the densest rho~(r*) (Step 3), via a
 //                radix select on the fp32 bit patterns; ties evict the older state
-//   gather       keys of the surviving and of the evicted states (operands of Eq. C.4)
-//   commit       Eq. 12: admitted keys/values into the evicted slots, the rest appended
+//   commit       Eq. 12: admitted keys/values into the evicted slots, the rest appended;
+//                keys of the surviving and of the evicted states copied out first
+//                (operands of Eq. C.4)
 #include "dkv.h"
 #include "dkv_internal.h"
 
@@ -50,7 +51,18 @@ __device__ __forceinline__ void copy_groups(int nrows, int per_row, Map map) {
   }
 }
 
-__global__ void k_prepare(Bank b, Ws w, int N, int64_t step) {
+// One 64-byte group: all four loads are issued before the stores.
+__device__ __forceinline__ void copy64(const uint4* src, uint4* dst) {
+  uint4 v[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) v[k] = src[k];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) dst[k] = v[k];
+}
+
+// Snapshot of occupancy and budgets per head and the prefix range of this update
+// (one block).
+__device__ __forceinline__ void prepare_body(const Bank& b, const Ws& w, int N, int64_t step) {
   __shared__ int s_min_budget, s_live;
   if (threadIdx.x == 0) { s_min_budget = INT_MAX; s_live = 0; }
   __syncthreads();
@@ -119,9 +131,10 @@ __device__ __forceinline__ float sq_sum(const T* p, int pl) {
 constexpr int NR_ROWS = 4;
 
 template <typename T>
-__global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
-                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d,
-                            __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
+__device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t head_stride, int rows_cap,
+                                               const int32_t* count, int count_is_occ, int N,
+                                               float* __restrict__ out, int64_t out_hs, int d,
+                                               __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
   const int h = blockIdx.y;
   const int row0 = (blockIdx.x * (blockDim.x / 32) + warp_id()) * NR_ROWS;
   const int n = min(count_is_occ ? count[h] : N, rows_cap);
@@ -154,6 +167,33 @@ __global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int ro
       ext[(int64_t)h * ext_hs + (int64_t)row * 32 + l] = v;
     }
   }
+}
+
+template <typename T>
+__global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
+                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d,
+                            __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
+  row_norms_body<T>(K, head_stride, rows_cap, count, count_is_occ, N, out, out_hs, d, ext, ext_hs, goff);
+}
+
+// First kernel of an update: the candidates' norms and extension rows, the zeroed
+// crossing histogram, and the update snapshot (prepare_body) in one extra block (last x,
+// head 0); the three share no data.
+template <typename T>
+__global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, int N, int64_t step, float goff) {
+  if (blockIdx.x == gridDim.x - 1) {
+    if (blockIdx.y == 0) prepare_body(b, w, N, step);
+    return;
+  }
+  {
+    const int64_t nh = (int64_t)b.H * w.hist_stride;
+    const int64_t nthr = (int64_t)(gridDim.x - 1) * gridDim.y * blockDim.x;
+    for (int64_t i = ((int64_t)blockIdx.y * (gridDim.x - 1) + blockIdx.x) * blockDim.x + threadIdx.x; i < nh;
+         i += nthr)
+      w.hist[i] = 0;
+  }
+  row_norms_body<T>(Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm, b.n_max, b.d, (__nv_bfloat16*)w.cext,
+                    (int64_t)b.n_max * 32, goff);
 }
 
 // Sort of the keys (fkey(score) << 32 | source index) per head: ascending score, equal
@@ -244,58 +284,69 @@ __device__ __forceinline__ int run_rank(const unsigned long long* r, unsigned lo
 
 // Phase 2: block (a, h) places the keys of run a: final position = index in run a plus
 // the number of smaller keys in every other run (keys are unique, so positions are
-// distinct and cover [0, N)).
-__global__ void __launch_bounds__(RUN) k_sort_rank(Ws w, int n_max, int identity) {
+// distinct and cover [0, N)).  The block then copies its candidates' keys, norms and
+// extension rows to their positions (the operand of the prefix passes in pi order).
+// Source order (empty bank, or the source-order policy): position = source index.
+__global__ void __launch_bounds__(RUN) k_sort_rank(Bank bk, Ws w, const char* __restrict__ Kc, int esize,
+                                                   int identity) {
   extern __shared__ unsigned long long runs[];
+  __shared__ int s_pos[RUN], s_src[RUN];
   const int h = blockIdx.y;
   const int N = w.L->N;
-  if (w.hd[h].empty || identity) return;
+  const int64_t hn = (int64_t)h * bk.n_max;
   const int nruns = (N + RUN - 1) / RUN;
   const int a = blockIdx.x;
   if (a >= nruns) return;                         // block-uniform
-  const unsigned long long* src = w.sortbuf + (int64_t)h * w.sort_stride;
-  for (int i = threadIdx.x; i < nruns * RUN / 2; i += RUN)
-    reinterpret_cast<ulonglong2*>(runs)[i] = reinterpret_cast<const ulonglong2*>(src)[i];
-  __syncthreads();
   const int t = threadIdx.x;
-  const unsigned long long x = runs[a * RUN + t];
-  if (x == ~0ull) return;                         // padding of the last run
-  int pos = t;
-  int b = 0;
-  for (; b + 4 <= nruns; b += 4) {
-    int c[4];
+  const bool ident = w.hd[h].empty || identity;
+  int nvalid;
+  if (ident) {
+    s_pos[t] = s_src[t] = a * RUN + t;
+    nvalid = min(RUN, N - a * RUN);
+  } else {
+    const unsigned long long* src = w.sortbuf + (int64_t)h * w.sort_stride;
+    for (int i = t; i < nruns * RUN / 2; i += RUN)
+      reinterpret_cast<ulonglong2*>(runs)[i] = reinterpret_cast<const ulonglong2*>(src)[i];
+    __syncthreads();
+    const unsigned long long x = runs[a * RUN + t];
+    nvalid = min(RUN, N - a * RUN);               // padding (~0) sorts to the end of the last run
+    int pos = t;
+    if (t < nvalid) {
+      int b = 0;
+      for (; b + 4 <= nruns; b += 4) {
+        int c[4];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) c[u] = b + u == a ? 0 : run_rank(runs + (b + u) * RUN, x);
-    pos += (c[0] + c[1]) + (c[2] + c[3]);
-  }
-  for (; b < nruns; ++b)
-    if (b != a) pos += run_rank(runs + b * RUN, x);
-  if (pos >= N) {
-    dev_fail(w.L, DEV_INCONSISTENT, 8800 + h);
-    return;
-  }
-  w.perm[(int64_t)h * n_max + pos] = (int32_t)(x & 0xffffffffu);
-}
-
-__global__ void k_permute(Bank b, Ws w, const char* __restrict__ Kc, int N, int esize) {
-  const int h = blockIdx.y;
-  const int rb = b.d * esize;
-  const int64_t hn = (int64_t)h * b.n_max;
-  const int32_t* perm = w.perm + hn;
-  const int kg = rb / 64;                      // key groups; then one extension group
-  copy_groups(N, kg + 1, [&](int j, int grp) -> Group4 {
-    const int src = perm[j];
-    if (src < 0 || src >= N) {   // pi must be a permutation of [0, N)
-      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 8000 + h);
-      return {nullptr, nullptr};
+        for (int u = 0; u < 4; ++u) c[u] = b + u == a ? 0 : run_rank(runs + (b + u) * RUN, x);
+        pos += (c[0] + c[1]) + (c[2] + c[3]);
+      }
+      for (; b < nruns; ++b)
+        if (b != a) pos += run_rank(runs + b * RUN, x);
+      if (pos >= N || x == ~0ull) {
+        dev_fail(w.L, DEV_INCONSISTENT, 8800 + h);
+        pos = -1;
+      } else {
+        w.perm[hn + pos] = (int32_t)(x & 0xffffffffu);
+      }
     }
-    if (grp < kg)
-      return {reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb) + 4 * grp,
-              reinterpret_cast<uint4*>((char*)w.kperm + (hn + j) * rb) + 4 * grp};
-    w.kperm_norm[hn + j] = w.cnorm[hn + src];
-    return {reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64),
-            reinterpret_cast<uint4*>((char*)w.kperm_ext + (hn + j) * 64)};
-  });
+    s_pos[t] = pos;
+    s_src[t] = (int)(x & 0xffffffffu);
+  }
+  __syncthreads();
+  const int rb = bk.d * esize;
+  const int kg = rb / 64;                         // key groups; then one extension group
+  for (int c = t; c < nvalid * (kg + 1); c += RUN) {
+    const int row = c / (kg + 1), grp = c - row * (kg + 1);
+    const int pos = s_pos[row], src = s_src[row];
+    if (pos < 0 || src < 0 || src >= N) continue;   // reported above
+    if (grp < kg) {
+      copy64(reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb) + 4 * grp,
+             reinterpret_cast<uint4*>((char*)w.kperm + (hn + pos) * rb) + 4 * grp);
+    } else {
+      w.kperm_norm[hn + pos] = w.cnorm[hn + src];
+      copy64(reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64),
+             reinterpret_cast<uint4*>((char*)w.kperm_ext + (hn + pos) * 64));
+    }
+  }
 }
 
 // Per head: c_r = #{i : cross_i <= r} and feasibility c_r <= e_r for r in [0, rmax].
@@ -661,100 +712,93 @@ __global__ void k_inv_base(Bank b, Ws w) {
     w.invb[(int64_t)h * w.invb_stride + i] = __frcp_rn(b.base[(int64_t)h * b.M_max + i]);
 }
 
-// Keys of the surviving states (rows of Eq. C.4's subtraction) and of the evicted
-// states (its columns), copied before the commit overwrites the evicted slots.
-__global__ void k_gather(Bank b, Ws w, int esize) {
-  const int h = blockIdx.y;
-  const DevHead hd = w.hd[h];
-  if (hd.empty || hd.e == 0) return;
-  const int rb = b.d * esize;
-  const int64_t bh = (int64_t)h * b.M_max;
-  const int64_t hn = (int64_t)h * b.n_max;
-  const int ns = hd.m_old - hd.e;
-  // rows [0, ns) survivors, [ns, ns + e) evicted
-  const int kg = rb / 64;
-  copy_groups(ns + hd.e, kg + 1, [&](int row, int grp) -> Group4 {
-    const bool surv = row < ns;
-    const int slot = surv ? w.surv_list[bh + row] : w.evict_list[hn + row - ns];
-    if (slot < 0 || slot >= hd.m_old) {
-      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
-      return {nullptr, nullptr};
-    }
-    if (grp < kg) {
-      char* dk = surv ? (char*)w.ksurv + (bh + row) * rb : (char*)w.kevict + (hn + row - ns) * rb;
-      return {reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb) + 4 * grp,
-              reinterpret_cast<uint4*>(dk) + 4 * grp};
-    }
-    if (surv) w.ksurv_norm[bh + row] = b.knorm[bh + slot];
-    else w.kevict_norm[hn + row - ns] = b.knorm[bh + slot];
-    char* dx = surv ? (char*)w.ksurv_ext + (bh + row) * 64 : (char*)w.kevict_ext + (hn + row - ns) * 64;
-    return {reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64), reinterpret_cast<uint4*>(dx)};
-  });
-}
-
-// Eq. 12: the j-th admitted candidate (pi order) goes to the j-th evicted slot, the
-// rest are appended after the old occupancy; keys and values are copied bit for bit.
+// Eq. 12 and the copies Eq. C.4 needs, in one pass.  Rows [0, ns) (only if e > 0): the
+// surviving states' keys are copied to the workspace (rows of the subtraction).  Then j:
+// for j < e the evicted slot's old key is copied out (columns of the subtraction) and,
+// by the same thread, the j-th admitted candidate (pi order) is written over it; the
+// admitted candidates j >= e are appended after the old occupancy.  Keys and values
+// are copied bit for bit.  An evicted slot is read and overwritten by one thread in
+// program order, appended slots lie above every survivor, so no slot is written while
+// another thread still reads it.
 __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int esize) {
   const int h = blockIdx.y;
   const DevHead hd = w.hd[h];
   const int64_t bh = (int64_t)h * b.M_max;
   const int64_t hn = (int64_t)h * b.n_max;
+  const int ns = hd.m_old - hd.e;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
-    const int m_new = hd.m_old - hd.e + hd.r;
+    const int m_new = ns + hd.r;
     w.hd[h].m_new = m_new;
     b.occ[h] = m_new;
-    if (m_new > hd.M) dev_fail(w.L, DEV_INCONSISTENT, 4000 + h);
+    if (m_new > hd.M || hd.e > hd.r) dev_fail(w.L, DEV_INCONSISTENT, 4000 + h);
   }
   const int rb = b.d * esize;
-  const int kg = rb / 64;   // per admitted row: key groups, value groups, one extension group
-  copy_groups(hd.r, 2 * kg + 1, [&](int j, int grp) -> Group4 {
+  const int kg = rb / 64;          // per row: key groups, value groups, one extension group
+  const int per_row = 2 * kg + 1;
+  // survivors are operands of the subtraction only when something is evicted (select
+  // lists them only then)
+  const int ng = hd.e > 0 ? ns : 0;
+  const int total = (ng + hd.r) * per_row;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
+    const int row = c / per_row, grp = c - row * per_row;
+    if (row < ng) {
+      // surviving state: key and its derived rows to the workspace (no values)
+      const int slot = w.surv_list[bh + row];
+      if (slot < 0 || slot >= hd.m_old) {
+        if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
+        continue;
+      }
+      if (grp < kg) {
+        copy64(reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb) + 4 * grp,
+               reinterpret_cast<uint4*>((char*)w.ksurv + (bh + row) * rb) + 4 * grp);
+      } else if (grp == 2 * kg) {
+        w.ksurv_norm[bh + row] = b.knorm[bh + slot];
+        copy64(reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64),
+               reinterpret_cast<uint4*>((char*)w.ksurv_ext + (bh + row) * 64));
+      }
+      continue;
+    }
+    const int j = row - ng;
     const int slot = j < hd.e ? w.evict_list[hn + j] : hd.m_old + (j - hd.e);
-    if (slot < 0 || slot >= hd.M) {
-      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
-      return {nullptr, nullptr};
-    }
     const int src = w.perm[hn + j];
-    if (src < 0 || src >= N) {
-      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 8500 + h);
-      return {nullptr, nullptr};
+    if (slot < 0 || slot >= hd.M || (j < hd.e && slot >= hd.m_old) || src < 0 || src >= N) {
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 5000 + h);
+      continue;
     }
-    if (grp < kg)
-      return {reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb) + 4 * grp,
-              reinterpret_cast<uint4*>((char*)b.k + (bh + slot) * rb) + 4 * grp};
-    if (grp < 2 * kg)
-      return {reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg),
-              reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb) + 4 * (grp - kg)};
-    b.knorm[bh + slot] = w.kperm_norm[hn + j];
-    b.prov_step[bh + slot] = w.L->step;
-    b.prov_src[bh + slot] = src;
-    w.slot_new[hn + j] = slot;
-    return {reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64),
-            reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64)};
-  });
+    if (grp < kg) {
+      uint4* dst = reinterpret_cast<uint4*>((char*)b.k + (bh + slot) * rb) + 4 * grp;
+      if (j < hd.e) copy64(dst, reinterpret_cast<uint4*>((char*)w.kevict + (hn + j) * rb) + 4 * grp);
+      copy64(reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb) + 4 * grp, dst);
+    } else if (grp < 2 * kg) {
+      copy64(reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg),
+             reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb) + 4 * (grp - kg));
+    } else {
+      uint4* dx = reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64);
+      if (j < hd.e) {
+        w.kevict_norm[hn + j] = b.knorm[bh + slot];
+        copy64(dx, reinterpret_cast<uint4*>((char*)w.kevict_ext + (hn + j) * 64));
+      }
+      b.knorm[bh + slot] = w.kperm_norm[hn + j];
+      b.prov_step[bh + slot] = w.L->step;
+      b.prov_src[bh + slot] = src;
+      w.slot_new[hn + j] = slot;
+      copy64(reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64), dx);
+    }
+  }
 }
 
 }  // namespace
 
-cudaError_t launch_prepare(const Bank& b, const Ws& w, int N, int64_t step, cudaStream_t s, Timer* t) {
-  timer_begin(t, "prepare", s);
-  k_prepare<<<1, 256, 0, s>>>(b, w, N, step);
-  timer_end(t, s);
-  return cudaGetLastError();
-}
-
 static float ext_goff(const KParams& kp) { return kp.eps * 0.5f / kp.inv_s2; }   // eps sigma^2 / 2
 
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
-                              Timer* t) {
-  dim3 grid((N + 8 * NR_ROWS - 1) / (8 * NR_ROWS), b.H);
-  __nv_bfloat16* ext = (__nv_bfloat16*)w.cext;
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
+                              cudaStream_t s, Timer* t) {
+  dim3 grid((N + 8 * NR_ROWS - 1) / (8 * NR_ROWS) + 1, b.H);   // + the prepare block
   timer_begin(t, "cand_norms", s);
   if (b.bf16)
-    k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)Kc, (int64_t)N * b.d, N, nullptr, 0, N,
-                                                    w.cnorm, b.n_max, b.d, ext, (int64_t)b.n_max * 32, ext_goff(kp));
+    k_cand_prepare<__nv_bfloat16><<<grid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, N, step, ext_goff(kp));
   else
-    k_row_norms<float><<<grid, 256, 0, s>>>((const float*)Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm,
-                                            b.n_max, b.d, ext, (int64_t)b.n_max * 32, ext_goff(kp));
+    k_cand_prepare<float><<<grid, 256, 0, s>>>(b, w, (const float*)Kc, N, step, ext_goff(kp));
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -780,19 +824,12 @@ cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_sort(const Bank& b, const Ws& w, int identity, cudaStream_t s, Timer* t) {
+cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t) {
   const int max_runs = (b.n_max + RUN - 1) / RUN;
   timer_begin(t, "sort", s);
   k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max, identity);
-  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(w, b.n_max, identity);
-  timer_end(t, s);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_permute(const Bank& b, const Ws& w, const void* Kc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N * (b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
-  timer_begin(t, "permute", s);
-  k_permute<<<grid, 256, 0, s>>>(b, w, (const char*)Kc, N, b.bf16 ? 2 : 4);
+  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(b, w, (const char*)Kc,
+                                                                           b.bf16 ? 2 : 4, identity);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -811,16 +848,9 @@ cudaError_t launch_select(const Bank& b, const Ws& w, int eviction, cudaStream_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather(const Bank& b, const Ws& w, cudaStream_t s, Timer* t) {
-  dim3 grid((b.M_max * (b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
-  timer_begin(t, "gather", s);
-  k_gather<<<grid, 256, 0, s>>>(b, w, b.bf16 ? 2 : 4);
-  timer_end(t, s);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t) {
-  dim3 grid((N * (2 * b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
+  // rows: ns survivors + r admitted = m_new <= M_max per head (grid-stride beyond)
+  dim3 grid((b.M_max * (2 * b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
   timer_begin(t, "commit", s);
   k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4);
   timer_end(t, s);

@@ -73,6 +73,8 @@ SIGNATURES = [
     ("dkv_bank_reset", _I, [_P, _P]),
     ("dkv_bank_admit", _I, [_P, _P, _P, _I, ctypes.c_int64, _P]),
     ("dkv_bank_compress", _I, [_P, _P]),
+    ("dkv_bank_evict", _I, [_P, _P]),
+    ("dkv_bank_commit", _I, [_P, _P]),
     ("dkv_bank_attend", _I, [_P, _P, _I, _P, _P, _I, _P, _P]),
     ("dkv_bank_import", _I, [_P, ctypes.POINTER(ctypes.c_int32), _P]),
     ("dkv_bank_sync", _I, [_P]),
@@ -176,6 +178,14 @@ def dkv_bank_admit(bank: int, Kc, Vc, N: int, step: int, stream=None) -> None:
 
 def dkv_bank_compress(bank: int, stream=None) -> None:
     _check(lib().dkv_bank_compress(bank, _stream(stream)), "dkv_bank_compress")
+
+
+def dkv_bank_evict(bank: int, stream=None) -> None:
+    _check(lib().dkv_bank_evict(bank, _stream(stream)), "dkv_bank_evict")
+
+
+def dkv_bank_commit(bank: int, stream=None) -> None:
+    _check(lib().dkv_bank_commit(bank, _stream(stream)), "dkv_bank_commit")
 
 
 def dkv_bank_attend(bank: int, Q, Nq: int, Kw, Vw, W: int, O, stream=None) -> None:
@@ -326,11 +336,19 @@ class BankLayer:
         N = Kc.shape[1]
         self._chk(Kc, (self.H, N, self.d), "Kc")
         self._chk(Vc, (self.H, N, self.d), "Vc")
-        self._pending = (Kc, Vc)   # keep the candidates alive until compress
+        self._pending = (Kc, Vc)   # keep the candidates alive until commit
         dkv_bank_admit(self.handle, Kc, Vc, N, step, stream)
 
     def compress(self, stream=None):
         dkv_bank_compress(self.handle, stream)
+
+    def evict(self, stream=None):
+        """First half of compress; leaves k, v and occupancy untouched."""
+        dkv_bank_evict(self.handle, stream)
+
+    def commit(self, stream=None):
+        """Second half of compress; order every reader of the old bank before it."""
+        dkv_bank_commit(self.handle, stream)
 
     def update(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):
         self.admit(Kc, Vc, step, stream)

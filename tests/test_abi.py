@@ -38,8 +38,8 @@ def _declared_functions():
 
 def test_header_declares_the_hot_path():
     names = _declared_functions()
-    for required in ("dkv_bank_create", "dkv_bank_admit", "dkv_bank_compress", "dkv_bank_attend",
-                     "dkv_bank_destroy", "dkv_bank_workspace_size"):
+    for required in ("dkv_bank_create", "dkv_bank_admit", "dkv_bank_compress", "dkv_bank_evict",
+                     "dkv_bank_commit", "dkv_bank_attend", "dkv_bank_destroy", "dkv_bank_workspace_size"):
         assert required in names
 
 
@@ -107,6 +107,8 @@ def test_host_only_entry_points():
     assert L.dkv_bank_create(ctypes.byref(h), 2, 64, None, 16, 1, None, None) == 1
     assert L.dkv_bank_admit(None, None, None, 1, 0, None) == 1
     assert L.dkv_bank_compress(None, None) == 1
+    assert L.dkv_bank_evict(None, None) == 1
+    assert L.dkv_bank_commit(None, None) == 1
     assert L.dkv_bank_attend(None, None, 1, None, None, 0, None, None) == 1
     assert L.dkv_bank_sync(None) == 1
     L.dkv_bank_destroy(None)

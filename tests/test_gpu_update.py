@@ -203,6 +203,72 @@ def test_call_order_and_argument_errors(dkv):
     bank.close()
 
 
+def test_evict_commit_split_matches_compress(dkv):
+    """Evict then commit, with the step's attention on a second stream ordered only before
+    the commit, leaves every bank buffer bit-identical to compress, and that attention
+    reads the pre-update bank (bit-identical to attention launched before compress)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=96, W=64, Nq=80, budgets=200, steps=7)
+    A = _bank(dkv, wl, dkv.DKV_SCORE_TENSOR)
+    B = _bank(dkv, wl, dkv.DKV_SCORE_TENSOR)
+    ro = synth.LayerRollout(wl, 0)
+    side = torch.cuda.Stream()
+    cur = torch.cuda.current_stream()
+    for t in range(wl.steps):
+        Q = to_dev(ro.queries(t), A.dtype)
+        Kw, Vw = (to_dev(x, A.dtype) for x in ro.window(t))
+        b = wl.admitted_block(t)
+        oa = A.attend(Q, Kw, Vw)
+        if b is not None:
+            K, V = (to_dev(x, A.dtype) for x in ro.block(b))
+            A.admit(K, V, b)
+            A.compress()
+        go = torch.cuda.Event()
+        go.record(cur)
+        side.wait_event(go)
+        ob = torch.empty_like(oa)
+        B.attend(Q, Kw, Vw, out=ob, stream=side)
+        done = torch.cuda.Event()
+        done.record(side)
+        if b is not None:
+            B.admit(K, V, b, stream=cur)
+            B.evict(stream=cur)
+        cur.wait_event(done)
+        if b is not None:
+            B.commit(stream=cur)
+        torch.cuda.synchronize()
+        A.sync()
+        B.sync()
+        assert torch.equal(oa, ob), t
+        for name in ("k", "v", "rho", "base", "knorm", "prov_step", "prov_src", "occupancy"):
+            assert torch.equal(getattr(A, name), getattr(B, name)), (t, name)
+    assert min(A.occupancy_host()) > 0
+    A.close()
+    B.close()
+
+
+def test_evict_commit_call_order(dkv):
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=16, budgets=32)
+    bank = _bank(dkv, wl, dkv.DKV_SCORE_FP32)
+    K = torch.zeros(2, 16, 128, dtype=torch.bfloat16, device="cuda")
+    for call in (bank.evict, bank.commit):          # nothing admitted
+        with pytest.raises(dkv.DkvError) as e:
+            call()
+        assert e.value.status == 3
+    bank.admit(K, K, 0)
+    with pytest.raises(dkv.DkvError) as e:          # commit needs evict first
+        bank.commit()
+    assert e.value.status == 3
+    bank.evict()
+    for call in (bank.evict, bank.compress, lambda: bank.admit(K, K, 1), lambda: bank.import_state([0, 0])):
+        with pytest.raises(dkv.DkvError) as e:
+            call()
+        assert e.value.status == 3
+    bank.commit()
+    bank.sync()
+    assert bank.occupancy_host() == [16, 16]
+    bank.close()
+
+
 def test_device_error_word_reports_inconsistent_bank(dkv):
     """A bank whose occupancy exceeds its budget (written behind the library's back) is
     reported by dkv_bank_sync as a device-side consistency failure, and the handle stays usable."""
