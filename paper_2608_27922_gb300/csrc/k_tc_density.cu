@@ -93,69 +93,65 @@ __device__ __forceinline__ float term1(float a) {
   return P == 2 ? r2 : r2 * r2;
 }
 
-// Two interactions a, b < 0 under one reciprocal R = 1 / (a b):
-//   |a|^-P + |b|^-P          (term2x2)
-//   wa |a|^-P + wb |b|^-P    (term2wx2)
-// in packed fp32x2 arithmetic: lane l of X and Y holds one pair (a, b), and each lane
-// rounds exactly like the scalar expression.
+// Two interactions X, Y < 0 share one reciprocal R = 1 / (X Y):
+//   |X|^-2 + |Y|^-2 = (X^2 + Y^2) R^2,   wX |X|^-2 + wY |Y|^-2 = (wX Y^2 + wY X^2) R^2,
+// in packed fp32x2 arithmetic (lane l of X and Y holds one pair; each lane rounds
+// exactly like the scalar expression), the last multiply fused into the accumulation:
+// acc += |X|^-P + |Y|^-P per lane.  For P = 1 the accumulator collects
+// (X + Y) / (X Y) = -(|X|^-1 + |Y|^-1); the caller negates the chunk total.
 template <int P>
-__device__ __forceinline__ float2 term2x2(float2 X, float2 Y) {
+__device__ __forceinline__ float2 acc2x2(float2 X, float2 Y, float2 acc) {
   const float2 Pm = __fmul2_rn(X, Y);
   const float2 R = make_float2(rcp_approx(Pm.x), rcp_approx(Pm.y));
-  if (P == 1) {
-    const float2 T = __fmul2_rn(__fadd2_rn(X, Y), R);
-    return make_float2(-T.x, -T.y);
-  }
+  if (P == 1) return __ffma2_rn(R, __fadd2_rn(X, Y), acc);
   const float2 R2 = __fmul2_rn(R, R);
-  if (P == 2) return __fmul2_rn(R2, __ffma2_rn(X, X, __fmul2_rn(Y, Y)));
+  if (P == 2) return __ffma2_rn(R2, __ffma2_rn(X, X, __fmul2_rn(Y, Y)), acc);
   const float2 X2 = __fmul2_rn(X, X), Y2 = __fmul2_rn(Y, Y);
-  return __fmul2_rn(__fmul2_rn(R2, R2), __ffma2_rn(X2, X2, __fmul2_rn(Y2, Y2)));
+  return __ffma2_rn(__fmul2_rn(R2, R2), __ffma2_rn(X2, X2, __fmul2_rn(Y2, Y2)), acc);
 }
 
+// acc += wX |X|^-P + wY |Y|^-P per lane (same conventions).
 template <int P>
-__device__ __forceinline__ float2 term2wx2(float2 X, float2 Y, float2 WX, float2 WY) {
+__device__ __forceinline__ float2 acc2wx2(float2 X, float2 Y, float2 WX, float2 WY, float2 acc) {
   const float2 Pm = __fmul2_rn(X, Y);
   const float2 R = make_float2(rcp_approx(Pm.x), rcp_approx(Pm.y));
-  if (P == 1) {
-    const float2 T = __fmul2_rn(R, __ffma2_rn(WX, Y, __fmul2_rn(WY, X)));
-    return make_float2(-T.x, -T.y);
-  }
+  if (P == 1) return __ffma2_rn(R, __ffma2_rn(WX, Y, __fmul2_rn(WY, X)), acc);
   const float2 R2 = __fmul2_rn(R, R);
-  if (P == 2) return __fmul2_rn(R2, __ffma2_rn(WX, __fmul2_rn(Y, Y), __fmul2_rn(WY, __fmul2_rn(X, X))));
+  if (P == 2) return __ffma2_rn(R2, __ffma2_rn(WX, __fmul2_rn(Y, Y), __fmul2_rn(WY, __fmul2_rn(X, X))), acc);
   const float2 X2 = __fmul2_rn(X, X), Y2 = __fmul2_rn(Y, Y);
-  return __fmul2_rn(__fmul2_rn(R2, R2), __ffma2_rn(WX, __fmul2_rn(Y2, Y2), __fmul2_rn(WY, __fmul2_rn(X2, X2))));
-}
-
-// Fixed-order binary tree over 8 packed values, then the two lanes.
-__device__ __forceinline__ float tree8x2(float2 (&t)[8]) {
-#pragma unroll
-  for (int s = 4; s > 0; s >>= 1)
-#pragma unroll
-    for (int k = 0; k < s; ++k) t[k] = __fadd2_rn(t[k], t[k + s]);
-  return t[0].x + t[0].y;
+  return __ffma2_rn(__fmul2_rn(R2, R2), __ffma2_rn(WX, __fmul2_rn(Y2, Y2), __fmul2_rn(WY, __fmul2_rn(X2, X2))),
+                    acc);
 }
 
 // Sum of |v_j|^-P over a full 32-column chunk: column j shares a reciprocal with
-// column j + 16.
+// column j + 16; two packed accumulators (even and odd pairs), added at the end.
 template <int P>
 __device__ __forceinline__ float chunk_sum(const float (&v)[32]) {
-  float2 t[8];
+  float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int k = 0; k < 8; ++k)
-    t[k] = term2x2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]));
-  return tree8x2(t);
+  for (int k = 0; k < 8; k += 2) {
+    a0 = acc2x2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]), a0);
+    a1 = acc2x2<P>(make_float2(v[2 * k + 2], v[2 * k + 3]), make_float2(v[2 * k + 18], v[2 * k + 19]), a1);
+  }
+  const float2 a = __fadd2_rn(a0, a1);
+  return P == 1 ? -(a.x + a.y) : a.x + a.y;
 }
 
-// Sum of wb_j |v_j|^-P over a full 32-column chunk (wb in shared memory, 8-byte aligned).
+// Sum of wb_j |v_j|^-P over a full 32-column chunk (wb in shared memory, 16-byte aligned).
 template <int P>
 __device__ __forceinline__ float chunk_sum_w(const float (&v)[32], const float* wb) {
-  const float2* w2 = reinterpret_cast<const float2*>(wb);
-  float2 t[8];
+  const float4* w4 = reinterpret_cast<const float4*>(wb);
+  float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int k = 0; k < 8; ++k)
-    t[k] = term2wx2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]), w2[k],
-                       w2[k + 8]);
-  return tree8x2(t);
+  for (int k = 0; k < 8; k += 2) {
+    const float4 wx = w4[k / 2], wy = w4[4 + k / 2];
+    a0 = acc2wx2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]),
+                    make_float2(wx.x, wx.y), make_float2(wy.x, wy.y), a0);
+    a1 = acc2wx2<P>(make_float2(v[2 * k + 2], v[2 * k + 3]), make_float2(v[2 * k + 18], v[2 * k + 19]),
+                    make_float2(wx.z, wx.w), make_float2(wy.z, wy.w), a1);
+  }
+  const float2 a = __fadd2_rn(a0, a1);
+  return P == 1 ? -(a.x + a.y) : a.x + a.y;
 }
 
 // Same over the first `lim` columns (lim < 32), term by term.
