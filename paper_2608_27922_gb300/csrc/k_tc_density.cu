@@ -61,11 +61,12 @@ constexpr int OFF_A = 0;
 constexpr int OFF_AX = TILE_BYTES;
 constexpr int OFF_B = OFF_AX + EXT_BYTES;                 // [STAGES] tiles
 constexpr int OFF_BX = OFF_B + STAGES * TILE_BYTES;       // [STAGES] extension tiles
-constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [2][BN]
-constexpr int OFF_XCH = OFF_META + 2 * BN * 4;            // float [2][2][BM]
+constexpr int META_BUFS = 4;                              // score weights of tiles t, t+1, t+2, t+3
+constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [META_BUFS][BN]
+constexpr int OFF_XCH = OFF_META + META_BUFS * BN * 4;    // float [2][2][BM]
 constexpr int OFF_FLAG = OFF_XCH + 2 * 2 * BM * 4;      // int: last-arrival flag of split tiles
 constexpr int OFF_BAR = OFF_FLAG + 16;
-constexpr size_t SMEM_BYTES = 1024 + OFF_BAR + 128;
+constexpr size_t SMEM_BYTES = OFF_BAR + 128;              // base 1024-aligned (checked)
 constexpr uint32_t LOAD_BYTES = TILE_BYTES + EXT_BYTES;
 
 struct TcJob {
@@ -178,19 +179,24 @@ template <int MODE, int P>
 __global__ void __launch_bounds__(THREADS, 2)
     tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
              const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx, TcJob j) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0u) {   // 128-byte-swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9900);
+    return;
+  }
+  uint8_t* smem = smem_raw;
   float* meta = reinterpret_cast<float*>(smem + OFF_META);
   float* xch = reinterpret_cast<float*>(smem + OFF_XCH);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* bar_a = bars + 0;
-  uint64_t* bar_full = bars + 1;    // [STAGES]
-  uint64_t* bar_empty = bars + 3;   // [STAGES]
-  uint64_t* bar_accf = bars + 5;    // [2]
-  uint64_t* bar_acce = bars + 7;    // [2]
+  // ready[b]: column tile t (b = t & 1) has landed AND the epilogue has released
+  // accumulator b (tile t - 2): the MMA issuer's only wait per tile
+  uint64_t* bar_rdy = bars + 1;     // [2]
+  uint64_t* bar_empty = bars + 3;   // [STAGES] MMA of the stage's tile complete
+  uint64_t* bar_accf = bars + 5;    // [2] accumulator b complete
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
-  uint64_t* bar_meta = bars + 10;   // [2] SCORE: 1 / b of the columns of accumulator b
+  uint64_t* bar_meta = bars + 10;   // [META_BUFS] SCORE: 1 / b of the columns of tile t (t % 4)
 
   const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
@@ -210,12 +216,12 @@ __global__ void __launch_bounds__(THREADS, 2)
 
   if (threadIdx.x == 0) {
     mbar_init(bar_a, 1);
-    for (int s = 0; s < STAGES; ++s) { mbar_init(bar_full + s, 1); mbar_init(bar_empty + s, 1); }
+    for (int s = 0; s < STAGES; ++s) mbar_init(bar_empty + s, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_accf + b, 1);
-      mbar_init(bar_acce + b, EPI_WARPS);
-      mbar_init(bar_meta + b, 1);
+      mbar_init(bar_rdy + b, EPI_WARPS + 1);   // the epilogue warps + the producer (with bytes)
     }
+    for (int q = 0; q < META_BUFS; ++q) mbar_init(bar_meta + q, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -235,25 +241,45 @@ __global__ void __launch_bounds__(THREADS, 2)
       tma_load_3d(smem + OFF_AX, &tmAx, bar_a, 0, row0, h);
       int issued = 0;
       for (int t = 0; t < ntiles; ++t) {
-        const int s = t % STAGES;
+        const int s = t % STAGES;   // == t & 1, the accumulator of tile t
+        // MMA(t - 2) complete: stage s is free, and (it waited for ready) the epilogue of
+        // tile t - 4 has finished with meta buffer t % 4
         if (!mbar_wait(bar_empty + s, ((t / STAGES) & 1) ^ 1, abort_flag)) break;
-        mbar_arrive_expect_tx(bar_full + s, LOAD_BYTES);
+        mbar_arrive_expect_tx(bar_rdy + s, LOAD_BYTES);
         const int col = c0 + t * BN;
         uint8_t* dst = smem + OFF_B + s * TILE_BYTES;
-        tma_load_3d(dst, &tmB, bar_full + s, 0, col, h);
-        tma_load_3d(dst + HALF_BYTES, &tmB, bar_full + s, 64, col, h);
-        tma_load_3d(smem + OFF_BX + s * EXT_BYTES, &tmBx, bar_full + s, 16, col, h);
+        tma_load_3d(dst, &tmB, bar_rdy + s, 0, col, h);
+        tma_load_3d(dst + HALF_BYTES, &tmB, bar_rdy + s, 64, col, h);
+        tma_load_3d(smem + OFF_BX + s * EXT_BYTES, &tmBx, bar_rdy + s, 16, col, h);
+        if (MODE == TM_SCORE) {
+          // 1 / b_j of the tile's columns (a whole 128-float row; values past the last
+          // column are not used)
+          const int q = t % META_BUFS;
+          mbar_arrive_expect_tx(bar_meta + q, BN * 4);
+          bulk_load(meta + q * BN, j.w.invb + (int64_t)h * j.w.invb_stride + col, BN * 4, bar_meta + q);
+        }
         issued = t + 1;
       }
       if (issued < ntiles) {
         *abort_flag = 1;
         dev_fail(j.w.L, DEV_TIMEOUT, 100 + MODE);
       }
-      // never leave with copies in flight: wait (bounded) for the last loads issued
+      // never leave with copies in flight: wait (bounded) for the last loads issued.  A
+      // ready phase also needs the epilogue's release, which an aborted CTA may never
+      // give; then wait a fixed 50 us, far longer than any copy takes to land.
       volatile int no_abort = 0;
       mbar_wait(bar_a, 0, &no_abort);
+      bool drained = true;
       for (int t = issued > STAGES ? issued - STAGES : 0; t < issued; ++t)
-        mbar_wait(bar_full + (t % STAGES), (t / STAGES) & 1, &no_abort);
+        drained = drained && mbar_wait(bar_rdy + (t % STAGES), (t / STAGES) & 1, abort_flag);
+      if (MODE == TM_SCORE)
+        for (int t = issued > META_BUFS ? issued - META_BUFS : 0; t < issued; ++t)
+          mbar_wait(bar_meta + (t % META_BUFS), (t / META_BUFS) & 1, &no_abort);
+      if (!drained) {
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 50000ull) {
+        }
+      }
     }
   } else if (warp == 1) {
     if (lane == 0 && ntiles > 0) {
@@ -266,15 +292,9 @@ __global__ void __launch_bounds__(THREADS, 2)
       for (int t = 0; ok && t < ntiles; ++t) {
         const int s = t % STAGES;
         const int b = t & 1;
-        if (!(ok = mbar_wait(bar_full + s, (t / STAGES) & 1, abort_flag))) break;
-        if (!(ok = mbar_wait(bar_acce + b, ((t >> 1) & 1) ^ 1, abort_flag))) break;
+        // one wait per tile: every other wait in this thread stalls the tensor pipe
+        if (!(ok = mbar_wait(bar_rdy + b, (t >> 1) & 1, abort_flag))) break;
         fence_after_sync();
-        if (MODE == TM_SCORE) {
-          // the epilogue of tile t - 2 has released meta[b]: fetch 1 / b_j of tile t
-          // (a whole 128-float row; the values past the last column are not used)
-          mbar_arrive_expect_tx(bar_meta + b, BN * 4);
-          bulk_load(meta + b * BN, j.w.invb + (int64_t)h * j.w.invb_stride + c0 + t * BN, BN * 4, bar_meta + b);
-        }
         const uint32_t b_base = smem_u32(smem + OFF_B + s * TILE_BYTES);
         const uint32_t bx_base = smem_u32(smem + OFF_BX + s * EXT_BYTES);
 #pragma unroll
@@ -295,9 +315,6 @@ __global__ void __launch_bounds__(THREADS, 2)
       if (done > 0) {
         volatile int no_abort = 0;
         mbar_wait(bar_accf + ((done - 1) & 1), ((done - 1) >> 1) & 1, &no_abort);
-        if (MODE == TM_SCORE)
-          for (int t = done > 2 ? done - 2 : 0; t < done; ++t)
-            mbar_wait(bar_meta + (t & 1), (t >> 1) & 1, &no_abort);
       }
     }
   } else {
@@ -333,6 +350,11 @@ __global__ void __launch_bounds__(THREADS, 2)
       }
     }
     if (MODE == TM_CROSS && active && half == 0) snap_row[0] = 0.f;
+    // both accumulators start free: this warp's release for tiles 0 and 1
+    if (lane == 0) {
+      mbar_arrive(bar_rdy + 0);
+      mbar_arrive(bar_rdy + 1);
+    }
 
     bool ok = true;
     for (int t = 0; t < ntiles; ++t) {
@@ -340,7 +362,9 @@ __global__ void __launch_bounds__(THREADS, 2)
       const int col0 = c0 + t * BN;
       const int nc = min(BN, c1 - col0);
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_accf + b, (t >> 1) & 1, abort_flag));
-      if (MODE == TM_SCORE && ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_meta + b, (t >> 1) & 1, abort_flag));
+      if (MODE == TM_SCORE && ok)
+        ok = __all_sync(0xffffffffu,
+                        mbar_wait(bar_meta + t % META_BUFS, (t / META_BUFS) & 1, abort_flag));
       float tot[2] = {0.f, 0.f};
       if (ok) {
         fence_after_sync();
@@ -353,7 +377,7 @@ __global__ void __launch_bounds__(THREADS, 2)
           tmem_wait_ld();
           const int lim = min(32, nc - cs);
           if (MODE == TM_SCORE) {
-            const float* ib = meta + b * BN + cs;
+            const float* ib = meta + (t % META_BUFS) * BN + cs;
             if (lim == 32) {
               tot[ch] = chunk_sum_w<P>(v, ib);
             } else {
@@ -420,7 +444,7 @@ __global__ void __launch_bounds__(THREADS, 2)
       if (ok) {
         fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar_acce + b);
+        if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile t + 2
       }
     }
     if (!ok) {
