@@ -15,6 +15,10 @@
 //   O = (2^(m_0 - m) O_0 + 2^(m_1 - m) O_1) / (2^(m_0 - m) l_0 + 2^(m_1 - m) l_1).
 // Warps: 0 TMA producer, 1 MMA issuer, 2-5 softmax group 0, 6-9 softmax group 1.
 // TMEM columns: S_0 [0,128), O_0 [128,256), S_1 [256,384), O_1 [384,512).
+// The MMA-issuing thread waits once per group and tile (any wait there stalls the
+// tensor pipe): p_full_g completes when the softmax has written P_g(i) AND V(i) and
+// K(i + 1) have landed (the producer arms it with their bytes; K has two slots per
+// group, so K(i + 1) loads while S_g(i) still reads K(i)).
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
@@ -35,11 +39,11 @@ constexpr int HB = TB / 2;              // one 64-column swizzle panel
 constexpr int THREADS = 64 + 256;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int OFF_Q = 0;
-constexpr int OFF_K = TB;               // [2 groups]
-constexpr int OFF_V = 3 * TB;           // [2 groups]
-constexpr int OFF_X = 5 * TB;           // float [2 groups][2 (m, l)][BQ]
+constexpr int OFF_K = TB;               // [2 groups][2 slots]
+constexpr int OFF_V = 5 * TB;           // [2 groups]
+constexpr int OFF_X = 7 * TB;           // float [2 groups][2 (m, l)][BQ]
 constexpr int OFF_BAR = OFF_X + 2 * 2 * BQ * 4;
-constexpr size_t SMEM_BYTES = 1024 + OFF_BAR + 256;
+constexpr size_t SMEM_BYTES = OFF_BAR + 256;   // base 1024-aligned (checked)
 constexpr float RESCALE_LOG2 = 8.0f;
 
 __device__ __forceinline__ float ex2(float x) {
@@ -103,17 +107,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_attend(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKb,
               const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmKw,
               const __grid_constant__ CUtensorMap tmVw, AttnJob j) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0u) {   // 128-byte-swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) dev_fail(j.L, DEV_INCONSISTENT, 9901);
+    return;
+  }
+  uint8_t* smem = smem_raw;
   float* xst = reinterpret_cast<float*>(smem + OFF_X);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;    // [2 groups]
-  uint64_t* k_empty = bars + 3;   // [2]
-  uint64_t* v_full = bars + 5;    // [2]
-  uint64_t* v_empty = bars + 7;   // [2]
+  uint64_t* k0_full = bars + 1;   // [2 groups] first K tile of the group
+  uint64_t* k_empty = bars + 3;   // [2 groups][2 slots] S_g of the slot's tile complete
+  uint64_t* v_empty = bars + 7;   // [2] PV_g complete (V slot free)
   uint64_t* s_full = bars + 9;    // [2]
-  uint64_t* p_full = bars + 11;   // [2]
+  uint64_t* p_full = bars + 11;   // [2] P_g(i) written, V(i) and K(i + 1) landed
   uint64_t* pv_done = bars + 13;  // [2]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 15);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
@@ -130,9 +137,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int g = 0; g < 2; ++g) {
-      mbar_init(k_full + g, 1); mbar_init(k_empty + g, 1);
-      mbar_init(v_full + g, 1); mbar_init(v_empty + g, 1);
-      mbar_init(s_full + g, 1); mbar_init(p_full + g, 4);
+      mbar_init(k0_full + g, 1);
+      mbar_init(k_empty + 2 * g, 1); mbar_init(k_empty + 2 * g + 1, 1);
+      mbar_init(v_empty + g, 1);
+      mbar_init(s_full + g, 1);
+      mbar_init(p_full + g, 4 + 1);   // four softmax warps + the producer (with bytes)
       mbar_init(pv_done + g, 1);
     }
     *abort_flag = 0;
@@ -149,43 +158,61 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0 && nt > 0) {
-      // ---------------- TMA producer: Q once; per group single-buffered K and V
+      // ---------------- TMA producer: Q once; per group K(0), then for each tile i the
+      // bytes of V(i) and K(i + 1) on p_full_g (phase i)
       prefetch_map(&tmQ);
       mbar_arrive_expect_tx(q_full, TB);
       tma_load_3d(smem + OFF_Q, &tmQ, q_full, 0, q0, h);
       tma_load_3d(smem + OFF_Q + HB, &tmQ, q_full, 64, q0, h);
-      int kiss[2] = {0, 0}, viss[2] = {0, 0};
+      const int n[2] = {tiles_of(0), tiles_of(1)};
+      auto load_tile = [&](bool is_k, int g, int i, void* dst, uint64_t* bar) {
+        const int u = tile_index(g, i);
+        const bool bank = u < nb;
+        const CUtensorMap* mp = is_k ? (bank ? &tmKb : &tmKw) : (bank ? &tmVb : &tmVw);
+        const int row = bank ? u * BK : (u - nb) * BK;
+        tma_load_3d(dst, mp, bar, 0, row, h);
+        tma_load_3d(static_cast<uint8_t*>(dst) + HB, mp, bar, 64, row, h);
+      };
+      for (int g = 0; g < 2; ++g)
+        if (n[g] > 0) {
+          mbar_arrive_expect_tx(k0_full + g, TB);
+          load_tile(true, g, 0, smem + OFF_K + (2 * g) * TB, k0_full + g);
+        }
+      int armed[2] = {0, 0};   // p_full phases armed per group
       bool ok = true;
-      const int n0 = tiles_of(0), n1 = tiles_of(1);
-      for (int i = 0; ok && i < n0; ++i) {
+      for (int i = 0; ok && i < n[0]; ++i) {
         for (int g = 0; g < 2 && ok; ++g) {
-          if (i >= (g == 0 ? n0 : n1)) continue;
-          const int u = tile_index(g, i);
-          const bool bank = u < nb;
-          const CUtensorMap* mk = bank ? &tmKb : &tmKw;
-          const CUtensorMap* mv = bank ? &tmVb : &tmVw;
-          const int row = bank ? u * BK : (u - nb) * BK;
-          if (!(ok = mbar_wait(k_empty + g, (i & 1) ^ 1, abort_flag))) break;
-          mbar_arrive_expect_tx(k_full + g, TB);
-          tma_load_3d(smem + OFF_K + g * TB, mk, k_full + g, 0, row, h);
-          tma_load_3d(smem + OFF_K + g * TB + HB, mk, k_full + g, 64, row, h);
-          kiss[g] = i + 1;
-          if (!(ok = mbar_wait(v_empty + g, (i & 1) ^ 1, abort_flag))) break;
-          mbar_arrive_expect_tx(v_full + g, TB);
-          tma_load_3d(smem + OFF_V + g * TB, mv, v_full + g, 0, row, h);
-          tma_load_3d(smem + OFF_V + g * TB + HB, mv, v_full + g, 64, row, h);
-          viss[g] = i + 1;
+          if (i >= n[g]) continue;
+          // PV_g(i - 1) complete: the V slot is free and p_full_g phase i - 1 is over
+          if (i > 0 && !(ok = mbar_wait(v_empty + g, (i - 1) & 1, abort_flag))) break;
+          const bool knext = i + 1 < n[g];
+          // S_g(i - 1) complete: K slot (i + 1) & 1 is free
+          if (knext && i > 0 && !(ok = mbar_wait(k_empty + 2 * g + ((i + 1) & 1), ((i - 1) >> 1) & 1, abort_flag)))
+            break;
+          mbar_arrive_expect_tx(p_full + g, knext ? 2 * TB : TB);
+          load_tile(false, g, i, smem + OFF_V + g * TB, p_full + g);
+          if (knext) load_tile(true, g, i + 1, smem + OFF_K + (2 * g + ((i + 1) & 1)) * TB, p_full + g);
+          armed[g] = i + 1;
         }
       }
       if (!ok) {
         *abort_flag = 1;
         dev_fail(j.L, DEV_TIMEOUT, 400);
       }
+      // never leave with copies in flight: earlier phases completed before this thread
+      // armed the next one; the last armed phase also needs the softmax, which an
+      // aborted CTA may never give: then wait a fixed 50 us, far longer than a copy takes
       volatile int no_abort = 0;
       mbar_wait(q_full, 0, &no_abort);
+      bool drained = true;
       for (int g = 0; g < 2; ++g) {
-        if (kiss[g] > 0) mbar_wait(k_full + g, (kiss[g] - 1) & 1, &no_abort);
-        if (viss[g] > 0) mbar_wait(v_full + g, (viss[g] - 1) & 1, &no_abort);
+        if (n[g] > 0) mbar_wait(k0_full + g, 0, &no_abort);
+        if (armed[g] > 0) drained = drained && mbar_wait(p_full + g, (armed[g] - 1) & 1, abort_flag);
+      }
+      if (!drained) {
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 50000ull) {
+        }
       }
     }
   } else if (warp == 1) {
@@ -198,23 +225,20 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int n[2] = {tiles_of(0), tiles_of(1)};
       bool ok = mbar_wait(q_full, 0, abort_flag);
       int pv_issued[2] = {0, 0};
-      auto issue_s = [&](int g, int i) -> bool {
-        if (!mbar_wait(k_full + g, i & 1, abort_flag)) return false;
-        fence_after_sync();
-        const uint32_t k_base = smem_u32(smem + OFF_K + g * TB);
+      // S_g(i): its K tile has landed (K(0): k0_full; K(i + 1): with p_full_g phase i)
+      auto issue_s = [&](int g, int i) {
+        const uint32_t k_base = smem_u32(smem + OFF_K + (2 * g + (i & 1)) * TB);
         const uint32_t sc = tmem + g * 256;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
           mma_bf16(sc, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
         }
-        mma_commit(k_empty + g);
+        mma_commit(k_empty + 2 * g + (i & 1));
         mma_commit(s_full + g);
-        return true;
       };
       auto issue_pv = [&](int g, int i) -> bool {
-        if (!mbar_wait(p_full + g, i & 1, abort_flag)) return false;
-        if (!mbar_wait(v_full + g, i & 1, abort_flag)) return false;
+        if (!mbar_wait(p_full + g, i & 1, abort_flag)) return false;   // the one wait
         fence_after_sync();
         const uint32_t v_base = smem_u32(smem + OFF_V + g * TB);
         const uint32_t pc = tmem + g * 256;          // P: packed bf16 pairs over S columns [0, 64)
@@ -228,12 +252,17 @@ __global__ void __launch_bounds__(THREADS, 1)
         return true;
       };
       for (int g = 0; g < 2 && ok; ++g)
-        if (n[g] > 0) ok = issue_s(g, 0);
+        if (n[g] > 0) {
+          if ((ok = mbar_wait(k0_full + g, 0, abort_flag))) {
+            fence_after_sync();
+            issue_s(g, 0);
+          }
+        }
       for (int i = 0; ok && i < n[0]; ++i) {
         for (int g = 0; g < 2 && ok; ++g) {
           if (i >= n[g]) continue;
           ok = issue_pv(g, i);
-          if (ok && i + 1 < n[g]) ok = issue_s(g, i + 1);
+          if (ok && i + 1 < n[g]) issue_s(g, i + 1);
         }
       }
       if (!ok) {
