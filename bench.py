@@ -65,7 +65,10 @@ def parse_args():
                     help="bank-reading attention passes per update (denoising passes; the update runs once)")
     ap.add_argument("--layers", type=int, default=1,
                     help="layers updated per step on this GPU (whole-stack throughput; > 1 selects the stack run)")
-    ap.add_argument("--streams", type=int, default=4, help="stream pairs the layers of a stack step spread over")
+    ap.add_argument("--streams", type=int, default=4, help="stream pairs the layers of a stack step spread over "
+                    "(--stack-mode streams)")
+    ap.add_argument("--stack-mode", choices=["grouped", "streams"], default="grouped",
+                    help="grouped: one handle over all layers, single launches; streams: one handle per layer")
     ap.add_argument("--distinct-layers", type=int, default=2,
                     help="stack run: layers with their own synthetic input stream (the rest reuse them)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -628,10 +631,12 @@ def run_reference(args):
 
 def run_stack(args):
     """Whole-stack throughput on one GPU: every step updates `--layers` independent layer
-    banks (attention || admit + evict, then commit, per layer), the layers spread over
-    `--streams` stream pairs and the whole step captured as one CUDA graph.  Inputs of
-    `--distinct-layers` synthetic layer streams are reused round-robin by the others
-    (each layer still has its own bank)."""
+    banks (attention || admit + evict, then commit), the whole step captured as one CUDA
+    graph.  `--stack-mode grouped` (default): one handle holds all layers and every call
+    is a single launch per kernel over all L x H heads (each layer keeps its own r*);
+    `streams`: one handle per layer, the layers spread over `--streams` stream pairs.
+    Inputs of `--distinct-layers` synthetic layer streams are reused round-robin by the
+    others (each layer still has its own bank)."""
     import torch
 
     torch.cuda.set_device(0)
@@ -654,16 +659,57 @@ def run_stack(args):
                        [inp.window(t, blocks, cat1) for t in range(W + K)]))
     P = max(1, args.attn_passes)
     mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
-    banks = [dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(l), wl.N, bf, score_mode=mode, device=dev)
-             for l in range(L)]
-    for bk in banks:
-        bk.reset()
-    outs = [torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev) for _ in range(L)]
+    grouped = args.stack_mode == "grouped"
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
-    mains = [torch.cuda.Stream(dev) for _ in range(S)]
-    sides = [torch.cuda.Stream(dev) for _ in range(S)]
+    if grouped:
+        # one handle holds all L layers (L x H heads, params.layer_heads = H): every call
+        # is one launch per kernel over all layers; the inputs are stacked along heads
+        budgets = [b for l in range(L) for b in wl.budgets_of_layer(l)]
+        banks = [dkv.BankLayer(L * wl.H, wl.d, budgets, wl.N, bf, score_mode=mode, device=dev, layer_heads=wl.H)]
+        banks[0].reset()
+        stack0 = lambda xs: torch.cat(xs, dim=0).contiguous()
+        admitted = sorted({wl.admitted_block(t) for t in range(W + K)} - {None})
+        s_blocks = {b: (stack0([inputs[l % D][0][b][0] for l in range(L)]),
+                        stack0([inputs[l % D][0][b][1] for l in range(L)])) for b in admitted}
+        s_queries = [stack0([inputs[l % D][1][t] for l in range(L)]) for t in range(W + K)]
+        def s_window(t):   # a window that is exactly an admitted block shares its tensors
+            parts = wl.window_parts(t)
+            if len(parts) == 1 and parts[0][1] == 0 and parts[0][2] == wl.N and parts[0][0] in s_blocks:
+                return s_blocks[parts[0][0]]
+            return (stack0([inputs[l % D][2][t][0] for l in range(L)]),
+                    stack0([inputs[l % D][2][t][1] for l in range(L)]))
+        s_windows = [s_window(t) for t in range(W + K)]
+        del inputs
+        out_all = torch.empty(L * wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
+        side = torch.cuda.Stream(dev)
 
-    def stack_step(t):
+        def stack_step(t):
+            cur = torch.cuda.current_stream(dev)
+            b = wl.admitted_block(t)
+            kw, vw = s_windows[t]
+            go = torch.cuda.Event()
+            go.record(cur)
+            side.wait_event(go)
+            for _ in range(P):
+                banks[0].attend(s_queries[t], kw, vw, out=out_all, stream=side)
+            done = torch.cuda.Event()
+            done.record(side)
+            if b is not None:
+                banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
+                banks[0].evict(stream=cur)
+            cur.wait_event(done)
+            if b is not None:
+                banks[0].commit(stream=cur)
+    else:
+        banks = [dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(l), wl.N, bf, score_mode=mode, device=dev)
+                 for l in range(L)]
+        for bk in banks:
+            bk.reset()
+        outs = [torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev) for _ in range(L)]
+        mains = [torch.cuda.Stream(dev) for _ in range(S)]
+        sides = [torch.cuda.Stream(dev) for _ in range(S)]
+
+    def stack_step_streams(t):
         cur = torch.cuda.current_stream(dev)
         fork = torch.cuda.Event()
         fork.record(cur)
@@ -694,6 +740,8 @@ def run_stack(args):
         for j in joins:
             cur.wait_event(j)
 
+    if not grouped:
+        stack_step = stack_step_streams
     stream = torch.cuda.current_stream(dev)
     for t in range(W):
         stack_step(t)
@@ -726,9 +774,10 @@ def run_stack(args):
         if wl.admitted_block(t) is not None:
             per_layer = []
             for bk in banks:
-                Ls, hs = bk.stats()
+                _, hs = bk.stats()
                 keys += sum(h.occupancy_before + wl.N for h in hs)
-                per_layer.append((Ls.r_star, sum(h.evicted for h in hs)))
+                for l, Ls in enumerate(bk.layer_stats()):
+                    per_layer.append((Ls.r_star, sum(h.evicted for h in hs[l * wl.H:(l + 1) * wl.H])))
             rstars.append(per_layer)
     clk = clocks.stop()
     for bk in banks:
@@ -739,10 +788,13 @@ def run_stack(args):
         "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
         "config": {"workload": f"{wl.name}: {L} layer(s) x {wl.H} heads per step, d={wl.d}, N={wl.N}, "
                                f"M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
-                   "score_mode": args.score_mode, "layers_per_gpu": L, "streams": f"{S} stream pairs",
+                   "score_mode": args.score_mode, "layers_per_gpu": L,
+                   "streams": ("one handle over all layers (single launches), attention || admit + evict, "
+                               "then commit" if grouped else f"one handle per layer on {S} stream pairs"),
                    "cuda_graphs": True, "inputs": f"{D} distinct synthetic layer streams, reused round-robin",
                    "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
-                   "parallelism": "layers of one GPU on concurrent streams"},
+                   "parallelism": "layers of one GPU, grouped launches" if grouped
+                   else "layers of one GPU on concurrent streams"},
         "blocks_per_s": K / (total_ms / 1e3),
         "e2e": None, "gpu_launches": None, "roofline": None, "cpu_baseline": None, "clocks": clk,
         "update": {"last_step_r_star_per_layer": [r for r, _ in rstars[-1]] if rstars else [],

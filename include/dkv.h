@@ -111,7 +111,12 @@ typedef struct {
   int32_t refresh_baselines; /* 0: baselines frozen at insertion (Eq. 5, default);
                            1: b = max(rho, delta) for every retained state after each
                            update (App. E "Density baseline" ablation)              */
-  int32_t reserved;     /* must be 0                                                   */
+  int32_t layer_heads;  /* 0: the H heads are one layer.  Else H is a multiple of it and
+                           the handle holds H / layer_heads independent layers of
+                           layer_heads heads each (rows [l * layer_heads, (l + 1) *
+                           layer_heads) of every [H][..] buffer): each layer has its own
+                           shared prefix r* (Eq. 11) and prefix range, and one call
+                           updates or reads all layers with single kernel launches      */
 } dkv_params_t;
 
 /* Caller-owned device buffers of one layer's banks.  M_max = max_h budgets[h];
@@ -237,7 +242,8 @@ dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* st
 dkv_status_t dkv_bank_sync(dkv_bank_t bank);
 
 /* Copies the statistics of the last update to host memory (synchronises with
- * the handle's last stream).  heads may be NULL; else it holds H entries.     */
+ * the handle's last stream).  layer holds one entry per layer (H / layer_heads,
+ * 1 when layer_heads = 0); heads may be NULL, else it holds H entries.        */
 dkv_status_t dkv_bank_stats(dkv_bank_t bank, dkv_layer_stats_t* layer, dkv_head_stats_t* heads);
 
 /* Copies the current per-head occupancy to host memory (synchronises).       */

@@ -101,7 +101,7 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* ba
   };
   const size_t Hh = (size_t)H, Nm = (size_t)n_max, Mm = (size_t)M_max;
   Ws w{};
-  w.L = (DevLayer*)take(sizeof(DevLayer));
+  w.L = (DevLayer*)take(Hh * sizeof(DevLayer));   // room for up to H layers
   w.hd = (DevHead*)take(Hh * sizeof(DevHead));
   w.budgets = (int32_t*)take(Hh * 4);
   w.cnorm = (float*)take(Hh * Nm * 4);
@@ -157,6 +157,7 @@ struct dkv_bank_s {
   std::vector<int32_t> budgets;
   bool tc = false;
   int state = 0;   // 0: idle, 1: admitted, 2: evicted
+  int n_layers = 1;
   const void* Kc = nullptr;
   const void* Vc = nullptr;
   int N = 0;
@@ -198,7 +199,7 @@ const char* dkv_status_str(dkv_status_t s) {
   return "unknown status";
 }
 
-int32_t dkv_version(void) { return 110; }
+int32_t dkv_version(void) { return 120; }
 
 dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   if (!out || d <= 0) return DKV_ERR_ARG;
@@ -212,7 +213,7 @@ dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   out->order = DKV_ORDER_SCORE;
   out->eviction = DKV_EVICT_MANDATORY_DENSEST;
   out->refresh_baselines = 0;
-  out->reserved = 0;
+  out->layer_heads = 0;
   return DKV_OK;
 }
 
@@ -236,7 +237,8 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   const dkv_params_t& p = *params;
   if (!(p.tau > 1.0f) || !(p.eps > 0.0f) || !(p.delta > 0.0f) || !(p.sigma >= 0.0f) ||
       !(p.p == 1.0f || p.p == 2.0f || p.p == 4.0f) || (p.sync_heads != 0 && p.sync_heads != 1) ||
-      (p.score_mode != DKV_SCORE_TENSOR && p.score_mode != DKV_SCORE_FP32) || p.reserved != 0 ||
+      (p.score_mode != DKV_SCORE_TENSOR && p.score_mode != DKV_SCORE_FP32) ||
+      p.layer_heads < 0 || p.layer_heads > H || (p.layer_heads > 0 && H % p.layer_heads != 0) ||
       (p.order != DKV_ORDER_SCORE && p.order != DKV_ORDER_SOURCE) ||
       (p.eviction != DKV_EVICT_MANDATORY_DENSEST && p.eviction != DKV_EVICT_DENSEST &&
        p.eviction != DKV_EVICT_MANDATORY_SOURCE) ||
@@ -282,6 +284,8 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   b.prov_step = buf->prov_step; b.prov_src = buf->prov_src; b.occ = buf->occupancy;
   b.H = H; b.d = d; b.M_max = M_max; b.n_max = n_max; b.bf16 = bf16;
   ws_layout(H, d, M_max, n_max, bf16, &bk->w, (char*)buf->workspace);
+  bk->w.layer_heads = p.layer_heads > 0 ? p.layer_heads : H;
+  bk->n_layers = H / bk->w.layer_heads;
   const float sg = bk->params.sigma;
   bk->kp.inv_s2 = 1.0f / (sg * sg);
   bk->kp.eps = p.eps;
@@ -293,7 +297,7 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   bk->kp.eviction = p.eviction;
   bk->kp.refresh = p.refresh_baselines;
   // workspace header: zeroed layer state and the per-head budgets (one-time, synchronous)
-  cudaError_t e = cudaMemset(bk->w.L, 0, sizeof(DevLayer));
+  cudaError_t e = cudaMemset(bk->w.L, 0, sizeof(DevLayer) * bk->n_layers);
   if (e == cudaSuccess) e = cudaMemset(bk->w.hd, 0, sizeof(DevHead) * H);
   if (e == cudaSuccess) e = cudaMemset(bk->w.cnt, 0, sizeof(int32_t) * H * bk->w.cnt_stride);
   if (e == cudaSuccess) e = cudaMemcpy(bk->w.budgets, budgets, sizeof(int32_t) * H, cudaMemcpyHostToDevice);
@@ -425,12 +429,15 @@ dkv_status_t dkv_bank_sync(dkv_bank_t bank) {
 dkv_status_t dkv_bank_stats(dkv_bank_t bank, dkv_layer_stats_t* layer, dkv_head_stats_t* heads) {
   if (!bank || !layer) return DKV_ERR_ARG;
   if (cudaStreamSynchronize(bank->last) != cudaSuccess) return DKV_ERR_CUDA;
-  DevLayer L;
-  if (cudaMemcpy(&L, bank->w.L, sizeof(L), cudaMemcpyDeviceToHost) != cudaSuccess) return DKV_ERR_CUDA;
-  layer->r_star = L.r_star;
-  layer->rmax = L.rmax;
-  layer->n_candidates = L.N;
-  layer->empty_init = L.empty_all;
+  std::vector<DevLayer> L(bank->n_layers);
+  if (cudaMemcpy(L.data(), bank->w.L, sizeof(DevLayer) * bank->n_layers, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return DKV_ERR_CUDA;
+  for (int l = 0; l < bank->n_layers; ++l) {
+    layer[l].r_star = L[l].r_star;
+    layer[l].rmax = L[l].rmax;
+    layer[l].n_candidates = L[l].N;
+    layer[l].empty_init = L[l].empty_all;
+  }
   if (heads) {
     std::vector<DevHead> hd(bank->b.H);
     if (cudaMemcpy(hd.data(), bank->w.hd, sizeof(DevHead) * bank->b.H, cudaMemcpyDeviceToHost) != cudaSuccess)

@@ -25,7 +25,7 @@ struct Bank {
 
 // Device workspace, carved from the caller's workspace buffer (dkv_api.cu).
 struct Ws {
-  DevLayer* L;
+  DevLayer* L;          // [H / layer_heads] per-layer state; L[0] also holds the error word
   DevHead* hd;          // [H]
   int32_t* budgets;     // [H]
   float* cnorm;         // [H][n_max]     ||k_x||^2 of the candidates (source order)
@@ -57,7 +57,11 @@ struct Ws {
   float* part;          // [2][H][part_stride] per-row partial sums of column-split passes
   int32_t* cnt;         // [H][cnt_stride] arrival counters of column-split row tiles (kept 0)
   int hist_stride, snap_stride, feas_words, part_stride, cnt_stride, invb_stride, sort_stride;
+  int layer_heads;      // heads per layer (the handle's heads form H / layer_heads layers)
 };
+
+// Per-layer state of head h.
+__host__ __device__ inline DevLayer* layer_of(const Ws& w, int h) { return w.L + h / w.layer_heads; }
 
 // Computes the sub-buffer offsets of the workspace; returns the total bytes.
 size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* base);

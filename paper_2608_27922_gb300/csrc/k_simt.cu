@@ -43,8 +43,8 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
 
   const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
-  const int N = j.w.L->N;
-  const int rmax = j.w.L->rmax;
+  const int N = layer_of(j.w, h)->N;
+  const int rmax = layer_of(j.w, h)->rmax;
   int nrows = 0, c0 = 0, c1 = 0;
   if (MODE == PM_SCORE) { nrows = hd.empty ? 0 : N;                 c1 = hd.m_old; }
   if (MODE == PM_CROSS) { nrows = hd.empty ? 0 : hd.m_old;          c1 = rmax; }

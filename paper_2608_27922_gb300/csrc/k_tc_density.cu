@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(THREADS, 2)
 
   const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
-  const DevLayer L = *j.w.L;
+  const DevLayer L = *layer_of(j.w, h);
   int nrows, c0, c1;
   job_range(MODE, hd, L, nrows, c0, c1);
   const int row0 = blockIdx.x * BM;

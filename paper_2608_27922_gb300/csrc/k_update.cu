@@ -60,11 +60,20 @@ __device__ __forceinline__ void copy64(const uint4* src, uint4* dst) {
   for (int k = 0; k < 4; ++k) dst[k] = v[k];
 }
 
-// Snapshot of occupancy and budgets per head and the prefix range of this update
-// (one block).
+// Snapshot of occupancy and budgets per head and the prefix range of this update,
+// per layer (one block): rmax = min(N, min over the layer's live heads of M_h).
 __device__ __forceinline__ void prepare_body(const Bank& b, const Ws& w, int N, int64_t step) {
-  __shared__ int s_min_budget, s_live;
-  if (threadIdx.x == 0) { s_min_budget = INT_MAX; s_live = 0; }
+  const int G = b.H / w.layer_heads;
+  // per layer, until the last phase: rmax holds the minimum budget of its live heads and
+  // empty_all their count
+  for (int g = threadIdx.x; g < G; g += blockDim.x) {
+    DevLayer* L = w.L + g;
+    L->N = N;
+    L->step = step;
+    L->r_star = 0;
+    L->rmax = INT_MAX;
+    L->empty_all = 0;
+  }
   __syncthreads();
   for (int h = threadIdx.x; h < b.H; h += blockDim.x) {
     int m = b.occ[h];
@@ -77,15 +86,18 @@ __device__ __forceinline__ void prepare_body(const Bank& b, const Ws& w, int N, 
     hd.m_old = m; hd.M = M; hd.r = 0; hd.e = 0; hd.n_mand = 0; hd.n_pre = 0; hd.m_new = m;
     hd.empty = (m == 0);
     w.hd[h] = hd;
-    if (m > 0) { atomicMin(&s_min_budget, M); atomicAdd(&s_live, 1); }
+    if (m > 0) {
+      DevLayer* L = layer_of(w, h);
+      atomicMin(&L->rmax, M);
+      atomicAdd(&L->empty_all, 1);
+    }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    w.L->N = N;
-    w.L->step = step;
-    w.L->empty_all = (s_live == 0);
-    w.L->rmax = s_live ? min(N, s_min_budget) : 0;
-    w.L->r_star = 0;
+  for (int g = threadIdx.x; g < G; g += blockDim.x) {
+    DevLayer* L = w.L + g;
+    const int live = __ldcg(&L->empty_all), min_budget = __ldcg(&L->rmax);
+    L->empty_all = live == 0;
+    L->rmax = live ? min(N, min_budget) : 0;
   }
 }
 
@@ -245,7 +257,7 @@ __device__ __forceinline__ void cas_shfl(unsigned long long (&x)[SKPT], int t, i
 // every run comes out ascending.
 __global__ void __launch_bounds__(256) k_sort_runs(Ws w, int n_max, int identity) {
   const int h = blockIdx.y;
-  const int N = w.L->N;
+  const int N = layer_of(w, h)->N;
   // empty bank: source order (Alg. 1, m = 0 branch); source-order policy: the same
   if (w.hd[h].empty || identity) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x)
@@ -292,7 +304,7 @@ __global__ void __launch_bounds__(RUN) k_sort_rank(Bank bk, Ws w, const char* __
   extern __shared__ unsigned long long runs[];
   __shared__ int s_pos[RUN], s_src[RUN];
   const int h = blockIdx.y;
-  const int N = w.L->N;
+  const int N = layer_of(w, h)->N;
   const int64_t hn = (int64_t)h * bk.n_max;
   const int nruns = (N + RUN - 1) / RUN;
   const int a = blockIdx.x;
@@ -361,15 +373,18 @@ __device__ __forceinline__ DevHead ld_head_cg(const DevHead* p) {
 }
 
 // One block per head: violator counts c_r (prefix sums of the crossing histogram),
-// budgets e_r (Eq. 10) and the feasibility bit of every prefix r; the last block to
-// finish combines the heads (Eq. 11) and sets r, e of every head.
+// budgets e_r (Eq. 10) and the feasibility bit of every prefix r; the last block of a
+// layer to finish combines that layer's heads (Eq. 11) and sets r, e of each of them.
 __global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   __shared__ int s_tot[BIG];
   __shared__ int s_best, s_last;
   const int h = blockIdx.x;
   const DevHead hd = w.hd[h];
-  const int rmax = w.L->rmax;
-  const int N = w.L->N;
+  DevLayer* lay = layer_of(w, h);
+  const int rmax = lay->rmax;
+  const int N = lay->N;
+  const int lh = w.layer_heads;
+  const int h0 = h / lh * lh;   // first head of this layer
   uint32_t* feas = w.feas + (int64_t)h * w.feas_words;
   const int nw = (rmax + 1 + 31) / 32;
   if (threadIdx.x == 0) s_best = 0;
@@ -409,7 +424,7 @@ __global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   if (threadIdx.x == 0) {
     if (!hd.empty) w.hd[h].r = s_best;   // largest feasible prefix of this head alone
     __threadfence();
-    s_last = atomicAdd(&w.L->arrive, 1) == (int)gridDim.x - 1;
+    s_last = atomicAdd(&lay->arrive, 1) == lh - 1;   // the layer's last head to arrive
   }
   __syncthreads();
   if (!s_last) return;
@@ -420,7 +435,7 @@ __global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   if (sync_heads) {
     for (int i = threadIdx.x; i < nw; i += blockDim.x) {
       uint32_t a = 0xffffffffu;
-      for (int hh = 0; hh < b.H; ++hh) a &= __ldcg(w.feas + (int64_t)hh * w.feas_words + i);
+      for (int hh = h0; hh < h0 + lh; ++hh) a &= __ldcg(w.feas + (int64_t)hh * w.feas_words + i);
       if (i == nw - 1 && ((rmax + 1) & 31)) a &= (1u << ((rmax + 1) & 31)) - 1u;
       if (i == 0) a |= 1u;
       if (a) atomicMax(&s_best, i * 32 + 31 - __clz(a));
@@ -431,7 +446,7 @@ __global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   __shared__ int s_rmax_used, s_rmin_used;
   if (threadIdx.x == 0) { s_rmax_used = 0; s_rmin_used = INT_MAX; }
   __syncthreads();
-  for (int hh = threadIdx.x; hh < b.H; hh += blockDim.x) {
+  for (int hh = h0 + threadIdx.x; hh < h0 + lh; hh += blockDim.x) {
     DevHead d = ld_head_cg(w.hd + hh);
     int r;
     if (d.empty) r = min(N, d.M);
@@ -446,8 +461,8 @@ __global__ void __launch_bounds__(BIG) k_rstar(Bank b, Ws w, int sync_heads) {
   // reported r*: Alg. 1's min(N, M) when every head starts empty (min over per-head budgets),
   // the shared prefix when synchronised, else the largest per-head prefix
   if (threadIdx.x == 0) {
-    w.L->r_star = w.L->empty_all ? s_rmin_used : (sync_heads ? rstar : s_rmax_used);
-    w.L->arrive = 0;
+    lay->r_star = lay->empty_all ? s_rmin_used : (sync_heads ? rstar : s_rmax_used);
+    lay->arrive = 0;
   }
 }
 
@@ -779,7 +794,7 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
         copy64(dx, reinterpret_cast<uint4*>((char*)w.kevict_ext + (hn + j) * 64));
       }
       b.knorm[bh + slot] = w.kperm_norm[hn + j];
-      b.prov_step[bh + slot] = w.L->step;
+      b.prov_step[bh + slot] = layer_of(w, h)->step;
       b.prov_src[bh + slot] = src;
       w.slot_new[hn + j] = slot;
       copy64(reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64), dx);

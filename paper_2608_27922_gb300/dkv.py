@@ -32,7 +32,7 @@ class dkv_params_t(ctypes.Structure):
     _fields_ = [("tau", ctypes.c_float), ("sigma", ctypes.c_float), ("p", ctypes.c_float),
                 ("eps", ctypes.c_float), ("delta", ctypes.c_float), ("sync_heads", ctypes.c_int32),
                 ("score_mode", ctypes.c_int32), ("order", ctypes.c_int32), ("eviction", ctypes.c_int32),
-                ("refresh_baselines", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("refresh_baselines", ctypes.c_int32), ("layer_heads", ctypes.c_int32)]
 
 
 class dkv_buffers_t(ctypes.Structure):
@@ -201,11 +201,11 @@ def dkv_bank_sync(bank: int) -> None:
     _check(lib().dkv_bank_sync(bank), "dkv_bank_sync")
 
 
-def dkv_bank_stats(bank: int, H: int) -> Tuple[dkv_layer_stats_t, List[dkv_head_stats_t]]:
-    L = dkv_layer_stats_t()
+def dkv_bank_stats(bank: int, H: int, n_layers: int = 1) -> Tuple[List[dkv_layer_stats_t], List[dkv_head_stats_t]]:
+    Ls = (dkv_layer_stats_t * n_layers)()
     arr = (dkv_head_stats_t * H)()
-    _check(lib().dkv_bank_stats(bank, ctypes.byref(L), arr), "dkv_bank_stats")
-    return L, list(arr)
+    _check(lib().dkv_bank_stats(bank, Ls, arr), "dkv_bank_stats")
+    return list(Ls), list(arr)
 
 
 def dkv_bank_occupancy(bank: int, H: int) -> List[int]:
@@ -276,8 +276,9 @@ def _view(ptr: int, shape, dtype: torch.dtype, device) -> torch.Tensor:
 
 
 class BankLayer:
-    """One layer's H per-head banks: allocates the caller-owned buffers with torch and
-    drives the C ABI.  All methods enqueue on the current (or given) stream."""
+    """H per-head banks (one layer, or H / layer_heads layers when the layer_heads
+    parameter is set): allocates the caller-owned buffers with torch and drives the C
+    ABI.  All methods enqueue on the current (or given) stream."""
 
     def __init__(self, H: int, d: int, budgets: Sequence[int], n_max: int, dtype: torch.dtype = torch.bfloat16,
                  params: Optional[dkv_params_t] = None, device="cuda", **param_overrides):
@@ -295,6 +296,7 @@ class BankLayer:
         for k, v in param_overrides.items():
             setattr(p, k, v)
         self.params = p
+        self.n_layers = H // p.layer_heads if p.layer_heads > 0 else 1
         dev = self.device
         self.k = torch.zeros(H, self.M_max, d, dtype=dtype, device=dev)
         self.v = torch.zeros(H, self.M_max, d, dtype=dtype, device=dev)
@@ -375,7 +377,13 @@ class BankLayer:
         dkv_bank_sync(self.handle)
 
     def stats(self):
-        return dkv_bank_stats(self.handle, self.H)
+        """(statistics of the first layer, per-head statistics of every head)."""
+        Ls, hs = dkv_bank_stats(self.handle, self.H, self.n_layers)
+        return Ls[0], hs
+
+    def layer_stats(self) -> List[dkv_layer_stats_t]:
+        """Statistics of each of the handle's layers (params.layer_heads heads each)."""
+        return dkv_bank_stats(self.handle, self.H, self.n_layers)[0]
 
     def occupancy_host(self) -> List[int]:
         return dkv_bank_occupancy(self.handle, self.H)

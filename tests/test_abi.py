@@ -65,7 +65,7 @@ int main(void) {
   printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t),
          sizeof(dkv_layer_stats_t), sizeof(dkv_head_stats_t), sizeof(dkv_intermediates_t),
          offsetof(dkv_buffers_t, workspace_bytes), offsetof(dkv_params_t, order), offsetof(dkv_params_t, eviction),
-         offsetof(dkv_params_t, refresh_baselines), offsetof(dkv_params_t, reserved));
+         offsetof(dkv_params_t, refresh_baselines), offsetof(dkv_params_t, layer_heads));
   return 0;
 }
 """
@@ -84,7 +84,7 @@ int main(void) {
                      ctypes.sizeof(dkv.dkv_layer_stats_t), ctypes.sizeof(dkv.dkv_head_stats_t),
                      ctypes.sizeof(dkv.dkv_intermediates_t), dkv.dkv_buffers_t.workspace_bytes.offset,
                      dkv.dkv_params_t.order.offset, dkv.dkv_params_t.eviction.offset,
-                     dkv.dkv_params_t.refresh_baselines.offset, dkv.dkv_params_t.reserved.offset]
+                     dkv.dkv_params_t.refresh_baselines.offset, dkv.dkv_params_t.layer_heads.offset]
 
 
 def test_host_only_entry_points():

@@ -1,0 +1,94 @@
+"""Several layers in one handle (params.layer_heads): every call updates or reads all
+layers with single launches, each layer keeping its own shared prefix r* (Eq. 11).
+
+The grouped handle is compared bit for bit with one handle per layer fed the same
+per-layer streams (those are themselves parity-tested against the oracle): bank
+contents, occupancy, provenance, densities, baselines, attention outputs and each
+layer's r* must be identical.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from gpu_util import to_dev
+
+pytestmark = pytest.mark.gpu
+
+BUFFERS = ("k", "v", "rho", "base", "knorm", "prov_step", "prov_src", "occupancy")
+
+
+@pytest.fixture(scope="module")
+def dkv():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_27922_gb300 import dkv as d
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    return d
+
+
+def _cat_heads(parts, dtype):
+    return torch.cat([to_dev(p, dtype) for p in parts], dim=0).contiguous()
+
+
+@pytest.mark.parametrize("mode", ["tc", "fp32"])
+@pytest.mark.parametrize("sync", [1, 0])
+def test_grouped_layers_match_one_handle_per_layer(dkv, mode, sync):
+    L, H = 3, 2
+    # per-layer budgets differ, so the layers fill, saturate and freeze at different steps
+    budgets = [300, 300, 190, 250, 420, 420]
+    wl = synth.get_workload("wan13b_layer_h12", L=L, H=H, N=96, W=96, Nq=64, budgets=budgets, steps=9)
+    sm = dkv.DKV_SCORE_TENSOR if mode == "tc" else dkv.DKV_SCORE_FP32
+    dt = torch.bfloat16
+    sep = [dkv.BankLayer(H, wl.d, wl.budgets_of_layer(l), wl.N, dt, score_mode=sm, sync_heads=sync)
+           for l in range(L)]
+    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, dt, score_mode=sm, sync_heads=sync, layer_heads=H)
+    assert grp.n_layers == L
+    for b in sep + [grp]:
+        b.reset()
+    ro = [synth.LayerRollout(wl, l) for l in range(L)]
+    rstars = []
+    for t in range(wl.steps):
+        qs = [ro[l].queries(t) for l in range(L)]
+        wins = [ro[l].window(t) for l in range(L)]
+        o_sep = [sep[l].attend(to_dev(qs[l], dt), to_dev(wins[l][0], dt), to_dev(wins[l][1], dt)) for l in range(L)]
+        o_grp = grp.attend(_cat_heads(qs, dt), _cat_heads([w[0] for w in wins], dt),
+                           _cat_heads([w[1] for w in wins], dt))
+        b = wl.admitted_block(t)
+        if b is not None:
+            blocks = [ro[l].block(b) for l in range(L)]
+            for l in range(L):
+                sep[l].admit(to_dev(blocks[l][0], dt), to_dev(blocks[l][1], dt), b)
+                sep[l].compress()
+            grp.admit(_cat_heads([x[0] for x in blocks], dt), _cat_heads([x[1] for x in blocks], dt), b)
+            grp.compress()
+        torch.cuda.synchronize()
+        for bk in sep + [grp]:
+            bk.sync()
+        assert torch.equal(torch.cat(o_sep, 0), o_grp), t
+        for name in BUFFERS:
+            g = getattr(grp, name)
+            for l in range(L):
+                want = getattr(sep[l], name)   # [H] or [H][M_l(, d)]; the grouped rows are longer
+                got = g[l * H:(l + 1) * H]
+                if want.dim() > 1:
+                    got = got[:, :want.shape[1]]
+                assert torch.equal(want, got), (t, name, l)
+        if b is not None:
+            ls = grp.layer_stats()
+            assert [x.r_star for x in ls] == [sep[l].stats()[0].r_star for l in range(L)], t
+            assert [x.rmax for x in ls] == [sep[l].stats()[0].rmax for l in range(L)], t
+            rstars.append(tuple(x.r_star for x in ls))
+    # the layers really did take different prefixes at some step
+    assert any(len(set(r)) > 1 for r in rstars), rstars
+    for bk in sep + [grp]:
+        bk.close()
+
+
+def test_layer_heads_must_divide_heads(dkv):
+    wl = synth.get_workload("wan13b_layer_h12", H=6, N=16, budgets=32)
+    for bad in (4, 7, -1):
+        with pytest.raises(dkv.DkvError) as e:
+            dkv.BankLayer(6, wl.d, wl.budgets_of_layer(0), 16, torch.bfloat16, layer_heads=bad)
+        assert e.value.status == 1
