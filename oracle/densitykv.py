@@ -27,6 +27,8 @@ What each function follows (paper sections / equations):
                          prefix length, shared cross-head prefix r*,
                          mandatory-then-densest eviction, commit, exact density
                          maintenance and frozen insertion baselines.
+* ``update_layer_sequential``  App. E "Within-block competition": the block's
+                         candidates offered one at a time (reading below).
 * ``attend``             softmax attention of queries over [bank | window]
                          with scale 1/sqrt(d_k) (Sec. 3.2 logit definition,
                          App. A Eq. "supp-logit"; Fig. 2 caption).
@@ -58,6 +60,12 @@ the design notes of the repository):
   after each update instead of keeping the insertion-time baseline.  In every
   variant r* is still the largest prefix feasible under Eqs. 9-11 for the
   candidates in the variant's order.
+* Within-block competition (App. E) is read as: the block's order fixed once
+  against the bank at block start, then one one-candidate update per position
+  of that order (the j-th candidate of every head together, so the shared prefix
+  of Eq. 11 is taken over the heads for each offer), provenance keeping the
+  candidate's source index; an all-empty bank is initialised by the whole block
+  as in the default.
 """
 from __future__ import annotations
 
@@ -70,7 +78,7 @@ import numpy as np
 __all__ = [
     "Params", "HeadBank", "LayerBank", "HeadRecord", "UpdateRecord",
     "soft_riesz", "sq_dist", "density", "potential_against",
-    "update_layer", "attend", "storage_bytes", "GIB",
+    "update_layer", "update_layer_sequential", "block_order", "attend", "storage_bytes", "GIB",
 ]
 
 GIB = float(1 << 30)
@@ -236,7 +244,8 @@ def _prefix_rho_tilde_literal(hb: HeadBank, Kc_pi: np.ndarray, prm: Params, rmax
     return out
 
 
-def _empty_init(hb: HeadBank, Kc: np.ndarray, Vc: np.ndarray, step: int, prm: Params) -> HeadRecord:
+def _empty_init(hb: HeadBank, Kc: np.ndarray, Vc: np.ndarray, step: int, prm: Params,
+                src: Optional[np.ndarray] = None) -> HeadRecord:
     """Alg. 1, m = 0 branch: admit the first min(N, M) source-ordered candidates, then set
     rho_i = Phi over the resulting bank and b_i = max(rho_i, delta)."""
     N = Kc.shape[0]
@@ -247,16 +256,18 @@ def _empty_init(hb: HeadBank, Kc: np.ndarray, Vc: np.ndarray, step: int, prm: Pa
     hb.rho = rho.astype(hb.store)
     hb.base = np.maximum(rho, prm.delta).astype(hb.store)
     hb.step = np.full(r, step, np.int64)
-    hb.src = np.arange(r, dtype=np.int64)
+    hb.src = (np.arange(r) if src is None else np.asarray(src[:r])).astype(np.int64)
     return HeadRecord(empty_init=True, r_used=r, admitted=np.arange(r), evicted=np.zeros(0, np.int64))
 
 
 def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
-                 prm: Params = Params(), literal: bool = False) -> UpdateRecord:
+                 prm: Params = Params(), literal: bool = False,
+                 src_index: Optional[np.ndarray] = None) -> UpdateRecord:
     """One DensityKV update of one layer (Algorithm 1, App. C), in place on ``bank``.
 
     Kc, Vc: candidate keys/values of the finalized block, [H][N][d] and [H][N][dv],
-    in source order.  ``step`` is recorded as the provenance of admitted states.
+    in source order.  ``step`` is recorded as the provenance of admitted states, with
+    the candidate's row as its source index, or src_index[h][row] when given.
     ``literal=True`` recomputes every prefix sum from scratch (tiny inputs).
     """
     assert prm.order in ("score", "source")
@@ -271,7 +282,8 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
     live = [h for h in range(H) if bank.heads[h].m > 0]
     for h in range(H):
         if bank.heads[h].m == 0:
-            recs[h] = _empty_init(bank.heads[h], Kc[h], Vc[h], step, prm)
+            recs[h] = _empty_init(bank.heads[h], Kc[h], Vc[h], step, prm,
+                                  None if src_index is None else src_index[h])
 
     rmax = min([N] + [bank.heads[h].M for h in live]) if live else 0
     if not live:
@@ -369,11 +381,59 @@ def update_layer(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
         else:
             hb.base = np.concatenate([hb.base[keep], np.maximum(rho_new, prm.delta)]).astype(hb.store)
         hb.step = np.concatenate([hb.step[keep], np.full(r, step, np.int64)])
-        hb.src = np.concatenate([hb.src[keep], adm.astype(np.int64)])
+        adm_src = adm if src_index is None else np.asarray(src_index[h])[adm]
+        hb.src = np.concatenate([hb.src[keep], adm_src.astype(np.int64)])
         recs[h] = HeadRecord(empty_init=False, s=s, pi=pi, counts=counts, e=e, cross=cross,
                              r_used=r, rho_tilde=rho_t, g_star=g_r, mandatory=mand,
                              evicted=R, admitted=adm)
     return UpdateRecord(r_star=r_star, rmax=rmax, heads=recs)
+
+
+def block_order(bank: LayerBank, Kc: np.ndarray, prm: Params = Params()) -> np.ndarray:
+    """pi_h of every head against the bank as it is now ([H][N]): ascending Eq. 6 score
+    (ties in source order), or source order under the source-order policy; the order
+    update_layer takes for a non-empty head (an empty head: source order)."""
+    Kc = np.asarray(Kc, dtype=np.float64)
+    H, N = Kc.shape[0], Kc.shape[1]
+    out = np.tile(np.arange(N), (H, 1))
+    for h, hb in enumerate(bank.heads):
+        if hb.m == 0 or prm.order == "source":
+            continue
+        Wxb = soft_riesz(sq_dist(Kc[h], hb.K), prm, hb.d)
+        s = (Wxb / hb.base.astype(np.float64)[None, :]).sum(axis=1) / hb.m
+        out[h] = np.argsort(s, kind="stable")
+    return out
+
+
+def update_layer_sequential(bank: LayerBank, Kc: np.ndarray, Vc: np.ndarray, step: int,
+                            prm: Params = Params()) -> List[UpdateRecord]:
+    """Within-block competition (App. E "Within-block competition"; Sec. 4 ablations):
+    sequential density-gated admission, so that earlier candidates of the block act on
+    later ones.  Reading: the block's order is fixed once, as the default order against
+    the bank at block start (block_order); the candidates are then offered one per head
+    at a time (the j-th of every head's order, for j = 0 .. N-1), each offer a complete
+    one-candidate update (Eqs. 6-12 with N = 1: the growth gate, eviction, commit and the
+    frozen baseline of the admitted state), the candidate keeping its source index in the
+    block as provenance.  A bank whose heads are all empty is initialised by the whole
+    block (Alg. 1, m = 0 branch) exactly as in the default; a partly empty bank is not
+    accepted (an empty head would otherwise start from a single state whose baseline is
+    delta, and then reject every later candidate)."""
+    empty = [hb.m == 0 for hb in bank.heads]
+    if all(empty):
+        return [update_layer(bank, Kc, Vc, step, prm)]
+    if any(empty):
+        raise ValueError("sequential admission needs every head empty or every head non-empty")
+    Kc = np.asarray(Kc, dtype=np.float64)
+    Vc = np.asarray(Vc, dtype=np.float64)
+    H, N = Kc.shape[0], Kc.shape[1]
+    pi = block_order(bank, Kc, prm)
+    rows = np.arange(H)
+    recs = []
+    for j in range(N):
+        c = pi[:, j]
+        recs.append(update_layer(bank, Kc[rows, c][:, None], Vc[rows, c][:, None], step, prm,
+                                 src_index=c[:, None]))
+    return recs
 
 
 def attend(hb: HeadBank, Q: np.ndarray, Kw: np.ndarray, Vw: np.ndarray) -> np.ndarray:

@@ -512,6 +512,87 @@ def check_policy_variants(O):
     assert outs["densest"] in ([1], [2])           # the densest of the pair instead
 
 
+
+def check_sequential_admission(O):
+    """Within-block competition (App. E), read as one-candidate updates in the order fixed
+    at block start.  Pinned independently of the oracle's code: (1) after every block the
+    cached densities equal the exact Soft-Riesz density over the bank (Eq. 3, self
+    excluded) and states of earlier blocks keep their frozen baselines and provenance;
+    (2) two identical candidates offered to a bank that is not full and lies far from them
+    are both admitted by the default update (their mutual interaction only enters their
+    new baselines), but sequentially the second is gated out: once the first is in, the
+    duplicate would raise its density by w(0) = eps^-p, far beyond tau times its baseline,
+    and a bank with free room has no eviction budget for it (e_1 = 0); (3) the offers follow
+    the ascending Eq. 6 order of block start: with every bank state on the +e0 side,
+    x' = +0.25 e0 (source index 0) scores above x = -0.25 e0 (index 1), so x is offered and
+    admitted first and x' is gated out; (4) an all-empty bank is initialised by the whole
+    block as in the default, and a partly empty bank is refused."""
+    rng = np.random.default_rng(3)
+    for sync in (True, False):
+        prm = _prm(O, sync_heads=sync)
+        ob = O.LayerBank.empty([24, 30], 8)
+        O.update_layer_sequential(ob, rng.standard_normal((2, 16, 8)) * 2, rng.standard_normal((2, 16, 8)), 0, prm)
+        for t in range(1, 4):
+            before = [dict(zip(zip(hb.step.tolist(), hb.src.tolist()), hb.base.tolist())) for hb in ob.heads]
+            O.update_layer_sequential(ob, rng.standard_normal((2, 12, 8)) * 2, rng.standard_normal((2, 12, 8)), t, prm)
+            for h, hb in enumerate(ob.heads):
+                assert hb.m <= hb.M
+                K = hb.K.astype(np.float64)
+                d2 = ((K[:, None, :] - K[None, :, :]) ** 2).sum(-1)
+                W = (prm.eps + d2 / prm.sigma_for(8) ** 2) ** (-prm.p)
+                np.fill_diagonal(W, 0.0)
+                np.testing.assert_allclose(hb.rho.astype(np.float64), W.sum(axis=1), rtol=2e-6, atol=1e-30)
+                keys = list(zip(hb.step.tolist(), hb.src.tolist()))
+                assert len(set(keys)) == len(keys)
+                for k, b in zip(keys, hb.base.tolist()):
+                    if k[0] < t:
+                        assert before[h][k] == b
+                    else:
+                        assert k[0] == t and 0 <= k[1] < 12
+
+    prm = _prm(O)
+    e0 = np.eye(8)[0]
+
+    def far_bank():
+        r = np.random.default_rng(5)
+        K0 = r.standard_normal((1, 20, 8))
+        K0 = K0 / np.linalg.norm(K0, axis=2, keepdims=True) * 6.0
+        ob = O.LayerBank.empty([40], 8)
+        O.update_layer(ob, K0, K0, 0, prm)
+        return ob
+
+    block = np.stack([0.25 * e0, 0.25 * e0])[None]
+    default = far_bank()
+    assert O.update_layer(default, block, block, 1, prm).r_star == 2 and default.heads[0].m == 22
+    seq = far_bank()
+    assert [r.r_star for r in O.update_layer_sequential(seq, block, block, 1, prm)] == [1, 0]
+    hb = seq.heads[0]
+    assert hb.m == 21 and [s for st, s in zip(hb.step.tolist(), hb.src.tolist()) if st == 1] == [0]
+
+    u = np.random.default_rng(11).standard_normal((20, 8))
+    K0 = 6.0 * e0 + 3.0 * u / np.linalg.norm(u, axis=1, keepdims=True)   # first coordinate >= 3
+    ob = O.LayerBank.empty([40], 8)
+    O.update_layer(ob, K0[None], K0[None], 0, prm)
+    block = np.stack([0.25 * e0, -0.25 * e0])[None]
+    assert [r.r_star for r in O.update_layer_sequential(ob, block, block, 1, prm)] == [1, 0]
+    hb = ob.heads[0]
+    assert [s for st, s in zip(hb.step.tolist(), hb.src.tolist()) if st == 1] == [1]
+
+    K = np.random.default_rng(9).standard_normal((2, 10, 8))
+    a, b = O.LayerBank.empty([6, 8], 8), O.LayerBank.empty([6, 8], 8)
+    O.update_layer_sequential(a, K, K, 0, prm)
+    O.update_layer(b, K, K, 0, prm)
+    for ha, hb in zip(a.heads, b.heads):
+        assert np.array_equal(ha.K, hb.K) and np.array_equal(ha.base, hb.base)
+    b.heads[1] = O.HeadBank(M=8, d=8, dv=8)
+    try:
+        O.update_layer_sequential(b, K, K, 1, prm)
+    except ValueError:
+        pass
+    else:
+        raise AssertionError("a partly empty bank was accepted")
+
+
 ALL_CHECKS = [
     check_kernel_closed_forms,
     check_distance_identities,
@@ -525,4 +606,5 @@ ALL_CHECKS = [
     check_storage_accounting,
     check_attention_textbook,
     check_policy_variants,
+    check_sequential_admission,
 ]

@@ -70,6 +70,10 @@ MUTANTS = [
     ("refresh_ignored", "if prm.refresh_baselines:\n", "if False:\n"),
     ("source_order_ignored", 'if prm.order == "score" else np.arange(N)', 'if True else np.arange(N)'),
     ("densest_keeps_mandatory_first", 'if prm.evict == "densest":', 'if prm.evict == "never":'),
+    ("sequential_source_order", "        c = pi[:, j]\n", "        c = np.arange(H) * 0 + j\n"),
+    ("sequential_src_dropped", "adm_src = adm if src_index is None else np.asarray(src_index[h])[adm]",
+     "adm_src = adm"),
+    ("block_order_descending", '        out[h] = np.argsort(s, kind="stable")', '        out[h] = np.argsort(-s, kind="stable")'),
 ]
 
 
