@@ -61,6 +61,9 @@ def parse_args():
     ap.add_argument("--eviction", choices=["mandatory_densest", "densest", "mandatory_source"],
                     default="mandatory_densest", help="eviction rule (policy ablation)")
     ap.add_argument("--refresh-baselines", action="store_true", help="refresh b after every update (ablation)")
+    ap.add_argument("--within-block", choices=["batch", "sequential"], default="batch",
+                    help="sequential: within-block competition, one candidate per head at a time (ablation; "
+                         "no graphs, no overlap, no e2e leg)")
     ap.add_argument("--attn-passes", type=int, default=1,
                     help="bank-reading attention passes per update (denoising passes; the update runs once)")
     ap.add_argument("--layers", type=int, default=1,
@@ -80,7 +83,11 @@ def parse_args():
                     help="run attention and the update on one stream instead of overlapping them")
     ap.add_argument("--no-graphs", action="store_true",
                     help="launch every step directly instead of replaying a captured CUDA graph")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.within_block == "sequential":
+        # the sequential path synchronises with its stream once per block: no graph capture
+        args.no_graphs = args.no_overlap = args.no_e2e = True
+    return args
 
 
 def dist_env():
@@ -286,8 +293,11 @@ def run_ours(args):
             for _ in range(P):
                 bank.attend(Q, KW, VW, out=out)
             if b is not None:
-                bank.admit(KC, VC, b)
-                bank.compress()
+                if args.within_block == "sequential":
+                    bank.update_sequential(KC, VC, b)
+                else:
+                    bank.admit(KC, VC, b)
+                    bank.compress()
             return
         # attention, admit and evict only read the bank (the update is atomic from the
         # reader's side), so they run concurrently; only the commit waits for attention
@@ -529,7 +539,8 @@ def run_ours(args):
                        "score_mode": args.score_mode, "layers_per_gpu": 1,
                        "attn_passes_per_update": max(1, args.attn_passes),
                        "policy": {"order": args.order, "eviction": args.eviction,
-                                  "refresh_baselines": bool(args.refresh_baselines)},
+                                  "refresh_baselines": bool(args.refresh_baselines),
+                                  "within_block": args.within_block},
                        "streams": "attention || admit + evict, then commit" if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",

@@ -229,6 +229,25 @@ dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream);
 dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const void* Kw,
                              const void* Vw, int32_t W, void* O, void* stream);
 
+/* Within-block competition (App. E "Within-block competition"): sequential,
+ * density-gated admission, so that earlier candidates of a block act on later
+ * ones.  The block's order is fixed once against the bank at block start (the
+ * order dkv_bank_admit would take); then, for j = 0 .. N-1, the j-th candidate of
+ * every head is offered as a complete one-candidate update (growth gate of
+ * Eqs. 8-11, eviction, commit of Eq. 12, density maintenance of Eq. C.4 and the
+ * frozen baseline of Eq. 5), the state recording its source index in the block
+ * as provenance.  A bank whose heads are all empty is initialised by the whole
+ * block (Alg. 1, m = 0), exactly as dkv_bank_admit + compress would; a bank with
+ * some empty heads returns DKV_ERR_STATE.
+ *   Kc, Vc  : device [H][N][d] as for dkv_bank_admit.
+ *   scratch : device, 256-byte aligned, >= dkv_sequential_scratch_size() bytes.
+ * Synchronises with `stream` once (to read the occupancy) and enqueues about a
+ * dozen launches per candidate: an ablation path, not the hot path.  Must not be
+ * called between admit and commit (DKV_ERR_STATE).                              */
+size_t dkv_sequential_scratch_size(int32_t H, int32_t d, int32_t n_max, int32_t dtype);
+dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N,
+                                        int64_t step, void* scratch, size_t scratch_bytes, void* stream);
+
 /* Declares that the caller has written bank contents directly (k, v, rho,
  * base, prov_*) and sets occupancy from the host array occupancy[0..H)
  * (0 <= occupancy[h] <= budgets[h]).  Recomputes the derived key norms.

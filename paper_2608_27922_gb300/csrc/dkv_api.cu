@@ -158,6 +158,7 @@ struct dkv_bank_s {
   bool tc = false;
   int state = 0;   // 0: idle, 1: admitted, 2: evicted
   int n_layers = 1;
+  const int32_t* src_map = nullptr;   // provenance source index of each candidate (sequential admission)
   const void* Kc = nullptr;
   const void* Vc = nullptr;
   int N = 0;
@@ -372,7 +373,7 @@ dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream) {
   const KParams& kp = bank->kp;
   bank->last = s;
   bank->state = 0;
-  cudaError_t e = launch_commit(b, w, bank->Vc, bank->N, s, t);
+  cudaError_t e = launch_commit(b, w, bank->Vc, bank->N, bank->src_map, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_subtract_tc(b, w, kp, s, t) : launch_subtract_fp32(b, w, kp, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_newbase_tc(b, w, kp, s, t) : launch_newbase_fp32(b, w, kp, s, t);
   return cuda_status(e);
@@ -383,6 +384,92 @@ dkv_status_t dkv_bank_compress(dkv_bank_t bank, void* stream) {
   if (bank->state != 1) return DKV_ERR_STATE;
   const dkv_status_t st = dkv_bank_evict(bank, stream);
   return st != DKV_OK ? st : dkv_bank_commit(bank, stream);
+}
+
+// ---- sequential admission (within-block competition)
+namespace {
+struct SeqScratch {
+  char *kseq, *vseq, *k1, *v1;
+  int32_t *srcseq, *src1;
+};
+size_t seq_layout(int H, int d, int n_max, int bf16, SeqScratch* out, char* base) {
+  const size_t es = bf16 ? 2 : 4, rb = (size_t)d * es;
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> char* {
+    char* p = base ? base + off : nullptr;
+    off += (bytes + 255) & ~(size_t)255;
+    return p;
+  };
+  SeqScratch sc{};
+  sc.kseq = take((size_t)H * n_max * rb);
+  sc.vseq = take((size_t)H * n_max * rb);
+  sc.srcseq = (int32_t*)take((size_t)H * n_max * 4);
+  sc.k1 = take((size_t)H * rb);
+  sc.v1 = take((size_t)H * rb);
+  sc.src1 = (int32_t*)take((size_t)H * 4);
+  if (out) *out = sc;
+  return off;
+}
+}  // namespace
+
+size_t dkv_sequential_scratch_size(int32_t H, int32_t d, int32_t n_max, int32_t dtype) {
+  if (H < 1 || H > kMaxH || (d != 64 && d != 128) || n_max < 1 || n_max > kMaxN) return 0;
+  if (dtype != DKV_DTYPE_BF16 && dtype != DKV_DTYPE_FP32) return 0;
+  return seq_layout(H, d, n_max, dtype == DKV_DTYPE_BF16, nullptr, nullptr);
+}
+
+dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
+                                        void* scratch, size_t scratch_bytes, void* stream) {
+  if (!bank || !Kc || !Vc || !scratch) return DKV_ERR_ARG;
+  if (bank->state != 0) return DKV_ERR_STATE;
+  if (N < 1 || N > bank->b.n_max) return DKV_ERR_SHAPE;
+  if (step < 0 || step > 0x7fffffffLL) return DKV_ERR_ARG;
+  if (!aligned(Kc, 16) || !aligned(Vc, 16) || !aligned(scratch, 256)) return DKV_ERR_ARG;
+  const Bank& b = bank->b;
+  if (scratch_bytes < seq_layout(b.H, b.d, b.n_max, b.bf16, nullptr, nullptr)) return DKV_ERR_NOMEM;
+  cudaStream_t s = (cudaStream_t)stream;
+  bank->last = s;
+  // every head empty: the whole block initialises the bank (Alg. 1, m = 0), as by default
+  std::vector<int32_t> occ(b.H);
+  if (cudaStreamSynchronize(s) != cudaSuccess ||
+      cudaMemcpy(occ.data(), b.occ, sizeof(int32_t) * b.H, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return DKV_ERR_CUDA;
+  int n_empty = 0;
+  for (int h = 0; h < b.H; ++h) n_empty += occ[h] == 0;
+  if (n_empty == b.H) {
+    const dkv_status_t st = dkv_bank_admit(bank, Kc, Vc, N, step, stream);
+    return st != DKV_OK ? st : dkv_bank_compress(bank, stream);
+  }
+  if (n_empty > 0) return DKV_ERR_STATE;
+  // the block's order against the bank at block start, then its rows in that order
+  SeqScratch sc;
+  seq_layout(b.H, b.d, b.n_max, b.bf16, &sc, (char*)scratch);
+  const Ws& w = bank->w;
+  Timer* t = &bank->timer;
+  const KParams& kp = bank->kp;
+  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, kp, s, t);
+  if (e == cudaSuccess && kp.order == DKV_ORDER_SCORE)
+    e = bank->tc ? launch_score_tc(b, w, Kc, N, kp, s, t) : launch_score_fp32(b, w, Kc, N, kp, s, t);
+  if (e == cudaSuccess) e = launch_sort(b, w, Kc, kp.order == DKV_ORDER_SOURCE, s, t);
+  if (e == cudaSuccess) e = launch_seq_gather(b, w, Kc, Vc, N, sc.kseq, sc.vseq, sc.srcseq, s);
+  if (e != cudaSuccess) return DKV_ERR_CUDA;
+  // one one-candidate update per position j: the j-th candidate of every head
+  const size_t rb = (size_t)b.d * (b.bf16 ? 2 : 4);
+  for (int j = 0; j < N; ++j) {
+    e = cudaMemcpy2DAsync(sc.k1, rb, sc.kseq + j * rb, (size_t)N * rb, rb, b.H, cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(sc.v1, rb, sc.vseq + j * rb, (size_t)N * rb, rb, b.H, cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(sc.src1, 4, sc.srcseq + j, (size_t)N * 4, 4, b.H, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return DKV_ERR_CUDA;
+    dkv_status_t st = dkv_bank_admit(bank, sc.k1, sc.v1, 1, step, stream);
+    if (st != DKV_OK) return st;
+    bank->src_map = sc.src1;
+    st = dkv_bank_compress(bank, stream);
+    bank->src_map = nullptr;
+    if (st != DKV_OK) return st;
+  }
+  return DKV_OK;
 }
 
 dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const void* Kw, const void* Vw,

@@ -83,7 +83,11 @@ cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStre
 // update back half (compress)
 cudaError_t launch_project_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_select(const Bank& b, const Ws& w, int eviction, cudaStream_t s, Timer* t);
-cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t);
+cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, const int32_t* src_map, cudaStream_t s,
+                          Timer* t);
+// sequential admission: the block in pi order (keys, values, source indices) into scratch
+cudaError_t launch_seq_gather(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, void* Kseq,
+                              void* Vseq, int32_t* srcseq, cudaStream_t s);
 cudaError_t launch_subtract_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_newbase_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // tensor-core (tcgen05) versions of the pair passes, bf16 and d = 128 only

@@ -735,7 +735,8 @@ __global__ void k_inv_base(Bank b, Ws w) {
 // are copied bit for bit.  An evicted slot is read and overwritten by one thread in
 // program order, appended slots lie above every survivor, so no slot is written while
 // another thread still reads it.
-__global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int esize) {
+__global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int esize,
+                         const int32_t* __restrict__ src_map) {
   const int h = blockIdx.y;
   const DevHead hd = w.hd[h];
   const int64_t bh = (int64_t)h * b.M_max;
@@ -795,10 +796,32 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
       }
       b.knorm[bh + slot] = w.kperm_norm[hn + j];
       b.prov_step[bh + slot] = layer_of(w, h)->step;
-      b.prov_src[bh + slot] = src;
+      b.prov_src[bh + slot] = src_map ? src_map[(int64_t)h * N + src] : src;
       w.slot_new[hn + j] = slot;
       copy64(reinterpret_cast<const uint4*>((const char*)w.kperm_ext + (hn + j) * 64), dx);
     }
+  }
+}
+
+// The block's keys, values and source indices in pi order (sequential admission:
+// position j of every head is offered together).  Rows are copied bit for bit.
+__global__ void k_seq_gather(Bank b, Ws w, const char* __restrict__ Kc, const char* __restrict__ Vc, int N,
+                             int esize, char* __restrict__ Kseq, char* __restrict__ Vseq, int32_t* __restrict__ srcseq) {
+  const int h = blockIdx.y;
+  const int rb = b.d * esize;
+  const int kg = rb / 64;   // per position: key groups, value groups
+  const int64_t hn = (int64_t)h * b.n_max;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N * 2 * kg; c += gridDim.x * blockDim.x) {
+    const int j = c / (2 * kg), grp = c - j * (2 * kg);
+    const int src = w.perm[hn + j];
+    if (src < 0 || src >= N) {
+      if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 8600 + h);
+      continue;
+    }
+    const int64_t so = ((int64_t)h * N + src) * rb, dof = ((int64_t)h * N + j) * rb;
+    if (grp < kg) copy64(reinterpret_cast<const uint4*>(Kc + so) + 4 * grp, reinterpret_cast<uint4*>(Kseq + dof) + 4 * grp);
+    else copy64(reinterpret_cast<const uint4*>(Vc + so) + 4 * (grp - kg), reinterpret_cast<uint4*>(Vseq + dof) + 4 * (grp - kg));
+    if (grp == 0) srcseq[(int64_t)h * N + j] = src;
   }
 }
 
@@ -863,12 +886,22 @@ cudaError_t launch_select(const Bank& b, const Ws& w, int eviction, cudaStream_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, cudaStream_t s, Timer* t) {
+cudaError_t launch_commit(const Bank& b, const Ws& w, const void* Vc, int N, const int32_t* src_map, cudaStream_t s,
+                          Timer* t) {
   // rows: ns survivors + r admitted = m_new <= M_max per head (grid-stride beyond)
   dim3 grid((b.M_max * (2 * b.d * (b.bf16 ? 2 : 4) / 64 + 1) + 255) / 256, b.H);
   timer_begin(t, "commit", s);
-  k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4);
+  k_commit<<<grid, 256, 0, s>>>(b, w, (const char*)Vc, N, b.bf16 ? 2 : 4, src_map);
   timer_end(t, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_gather(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, void* Kseq,
+                              void* Vseq, int32_t* srcseq, cudaStream_t s) {
+  const int kg = b.d * (b.bf16 ? 2 : 4) / 64;
+  dim3 grid((N * 2 * kg + 255) / 256, b.H);
+  k_seq_gather<<<grid, 256, 0, s>>>(b, w, (const char*)Kc, (const char*)Vc, N, b.bf16 ? 2 : 4, (char*)Kseq,
+                                    (char*)Vseq, srcseq);
   return cudaGetLastError();
 }
 

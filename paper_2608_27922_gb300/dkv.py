@@ -86,6 +86,8 @@ SIGNATURES = [
                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int32)]),
     ("dkv_candidate_order_noalloc", _I, [_P, _P, _I, _P, _I, _I, _I, ctypes.POINTER(dkv_params_t), _P, _P, _P]),
     ("dkv_selftest_wait_timeout", _I, [_I, ctypes.POINTER(ctypes.c_int64)]),
+    ("dkv_sequential_scratch_size", ctypes.c_size_t, [_I, _I, _I, _I]),
+    ("dkv_bank_update_sequential", _I, [_P, _P, _P, _I, ctypes.c_int64, _P, ctypes.c_size_t, _P]),
 ]
 
 DKV_NOALLOC_MAX_N = 16384
@@ -174,6 +176,16 @@ def dkv_bank_reset(bank: int, stream=None) -> None:
 
 def dkv_bank_admit(bank: int, Kc, Vc, N: int, step: int, stream=None) -> None:
     _check(lib().dkv_bank_admit(bank, _ptr(Kc), _ptr(Vc), N, step, _stream(stream)), "dkv_bank_admit")
+
+
+def dkv_sequential_scratch_size(H: int, d: int, n_max: int, dtype: int) -> int:
+    return int(lib().dkv_sequential_scratch_size(H, d, n_max, dtype))
+
+
+def dkv_bank_update_sequential(bank: int, Kc, Vc, N: int, step: int, scratch, scratch_bytes: int,
+                               stream=None) -> None:
+    _check(lib().dkv_bank_update_sequential(bank, _ptr(Kc), _ptr(Vc), N, step, _ptr(scratch), scratch_bytes,
+                                            _stream(stream)), "dkv_bank_update_sequential")
 
 
 def dkv_bank_compress(bank: int, stream=None) -> None:
@@ -355,6 +367,18 @@ class BankLayer:
     def update(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):
         self.admit(Kc, Vc, step, stream)
         self.compress(stream)
+
+    def update_sequential(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):
+        """Within-block competition: the block's candidates offered one at a time (the
+        C ABI's dkv_bank_update_sequential); synchronises once with the stream."""
+        N = Kc.shape[1]
+        self._chk(Kc, (self.H, N, self.d), "Kc")
+        self._chk(Vc, (self.H, N, self.d), "Vc")
+        if getattr(self, "_seq_scratch", None) is None:
+            n = dkv_sequential_scratch_size(self.H, self.d, self.n_max, self.dtype_code)
+            self._seq_scratch = torch.empty(n, dtype=torch.uint8, device=self.device)
+        dkv_bank_update_sequential(self.handle, Kc, Vc, N, step, self._seq_scratch, self._seq_scratch.numel(),
+                                   stream)
 
     def attend(self, Q: torch.Tensor, Kw: Optional[torch.Tensor], Vw: Optional[torch.Tensor],
                out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:

@@ -299,3 +299,56 @@ def test_bounded_wait_gives_up_and_context_stays_usable(dkv):
     assert st2 == 6
     wl = synth.get_workload("tiny_fp32_l1h2_d64", steps=3)
     _rollout(dkv, wl, "fp32", check_attn=False)
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_sequential_admission_matches_oracle(dkv, mode):
+    """Within-block competition (App. E): teacher-forced blocks, each offered one candidate
+    per head at a time in the order fixed at block start; the retained sets (keyed by
+    provenance) must match the oracle exactly, K/V bit for bit, rho and b within the
+    mode's density tolerance.  The first block (all heads empty) takes the whole block."""
+    import gpu_util
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=24, W=24, Nq=16, budgets=[56, 72], steps=6)
+    bank = _bank(dkv, wl, _mode(dkv, mode))
+    prm = gpu_util.oracle_params(bank)
+    _, dens = _tols(mode)
+    ro = synth.LayerRollout(wl, 0)
+    ob = oracle.LayerBank.empty(wl.budgets_of_layer(0), wl.d)
+    gated = 0
+    for t in range(wl.steps):
+        b = wl.admitted_block(t)
+        if b is None:
+            continue
+        K, V = ro.block(b)
+        load_state(bank, ob)
+        bank.update_sequential(to_dev(K, bank.dtype), to_dev(V, bank.dtype), b)
+        bank.sync()
+        recs = oracle.update_layer_sequential(ob, K, V, b, prm)
+        gated += sum(1 for r in recs if r.r_star == 0)
+        got, want = gpu_util.gpu_heads(bank), gpu_util.oracle_heads(ob)
+        for h in range(wl.H):
+            assert set(got[h]) == set(want[h]), (t, h, sorted(set(got[h]) ^ set(want[h]))[:6])
+            for key, (k, v, rho, base, _, _) in got[h].items():
+                wk, wv, wrho, wbase = want[h][key]
+                assert np.array_equal(k, wk.astype(np.float32)) and np.array_equal(v, wv.astype(np.float32)), key
+                assert abs(rho - wrho) <= dens * max(abs(wrho), 1e-30), (t, h, key, rho, wrho)
+                assert abs(base - wbase) <= dens * max(abs(wbase), 1e-30), (t, h, key, base, wbase)
+    assert gated > 0   # some offers were gated out: the candidates did compete
+    bank.close()
+
+
+def test_sequential_admission_call_errors(dkv):
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=8, budgets=16)
+    bank = _bank(dkv, wl, dkv.DKV_SCORE_FP32)
+    K = torch.randn(2, 8, 128, device="cuda").to(torch.bfloat16)
+    bank.update(K, K, 0)
+    bank.admit(K, K, 1)
+    with pytest.raises(dkv.DkvError) as e:          # between admit and commit
+        bank.update_sequential(K, K, 2)
+    assert e.value.status == 3
+    bank.compress()
+    bank.import_state([8, 0])                       # one head empty, one not
+    with pytest.raises(dkv.DkvError) as e:
+        bank.update_sequential(K, K, 2)
+    assert e.value.status == 3
+    bank.close()
