@@ -119,7 +119,8 @@ typedef struct {
                            updates or reads all layers with single kernel launches      */
 } dkv_params_t;
 
-/* Caller-owned device buffers of one layer's banks.  M_max = max_h budgets[h];
+/* Caller-owned device buffers of the handle's H per-head banks (one layer, or
+ * H / layer_heads layers stacked along heads).  M_max = max_h budgets[h];
  * head h's state lives in rows [h * M_max, h * M_max + budgets[h]).  Slots
  * [0, occupancy_h) of head h are the retained states; their order is not
  * meaningful (the bank is a set, Eq. 12).                                     */
