@@ -286,11 +286,13 @@ typedef struct {
 
 dkv_status_t dkv_bank_intermediates(dkv_bank_t bank, dkv_intermediates_t* out);
 
-/* Kernel timing: when enabled, every kernel the handle launches is bracketed
- * by CUDA events on its stream, and dkv_bank_kernel_times() returns, per
- * kernel name, the number of launches and the summed device milliseconds of
- * the launches whose events have completed (it synchronises).  Timing adds
- * two event records per launch; keep it off when not measuring.             */
+/* Kernel timing: enable = 1 brackets every kernel the handle launches with
+ * CUDA events on its stream, enable = 2 only the attention launches (0: off;
+ * other values: DKV_ERR_ARG).  dkv_bank_kernel_times() returns, per kernel
+ * name, the number of launches and the summed device milliseconds of the
+ * launches whose events have completed (it synchronises); with enable = 2 the
+ * other kernels are counted with 0 ms.  Timing adds two event records per
+ * timed launch; keep it off when not measuring.                             */
 dkv_status_t dkv_bank_set_timing(dkv_bank_t bank, int32_t enable);
 dkv_status_t dkv_bank_kernel_times(dkv_bank_t bank, int32_t max_kernels, char* names /* [max][48] */,
                                    int32_t* launches, double* total_ms, int32_t* n_kernels);

@@ -15,6 +15,7 @@ namespace dkv {
 // ------------------------------------------------------------------ timing hook
 struct Timer {
   bool on = false;
+  bool attend_only = false;   // bracket only the attention launches
   struct Rec {
     std::string name;
     cudaEvent_t a, b;
@@ -72,6 +73,16 @@ static void record(cudaEvent_t e, cudaStream_t s) {
 
 void timer_begin(Timer* t, const char* name, cudaStream_t s) {
   if (!t || !t->on) return;
+  if (t->attend_only && std::strncmp(name, "attend", 6) != 0) {   // counted, not timed
+    auto it = t->acc.find(name);
+    if (it == t->acc.end()) {
+      t->acc[name] = {1, 0.0};
+      t->order.push_back(name);
+    } else {
+      it->second.first += 1;
+    }
+    return;
+  }
   t->cur = name;
   t->cur_a = t->get();
   record(t->cur_a, s);
@@ -561,8 +572,10 @@ dkv_status_t dkv_bank_intermediates(dkv_bank_t bank, dkv_intermediates_t* out) {
 
 dkv_status_t dkv_bank_set_timing(dkv_bank_t bank, int32_t enable) {
   if (!bank) return DKV_ERR_ARG;
+  if (enable < 0 || enable > 2) return DKV_ERR_ARG;
   bank->timer.drain();
   bank->timer.on = enable != 0;
+  bank->timer.attend_only = enable == 2;
   if (!enable) {
     bank->timer.acc.clear();
     bank->timer.order.clear();

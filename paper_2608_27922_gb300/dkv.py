@@ -232,8 +232,9 @@ def dkv_bank_intermediates(bank: int) -> dkv_intermediates_t:
     return x
 
 
-def dkv_bank_set_timing(bank: int, enable: bool) -> None:
-    _check(lib().dkv_bank_set_timing(bank, 1 if enable else 0), "dkv_bank_set_timing")
+def dkv_bank_set_timing(bank: int, enable) -> None:
+    """enable: False/0 off, True/1 every kernel, 2 attention launches only (others counted)."""
+    _check(lib().dkv_bank_set_timing(bank, int(enable)), "dkv_bank_set_timing")
 
 
 def dkv_bank_kernel_times(bank: int) -> Dict[str, Tuple[int, float]]:
@@ -421,8 +422,8 @@ class BankLayer:
                 "rho_tilde": _view(x.rho_tilde, (H, M), torch.float32, self.device),
                 "slot_new": _view(x.slot_new, (H, n), torch.int32, self.device)}
 
-    def set_timing(self, on: bool):
-        dkv_bank_set_timing(self.handle, on)
+    def set_timing(self, on: bool, attention_only: bool = False):
+        dkv_bank_set_timing(self.handle, 2 if (on and attention_only) else int(bool(on)))
 
     def kernel_times(self):
         return dkv_bank_kernel_times(self.handle)

@@ -352,3 +352,28 @@ def test_sequential_admission_call_errors(dkv):
         bank.update_sequential(K, K, 2)
     assert e.value.status == 3
     bank.close()
+
+
+def test_kernel_timing_modes(dkv):
+    """set_timing(True) times every kernel; attention_only=True times only the attention
+    launches and counts the others (0 ms)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=2, N=64, W=64, Nq=64, budgets=128)
+    bank = _bank(dkv, wl, dkv.DKV_SCORE_TENSOR)
+    ro = synth.LayerRollout(wl, 0)
+    K, V = (to_dev(x, bank.dtype) for x in ro.block(0))
+    Q = to_dev(ro.queries(0), bank.dtype)
+    for only in (False, True):
+        bank.set_timing(True, attention_only=only)
+        bank.update(K, V, 0)
+        bank.attend(Q, K, V)
+        times = bank.kernel_times()
+        bank.set_timing(False)
+        assert times["attend_tc"][0] == 1 and times["attend_tc"][1] > 0
+        others = {k: v for k, v in times.items() if k != "attend_tc"}
+        assert others and all(n >= 1 for n, _ in others.values())
+        if only:
+            assert all(ms == 0 for _, ms in others.values())
+        else:
+            assert any(ms > 0 for _, ms in others.values())
+        bank.reset()
+    bank.close()
