@@ -217,7 +217,10 @@ dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream);
  * evicted slots, then appended), density maintenance of the survivors (Eq. C.4)
  * and the frozen baselines of the admitted states (Eq. 5).  Overwrites k, v and
  * occupancy: every reader of the pre-update bank (attention on another stream)
- * must be ordered before it.  Valid only right after evict (else DKV_ERR_STATE). */
+ * must be ordered before it.  Valid only right after evict (else DKV_ERR_STATE).
+ * The new baselines run on a stream owned by the handle, forked from and joined
+ * back into `stream` by events (also under stream capture); work enqueued on
+ * `stream` afterwards is ordered after all of it.                               */
 dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream);
 
 /* Bank-reading attention (Sec. 3.2, Fig. 2):

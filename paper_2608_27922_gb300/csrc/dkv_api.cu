@@ -170,6 +170,15 @@ struct dkv_bank_s {
   int state = 0;   // 0: idle, 1: admitted, 2: evicted
   int n_layers = 1;
   const int32_t* src_map = nullptr;   // provenance source index of each candidate (sequential admission)
+  // commit runs the survivor pass and the new-baselines pass side by side (they touch
+  // disjoint slots): the latter on this library-owned stream, forked and joined by events
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  ~dkv_bank_s() {
+    if (ev_fork) cudaEventDestroy(ev_fork);
+    if (ev_join) cudaEventDestroy(ev_join);
+    if (side) cudaStreamDestroy(side);
+  }
   const void* Kc = nullptr;
   const void* Vc = nullptr;
   int N = 0;
@@ -308,6 +317,12 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   bk->kp.order = p.order;
   bk->kp.eviction = p.eviction;
   bk->kp.refresh = p.refresh_baselines;
+  if (cudaStreamCreateWithFlags(&bk->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&bk->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&bk->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+    delete bk;
+    return DKV_ERR_CUDA;
+  }
   // workspace header: zeroed layer state and the per-head budgets (one-time, synchronous)
   cudaError_t e = cudaMemset(bk->w.L, 0, sizeof(DevLayer) * bk->n_layers);
   if (e == cudaSuccess) e = cudaMemset(bk->w.hd, 0, sizeof(DevHead) * H);
@@ -385,8 +400,15 @@ dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream) {
   bank->last = s;
   bank->state = 0;
   cudaError_t e = launch_commit(b, w, bank->Vc, bank->N, bank->src_map, s, t);
+  // Eq. C.4 (survivors) on `stream` beside Eq. 5 (admitted states) on the handle's own
+  // stream: disjoint slots, read-only inputs; `stream` waits for both
+  if (e == cudaSuccess) e = cudaEventRecord(bank->ev_fork, s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(bank->side, bank->ev_fork, 0);
+  if (e == cudaSuccess)
+    e = bank->tc ? launch_newbase_tc(b, w, kp, bank->side, t) : launch_newbase_fp32(b, w, kp, bank->side, t);
+  if (e == cudaSuccess) e = cudaEventRecord(bank->ev_join, bank->side);
   if (e == cudaSuccess) e = bank->tc ? launch_subtract_tc(b, w, kp, s, t) : launch_subtract_fp32(b, w, kp, s, t);
-  if (e == cudaSuccess) e = bank->tc ? launch_newbase_tc(b, w, kp, s, t) : launch_newbase_fp32(b, w, kp, s, t);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, bank->ev_join, 0);
   return cuda_status(e);
 }
 
