@@ -300,8 +300,14 @@ def run_ours(args):
                     bank.compress()
             return
         # attention, admit and evict only read the bank (the update is atomic from the
-        # reader's side), so they run concurrently; only the commit waits for attention
+        # reader's side); with one attention pass per update attention starts once admit has
+        # run, so the tensor-heavy score and crossing passes have the GPU to themselves and
+        # attention fills the latency-bound evict phase (several passes: attention dominates
+        # and starts at once); only the commit waits for attention
         cur = torch.cuda.current_stream(dev)
+        late = P == 1
+        if b is not None and late:
+            bank.admit(KC, VC, b, stream=cur)
         go = torch.cuda.Event()
         go.record(cur)
         side.wait_event(go)
@@ -310,7 +316,8 @@ def run_ours(args):
         done = torch.cuda.Event()
         done.record(side)
         if b is not None:
-            bank.admit(KC, VC, b, stream=cur)
+            if not late:
+                bank.admit(KC, VC, b, stream=cur)
             bank.evict(stream=cur)
         cur.wait_event(done)
         if b is not None:
@@ -460,6 +467,9 @@ def run_ours(args):
                     bank.admit(kc, vc, ab)
                     bank.compress()
             else:
+                late = P == 1
+                if ab is not None and late:
+                    bank.admit(kc, vc, ab, stream=cur)
                 go = torch.cuda.Event()
                 go.record(cur)
                 side.wait_event(go)
@@ -468,7 +478,8 @@ def run_ours(args):
                 att_done = torch.cuda.Event()
                 att_done.record(side)
                 if ab is not None:
-                    bank.admit(kc, vc, ab, stream=cur)
+                    if not late:
+                        bank.admit(kc, vc, ab, stream=cur)
                     bank.evict(stream=cur)
                 copy_s.wait_event(att_done)
                 with torch.cuda.stream(copy_s):
@@ -568,7 +579,8 @@ def run_ours(args):
                        "policy": {"order": args.order, "eviction": args.eviction,
                                   "refresh_baselines": bool(args.refresh_baselines),
                                   "within_block": args.within_block},
-                       "streams": "attention || admit + evict, then commit" if not args.no_overlap else "one stream",
+                       "streams": (("admit, then attention || evict" if P == 1 else "attention || admit + evict") + ", then commit")
+                       if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                        "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
@@ -725,6 +737,9 @@ def run_stack(args):
             cur = torch.cuda.current_stream(dev)
             b = wl.admitted_block(t)
             kw, vw = s_windows[t]
+            late = P == 1
+            if b is not None and late:
+                banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
             go = torch.cuda.Event()
             go.record(cur)
             side.wait_event(go)
@@ -733,7 +748,8 @@ def run_stack(args):
             done = torch.cuda.Event()
             done.record(side)
             if b is not None:
-                banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
+                if not late:
+                    banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
                 banks[0].evict(stream=cur)
             cur.wait_event(done)
             if b is not None:
@@ -827,8 +843,8 @@ def run_stack(args):
         "config": {"workload": f"{wl.name}: {L} layer(s) x {wl.H} heads per step, d={wl.d}, N={wl.N}, "
                                f"M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
                    "score_mode": args.score_mode, "layers_per_gpu": L,
-                   "streams": ("one handle over all layers (single launches), attention || admit + evict, "
-                               "then commit" if grouped else f"one handle per layer on {S} stream pairs"),
+                   "streams": ("one handle over all layers (single launches), admit, then attention || "
+                               "evict, then commit" if grouped else f"one handle per layer on {S} stream pairs"),
                    "cuda_graphs": True, "inputs": f"{D} distinct synthetic layer streams, reused round-robin",
                    "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                    "parallelism": "layers of one GPU, grouped launches" if grouped
