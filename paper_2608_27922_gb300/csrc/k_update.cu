@@ -864,8 +864,10 @@ cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s) {
 
 cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t) {
   const int max_runs = (b.n_max + RUN - 1) / RUN;
-  timer_begin(t, "sort", s);
+  timer_begin(t, "sort_runs", s);
   k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max, identity);
+  timer_end(t, s);
+  timer_begin(t, "sort_rank", s);
   k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(b, w, (const char*)Kc,
                                                                            b.bf16 ? 2 : 4, identity);
   timer_end(t, s);

@@ -92,3 +92,40 @@ def test_layer_heads_must_divide_heads(dkv):
         with pytest.raises(dkv.DkvError) as e:
             dkv.BankLayer(6, wl.d, wl.budgets_of_layer(0), 16, torch.bfloat16, layer_heads=bad)
         assert e.value.status == 1
+
+
+def test_grouped_layers_fullsize(dkv):
+    """Three Wan-1.3B-shaped layers (12 heads, N = 4,680, M = 9,360) in one handle against
+    three one-layer handles, bit for bit, over the first five steps (fill and eviction)."""
+    L = 3
+    wl = synth.get_workload("wan13b_stack_l30h12", L=L)
+    H, dt = wl.H, torch.bfloat16
+    sep = [dkv.BankLayer(H, wl.d, wl.budgets_of_layer(l), wl.N, dt) for l in range(L)]
+    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, dt, layer_heads=H)
+    for b in sep + [grp]:
+        b.reset()
+    ro = [synth.LayerRollout(wl, l) for l in range(L)]
+    evicted = 0
+    for t in range(5):
+        wins = [ro[l].window(t) for l in range(L)]
+        qs = [ro[l].queries(t) for l in range(L)]
+        o_sep = [sep[l].attend(to_dev(qs[l], dt), to_dev(wins[l][0], dt), to_dev(wins[l][1], dt)) for l in range(L)]
+        o_grp = grp.attend(_cat_heads(qs, dt), _cat_heads([w[0] for w in wins], dt), _cat_heads([w[1] for w in wins], dt))
+        b = wl.admitted_block(t)
+        if b is not None:
+            blocks = [ro[l].block(b) for l in range(L)]
+            for l in range(L):
+                sep[l].update(to_dev(blocks[l][0], dt), to_dev(blocks[l][1], dt), b)
+            grp.update(_cat_heads([x[0] for x in blocks], dt), _cat_heads([x[1] for x in blocks], dt), b)
+        torch.cuda.synchronize()
+        for bk in sep + [grp]:
+            bk.sync()
+        assert torch.equal(torch.cat(o_sep, 0), o_grp), t
+        for name in BUFFERS:
+            assert torch.equal(torch.cat([getattr(sep[l], name) for l in range(L)], 0), getattr(grp, name)), (t, name)
+        if b is not None:
+            assert [x.r_star for x in grp.layer_stats()] == [sep[l].stats()[0].r_star for l in range(L)], t
+            evicted += sum(h.evicted for h in grp.stats()[1])
+    assert evicted > 0
+    for bk in sep + [grp]:
+        bk.close()
