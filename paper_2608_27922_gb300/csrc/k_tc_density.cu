@@ -61,7 +61,10 @@ constexpr int OFF_A = 0;
 constexpr int OFF_AX = TILE_BYTES;
 constexpr int OFF_B = OFF_AX + EXT_BYTES;                 // [STAGES] tiles
 constexpr int OFF_BX = OFF_B + STAGES * TILE_BYTES;       // [STAGES] extension tiles
-constexpr int META_BUFS = 4;                              // score weights of tiles t, t+1, t+2, t+3
+// score weights of tiles t .. t+4: buffer t % 5 is refilled for tile t + 5 once the MMA
+// of tile t + 3 has completed, which needs every epilogue warp's release of tile t + 1,
+// given only after that warp finished tile t (the release can precede a tile's arithmetic)
+constexpr int META_BUFS = 5;
 constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [META_BUFS][BN]
 constexpr int OFF_XCH = OFF_META + META_BUFS * BN * 4;    // float [2][2][BM]
 constexpr int OFF_FLAG = OFF_XCH + 2 * 2 * BM * 4;      // int: last-arrival flag of split tiles
@@ -366,6 +369,7 @@ __global__ void __launch_bounds__(THREADS, 2)
         ok = __all_sync(0xffffffffu,
                         mbar_wait(bar_meta + t % META_BUFS, (t / META_BUFS) & 1, abort_flag));
       float tot[2] = {0.f, 0.f};
+      constexpr bool kEarlyRelease = MODE == TM_SCORE || MODE == TM_SUB || MODE == TM_NEWBASE;
       if (ok) {
         fence_after_sync();
 #pragma unroll
@@ -375,6 +379,13 @@ __global__ void __launch_bounds__(THREADS, 2)
           float v[32];
           tmem_ld32(lane_base + b * BN + cs, v);
           tmem_wait_ld();
+          // row-sum passes: after the warp's last TMEM load of the tile the accumulator is
+          // released before that chunk's arithmetic (the values are in registers)
+          if (kEarlyRelease && (ch == 1 || cs + 32 >= nc)) {
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile t + 2
+          }
           const int lim = min(32, nc - cs);
           if (MODE == TM_SCORE) {
             const float* ib = meta + (t % META_BUFS) * BN + cs;
@@ -441,7 +452,8 @@ __global__ void __launch_bounds__(THREADS, 2)
       } else {
         acc += tot[0] + tot[1];
       }
-      if (ok) {
+      // a warp whose half lies past the tile's last column loaded nothing: release here too
+      if (ok && (!kEarlyRelease || half * 64 >= nc)) {
         fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile t + 2
