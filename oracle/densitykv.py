@@ -33,6 +33,11 @@ What each function follows (paper sections / equations):
                          with scale 1/sqrt(d_k) (Sec. 3.2 logit definition,
                          App. A Eq. "supp-logit"; Fig. 2 caption).
 * ``storage_bytes``      App. D persistent-storage accounting.
+* ``rope_rezero``        App. A: memory keys carry temporal RoPE coordinate 0
+                         (spatial coordinates kept); offered keys that carry
+                         their frame's temporal rotation are rotated back.
+* ``round_nearest_bf16`` the storage rounding of rotated bf16 keys (nearest,
+                         ties to even), from its definition.
 
 Readings taken where the paper is silent or ambiguous (each is restated in
 the design notes of the repository):
@@ -79,6 +84,7 @@ __all__ = [
     "Params", "HeadBank", "LayerBank", "HeadRecord", "UpdateRecord",
     "soft_riesz", "sq_dist", "density", "potential_against",
     "update_layer", "update_layer_sequential", "block_order", "attend", "storage_bytes", "GIB",
+    "rope_rezero", "round_nearest_bf16",
 ]
 
 GIB = float(1 << 30)
@@ -448,6 +454,69 @@ def attend(hb: HeadBank, Q: np.ndarray, Kw: np.ndarray, Vw: np.ndarray) -> np.nd
     P = np.exp(S)
     P /= P.sum(axis=1, keepdims=True)
     return P @ Vall
+
+
+def round_nearest_bf16(x: np.ndarray) -> np.ndarray:
+    """Nearest bfloat16 value (8 significant bits, ties to even) of float64 values, as float64.
+
+    Written from the definition: x = m 2^e with 1/2 <= |m| < 1 (frexp, exact), the
+    significand scaled to 8 integer bits, rounded to the nearest integer with ties to even
+    (rint), and scaled back.  One rounding from float64, so no double rounding through
+    float32.  Normal range only (keys and values are O(1)); zeros stay zeros.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)
+    out = np.ldexp(np.rint(m * 256.0), e - 8)
+    nz = out[x != 0]
+    assert np.all(np.isfinite(out)) and np.all(np.abs(nz) >= 2.0 ** -126), "outside the bf16 normal range"
+    return out
+
+
+def rope_rezero(K: np.ndarray, t_coord: np.ndarray, theta: np.ndarray, layout: str = "interleaved",
+                storage: Optional[str] = "bf16") -> np.ndarray:
+    """Offered keys moved to temporal rotary coordinate 0 (App. A: the backbones attend to
+    nonlocal memory keys with the temporal RoPE coordinate set to 0 and the spatial ones
+    kept, and the bank stores exactly those keys).
+
+    K [H][N][d] carries, in every rotation pair j with theta_j != 0, the rotation by the
+    angle a = t_x theta_j of its token's temporal coordinate t_x (t_coord [N], shared by
+    the heads): a pair (x, y) of the unrotated key appears as
+    (x cos a - y sin a, x sin a + y cos a).  Setting the coordinate to 0 rotates it back
+    by -a:  x0 = x cos a + y sin a,  y0 = y cos a - x sin a.  Pairs with theta_j = 0
+    (the spatial bands) are left as they are.  layout "interleaved": pair j is elements
+    (2j, 2j+1); "half": (j, j + d/2).  theta is float32 [d/2]; the angle t theta is
+    formed exactly in float64 and the rotation evaluated in float64, then rounded once
+    to the storage precision ("bf16": nearest bfloat16, ties to even; "fp32": nearest
+    float32; None: the float64 values).
+    """
+    K = np.asarray(K, dtype=np.float64)
+    H, N, d = K.shape
+    th = np.asarray(theta, dtype=np.float32).astype(np.float64)
+    assert th.shape == (d // 2,)
+    t = np.asarray(t_coord, dtype=np.int64).astype(np.float64)
+    assert t.shape == (N,)
+    if layout == "interleaved":
+        xi, yi = np.arange(0, d, 2), np.arange(1, d, 2)
+    elif layout == "half":
+        xi, yi = np.arange(d // 2), np.arange(d // 2, d)
+    else:
+        raise ValueError(layout)
+    a = t[:, None] * th[None, :]                  # [N][d/2], exact in float64
+    c, s = np.cos(a), np.sin(a)
+    x, y = K[:, :, xi], K[:, :, yi]
+    out = K.copy()
+    out[:, :, xi] = x * c + y * s
+    out[:, :, yi] = y * c - x * s
+    keep = th == 0.0                              # unrotated pairs stay bit for bit
+    out[:, :, xi[keep]] = K[:, :, xi[keep]]
+    out[:, :, yi[keep]] = K[:, :, yi[keep]]
+    if storage is None:
+        return out
+    if storage == "bf16":
+        return round_nearest_bf16(out)
+    if storage == "fp32":
+        return out.astype(np.float32).astype(np.float64)
+    raise ValueError(storage)
 
 
 def storage_bytes(L: int, H: int, n: int, dk: int = 128, dv: int = 128,

@@ -15,7 +15,10 @@ Sources of truth used:
   * a worked example derived by hand with exact rational arithmetic;
   * the (eps, sigma) scale equivalence of App. B "Parameterization";
   * storage figures printed in App. D (golden file);
-  * textbook softmax attention (torch scaled_dot_product_attention in fp64).
+  * textbook softmax attention (torch scaled_dot_product_attention in fp64);
+  * brute-force nearest-value enumeration and torch's float32 -> bfloat16
+    conversion for the storage rounding; the rotary embedding written as complex
+    multiplication (RoFormer) for the temporal re-zeroing of App. A.
 """
 from __future__ import annotations
 
@@ -593,6 +596,112 @@ def check_sequential_admission(O):
         raise AssertionError("a partly empty bank was accepted")
 
 
+# --------------------------------------------------------------------------- storage rounding
+def _bf16_neighbours(v):
+    """Brute force: every bf16 value within two bf16 steps of v (8 significant bits)."""
+    if v == 0.0:
+        return [0.0]
+    e = math.floor(math.log2(abs(v)))
+    out = set()
+    for ee in (e - 1, e, e + 1):
+        step = 2.0 ** (ee - 7)
+        base = math.floor(abs(v) / step)
+        for k in range(base - 2, base + 3):
+            if 128 <= k < 256:
+                out.add(math.copysign(k * step, v))
+    return sorted(out)
+
+
+def check_round_nearest_bf16(O):
+    rng = np.random.default_rng(41)
+    # brute force: the nearest of the enumerated bf16 values, ties to the even significand
+    xs = np.concatenate([rng.normal(size=400) * 4.0, rng.uniform(-1e3, 1e3, size=100)])
+    got = O.round_nearest_bf16(xs)
+    for x, g in zip(xs, got):
+        cand = _bf16_neighbours(float(x))
+        best = min(abs(c - x) for c in cand)
+        near = [c for c in cand if abs(c - x) == best]
+        if len(near) == 2:       # tie: the one whose 8-bit significand is even
+            near = [c for c in near if int(abs(c) / 2.0 ** (math.floor(math.log2(abs(c))) - 7)) % 2 == 0]
+        assert g == near[0], (x, g, near)
+    # hand cases: ties to even around 1, and one float64 value just above a tie, which
+    # rounds up here but to the even neighbour 1 if it went through float32 first
+    hand = np.array([1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, 1 + 2.0 ** -8 + 2.0 ** -30, -(1 + 2.0 ** -8 + 2.0 ** -30),
+                     0.0, 255.0, 257.0, 259.0])
+    want = np.array([1.0, 1 + 2.0 ** -6, 1 + 2.0 ** -7, -(1 + 2.0 ** -7), 0.0, 255.0, 256.0, 260.0])
+    assert np.array_equal(O.round_nearest_bf16(hand), want), O.round_nearest_bf16(hand)
+    # float32 inputs: the library conversion (torch float32 -> bfloat16 rounds to nearest even)
+    import torch
+    f = (rng.normal(size=2000) * 3.0).astype(np.float32)
+    lib = torch.from_numpy(f).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(O.round_nearest_bf16(f.astype(np.float64)), lib)
+
+
+# --------------------------------------------------------------------------- App. A: temporal RoPE coordinate 0
+def _rope_forward(K0, t, theta, layout):
+    """Rotary embedding of temporal coordinate t written as complex multiplication:
+    pair j as z = x + i y, rotated to z e^{i t theta_j} (RoFormer convention)."""
+    K0 = np.asarray(K0, dtype=np.float64)
+    d = K0.shape[-1]
+    xi, yi = (np.arange(0, d, 2), np.arange(1, d, 2)) if layout == "interleaved" else \
+        (np.arange(d // 2), np.arange(d // 2, d))
+    z = K0[..., xi] + 1j * K0[..., yi]
+    z = z * np.exp(1j * np.asarray(t, dtype=np.float64)[:, None] * np.asarray(theta, np.float32).astype(np.float64))
+    out = K0.copy()
+    out[..., xi], out[..., yi] = z.real, z.imag
+    return out
+
+
+def check_rope_rezero(O):
+    rng = np.random.default_rng(43)
+    H, N, d = 2, 7, 16
+    theta = np.zeros(d // 2, dtype=np.float32)
+    theta[:3] = 10000.0 ** (-np.arange(3) / 3.0)      # a temporal band of three pairs; the rest spatial
+    t = np.array([0, 1, 1, 2, 5, 37, -4])
+    K0 = rng.normal(size=(H, N, d))
+    for layout in ("interleaved", "half"):
+        # rotating back undoes the forward embedding (the sign and direction of the angle)
+        Kt = _rope_forward(K0, t, theta, layout)
+        back = O.rope_rezero(Kt, t, theta, layout, storage=None)
+        assert np.allclose(back, K0, rtol=0, atol=1e-12), layout
+        # rotations keep norms and, at a common coordinate, inner products
+        assert np.allclose(np.linalg.norm(back, axis=-1), np.linalg.norm(Kt, axis=-1), rtol=1e-13)
+        same = t == 1
+        g1 = np.einsum("hnd,hmd->hnm", Kt[:, same], Kt[:, same])
+        g0 = np.einsum("hnd,hmd->hnm", back[:, same], back[:, same])
+        assert np.allclose(g0, g1, rtol=1e-12, atol=1e-12)
+        # coordinate 0 and the spatial pairs come back bit for bit
+        Kb = O.round_nearest_bf16(rng.normal(size=(H, N, d)))
+        out = O.rope_rezero(Kb, t, theta, layout)
+        assert np.array_equal(out[:, t == 0], Kb[:, t == 0])
+        sp = np.nonzero(theta == 0)[0]
+        idx = np.concatenate([2 * sp, 2 * sp + 1]) if layout == "interleaved" else np.concatenate([sp, sp + d // 2])
+        assert np.array_equal(out[..., idx], Kb[..., idx])
+        # the stored keys are the nearest bf16 values of the exact rotation
+        exact = O.rope_rezero(Kb, t, theta, layout, storage=None)
+        assert np.array_equal(out, O.round_nearest_bf16(exact))
+        assert np.array_equal(O.rope_rezero(Kb, t, theta, layout, storage="fp32"),
+                              exact.astype(np.float32).astype(np.float64))
+    # a quarter turn by hand: theta = pi/2 (as float32), t = 1: (x, y) -> (y, -x)
+    th = np.zeros(2, dtype=np.float32)
+    th[0] = np.float32(np.pi / 2)
+    k = np.array([[[3.0, 5.0, 7.0, 11.0]]])
+    q = O.rope_rezero(k, np.array([1]), th, "interleaved", storage=None)
+    assert np.allclose(q, [[[5.0, -3.0, 7.0, 11.0]]], rtol=0, atol=1e-6), q
+    q = O.rope_rezero(k, np.array([1]), th, "half", storage=None)     # pair 0 = elements (0, 2)
+    assert np.allclose(q, [[[7.0, 5.0, -3.0, 11.0]]], rtol=0, atol=1e-6), q
+    # two quarter turns are a half turn: t = 2 -> (-x, -y)
+    q = O.rope_rezero(k, np.array([2]), th, "interleaved", storage=None)
+    assert np.allclose(q, [[[-3.0, -5.0, 7.0, 11.0]]], rtol=0, atol=1e-6), q
+    # half layout is interleaved layout on the channel-permuted key
+    perm = np.empty(d, dtype=np.int64)
+    perm[0::2], perm[1::2] = np.arange(d // 2), np.arange(d // 2, d)
+    Kt = rng.normal(size=(H, N, d))
+    a = O.rope_rezero(Kt, t, theta, "half", storage=None)[..., perm]
+    b = O.rope_rezero(Kt[..., perm], t, theta, "interleaved", storage=None)
+    assert np.array_equal(a, b)
+
+
 ALL_CHECKS = [
     check_kernel_closed_forms,
     check_distance_identities,
@@ -607,4 +716,6 @@ ALL_CHECKS = [
     check_attention_textbook,
     check_policy_variants,
     check_sequential_admission,
+    check_round_nearest_bf16,
+    check_rope_rezero,
 ]

@@ -74,6 +74,13 @@ MUTANTS = [
     ("sequential_src_dropped", "adm_src = adm if src_index is None else np.asarray(src_index[h])[adm]",
      "adm_src = adm"),
     ("block_order_descending", '        out[h] = np.argsort(s, kind="stable")', '        out[h] = np.argsort(-s, kind="stable")'),
+    ("rope_x_sign", "out[:, :, xi] = x * c + y * s", "out[:, :, xi] = x * c - y * s"),
+    ("rope_y_sign", "out[:, :, yi] = y * c - x * s", "out[:, :, yi] = y * c + x * s"),
+    ("rope_half_as_interleaved", "        xi, yi = np.arange(d // 2), np.arange(d // 2, d)",
+     "        xi, yi = np.arange(0, d, 2), np.arange(1, d, 2)"),
+    ("rope_first_token_time", "a = t[:, None] * th[None, :]", "a = t[:1, None] * th[None, :]"),
+    ("bf16_ties_up", "out = np.ldexp(np.rint(m * 256.0), e - 8)", "out = np.ldexp(np.floor(m * 256.0 + 0.5), e - 8)"),
+    ("bf16_through_fp32", "m, e = np.frexp(x)", "m, e = np.frexp(x.astype(np.float32).astype(np.float64))"),
 ]
 
 
