@@ -83,11 +83,35 @@ def parse_args():
                     help="run attention and the update on one stream instead of overlapping them")
     ap.add_argument("--no-graphs", action="store_true",
                     help="launch every step directly instead of replaying a captured CUDA graph")
+    ap.add_argument("--rope", choices=["off", "interleaved", "half"], default="off",
+                    help="blocks arrive rotated to their frames' temporal RoPE coordinates and admit "
+                         "rotates them back to coordinate 0 (dkv_bank_admit_rope)")
     args = ap.parse_args()
     if args.within_block == "sequential":
         # the sequential path synchronises with its stream once per block: no graph capture
         args.no_graphs = args.no_overlap = args.no_e2e = True
+        if args.rope != "off":
+            ap.error("--rope applies to the batch admission path")
+    if args.rope != "off" and args.layers > 1:
+        ap.error("--rope is measured on the single-layer step")
     return args
+
+
+def rotate_to_frames(K, t, theta, layout):
+    """Input synthesis for --rope: keys as a backbone's local window holds them, each
+    rotation pair turned by its token's temporal coordinate (z -> z e^{i t theta}),
+    rounded to the key type.  Runs once before timing, with torch on the host."""
+    import torch
+    Kf = K.to(torch.float64)
+    d = Kf.shape[-1]
+    xi, yi = (slice(0, d, 2), slice(1, d, 2)) if layout == "interleaved" else (slice(0, d // 2), slice(d // 2, d))
+    a = torch.as_tensor(t, dtype=torch.float64)[:, None] * torch.as_tensor(theta).to(torch.float64)[None, :]
+    c, s_ = torch.cos(a), torch.sin(a)
+    x, y = Kf[..., xi], Kf[..., yi]
+    out = Kf.clone()
+    out[..., xi] = x * c - y * s_
+    out[..., yi] = x * s_ + y * c
+    return out.to(K.dtype)
 
 
 def dist_env():
@@ -268,6 +292,18 @@ def run_ours(args):
     n_total = W + K + (0 if args.no_e2e else K)
     inp = Inputs(wl, layer, n_total)
     bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    if args.rope != "off":
+        import synth
+        theta = synth.temporal_rope_theta(wl.d, layout_first=args.rope == "interleaved")
+        inp.blocks = {b: (rotate_to_frames(torch.from_numpy(k).to(bf), wl.frame_coords(b), theta, args.rope).float()
+                          .numpy(), v) for b, (k, v) in inp.blocks.items()}
+        theta_d = torch.from_numpy(theta).to(dev)
+        tco = {b: torch.from_numpy(wl.frame_coords(b)).to(dev) for b in inp.blocks}
+        rope_kw = lambda b, tbuf=None: dict(
+            t_coord=tco[b] if tbuf is None else tbuf, theta=theta_d,
+            rope_layout={"interleaved": dkv.DKV_ROPE_INTERLEAVED, "half": dkv.DKV_ROPE_HALF}[args.rope])
+    else:
+        rope_kw = lambda b, tbuf=None: {}
     dblocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
     dq = [torch.from_numpy(q).to(dev, bf) for q in inp.queries[:W + K]]
     cat1 = lambda xs: torch.cat(xs, dim=1).contiguous()
@@ -296,7 +332,7 @@ def run_ours(args):
                 if args.within_block == "sequential":
                     bank.update_sequential(KC, VC, b)
                 else:
-                    bank.admit(KC, VC, b)
+                    bank.admit(KC, VC, b, **rope_kw(b))
                     bank.compress()
             return
         # attention, admit and evict only read the bank (the update is atomic from the
@@ -307,7 +343,7 @@ def run_ours(args):
         cur = torch.cuda.current_stream(dev)
         late = P == 1
         if b is not None and late:
-            bank.admit(KC, VC, b, stream=cur)
+            bank.admit(KC, VC, b, stream=cur, **rope_kw(b))
         go = torch.cuda.Event()
         go.record(cur)
         side.wait_event(go)
@@ -317,7 +353,7 @@ def run_ours(args):
         done.record(side)
         if b is not None:
             if not late:
-                bank.admit(KC, VC, b, stream=cur)
+                bank.admit(KC, VC, b, stream=cur, **rope_kw(b))
             bank.evict(stream=cur)
         cur.wait_event(done)
         if b is not None:
@@ -408,12 +444,14 @@ def run_ours(args):
         cat_pin = lambda xs: torch.cat(xs, dim=1).contiguous().pin_memory()
         host_win = [inp.window(W + K + i, host_blocks, cat_pin) for i in range(K)]
         host_out = torch.empty(wl.H, wl.Nq, wl.d, dtype=bf).pin_memory()
+        host_tco = {b: torch.from_numpy(wl.frame_coords(b)).pin_memory() for b in inp.blocks}
         win_lens = sorted({hw[0].shape[1] for hw in host_win})
         # two device input sets (allocated before any capture)
         sets = []
         for _ in range(2):
             kb = torch.empty(wl.H, wl.N, wl.d, dtype=bf, device=dev)
             sets.append({"q": torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev), "k": kb, "v": torch.empty_like(kb),
+                         "t": torch.empty(wl.N, dtype=torch.int32, device=dev),
                          "win": {n: (torch.empty(wl.H, n, wl.d, dtype=bf, device=dev),
                                      torch.empty(wl.H, n, wl.d, dtype=bf, device=dev)) for n in win_lens}})
         copy_s = torch.cuda.Stream(dev)   # O download
@@ -433,7 +471,9 @@ def run_ours(args):
                 kc, vc = st["k"], st["v"]
             else:
                 kc, vc = kw, vw   # the block leaving the window is the window block
-            return ab, st["q"], kw, vw, kc, vc, pairs
+            if ab is not None and args.rope != "off":   # the block's temporal coordinates
+                pairs.append((st["t"], host_tco[ab]))
+            return ab, st["q"], kw, vw, kc, vc, st["t"], pairs
 
         def upload(pairs, after):
             """Copies host -> device on the upload stream after event `after`; returns its
@@ -450,7 +490,7 @@ def run_ours(args):
             cur = torch.cuda.current_stream(dev)
             start = torch.cuda.Event()
             start.record(cur)
-            ab, qbuf, kw, vw, kc, vc, pairs = inputs_of(i)
+            ab, qbuf, kw, vw, kc, vc, tbuf, pairs = inputs_of(i)
             nbytes = 0
             if i == 0:   # nothing was prefetched for the first timed step
                 ready, nbytes = upload(pairs, start)
@@ -464,12 +504,12 @@ def run_ours(args):
                     bank.attend(qbuf, kw, vw, out=out)
                 host_out.copy_(out, non_blocking=True)
                 if ab is not None:
-                    bank.admit(kc, vc, ab)
+                    bank.admit(kc, vc, ab, **rope_kw(ab, tbuf))
                     bank.compress()
             else:
                 late = P == 1
                 if ab is not None and late:
-                    bank.admit(kc, vc, ab, stream=cur)
+                    bank.admit(kc, vc, ab, stream=cur, **rope_kw(ab, tbuf))
                 go = torch.cuda.Event()
                 go.record(cur)
                 side.wait_event(go)
@@ -479,7 +519,7 @@ def run_ours(args):
                 att_done.record(side)
                 if ab is not None:
                     if not late:
-                        bank.admit(kc, vc, ab, stream=cur)
+                        bank.admit(kc, vc, ab, stream=cur, **rope_kw(ab, tbuf))
                     bank.evict(stream=cur)
                 copy_s.wait_event(att_done)
                 with torch.cuda.stream(copy_s):
@@ -578,7 +618,8 @@ def run_ours(args):
                        "attn_passes_per_update": max(1, args.attn_passes),
                        "policy": {"order": args.order, "eviction": args.eviction,
                                   "refresh_baselines": bool(args.refresh_baselines),
-                                  "within_block": args.within_block},
+                                  "within_block": args.within_block,
+                                  "rope_rezero": args.rope},
                        "streams": (("admit, then attention || evict" if P == 1 else "attention || admit + evict") + ", then commit")
                        if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,

@@ -200,6 +200,36 @@ dkv_status_t dkv_bank_reset(dkv_bank_t bank, void* stream);
 dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N,
                             int64_t step, void* stream);
 
+typedef enum {
+  DKV_ROPE_INTERLEAVED = 0,   /* rotation pair j = elements (2j, 2j + 1)  */
+  DKV_ROPE_HALF = 1           /* rotation pair j = elements (j, j + d/2)  */
+} dkv_rope_layout_t;
+
+/* dkv_bank_admit for keys that still carry their temporal rotary position.
+ * The backbones attend to nonlocal memory keys with the temporal RoPE coordinate
+ * set to 0 and the spatial coordinates kept, and the bank stores exactly those
+ * keys (App. A, "Attention-logit" setup).  Keys taken from a local window carry the
+ * rotation of their frame's coordinate t_x instead; this call first rotates every
+ * pair j with theta[j] != 0 back by the angle t_x * theta[j]:
+ *     x0 = x cos a + y sin a,  y0 = y cos a - x sin a,   a = t_x theta_j,
+ * stores the result rounded to nearest (ties to even) in the key type, and then
+ * runs admit on the stored keys (scores, order, crossings and the keys committed
+ * by the following compress are those of the re-zeroed keys).  Values are not
+ * rotated.  The rounding is that of the exact rotation (fp32 evaluation with an
+ * error bound, float64 where the bound cannot decide it).
+ *   t_coord : device int32 [N], temporal coordinate of each candidate (shared by
+ *             all heads and layers of the handle), 4-byte aligned.
+ *   theta   : device fp32 [d/2], angular frequency of each rotation pair; 0 for
+ *             pairs outside the temporal band (left bit for bit).
+ *   layout  : dkv_rope_layout_t.
+ * Both arrays are read during the call's work on `stream` only.  The re-zeroed
+ * keys live in the workspace until the following compress, so Kc may be reused
+ * once this call's work has completed.  Errors as dkv_bank_admit, plus
+ * DKV_ERR_ARG for a null or misaligned t_coord / theta or an unknown layout.   */
+dkv_status_t dkv_bank_admit_rope(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N,
+                                 int64_t step, const int32_t* t_coord, const float* theta,
+                                 int32_t layout, void* stream);
+
 /* Step 3 + commit for the block given to the preceding admit (Sec. 3.4;
  * Alg. 1; Eq. 12; Eq. C.4).  After it completes on `stream`, occupancy,
  * k, v, rho, base, knorm and provenance describe the committed banks.

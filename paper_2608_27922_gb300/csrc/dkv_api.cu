@@ -346,8 +346,8 @@ dkv_status_t dkv_bank_reset(dkv_bank_t bank, void* stream) {
   return cuda_status(cudaMemsetAsync(bank->b.occ, 0, sizeof(int32_t) * bank->b.H, s));
 }
 
-dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
-                            void* stream) {
+static dkv_status_t admit_impl(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
+                               const RopeArgs* rope, void* stream) {
   if (!bank || !Kc || !Vc) return DKV_ERR_ARG;
   if (bank->state != 0) return DKV_ERR_STATE;
   if (N < 1 || N > bank->b.n_max) return DKV_ERR_SHAPE;
@@ -358,7 +358,8 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   const Ws& w = bank->w;
   Timer* t = &bank->timer;
   bank->last = s;
-  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, bank->kp, s, t);
+  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, bank->kp, rope, s, t);
+  if (rope) Kc = w.kevict;   // the re-zeroed keys, same [H][N][d] layout
   if (e == cudaSuccess)
     if (bank->kp.order == DKV_ORDER_SCORE)   // source order needs no scores (App. E)
       e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
@@ -372,6 +373,20 @@ dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int
   bank->N = N;
   bank->step = step;
   return DKV_OK;
+}
+
+dkv_status_t dkv_bank_admit(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
+                            void* stream) {
+  return admit_impl(bank, Kc, Vc, N, step, nullptr, stream);
+}
+
+dkv_status_t dkv_bank_admit_rope(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
+                                 const int32_t* t_coord, const float* theta, int32_t layout, void* stream) {
+  if (!bank) return DKV_ERR_ARG;
+  if (!t_coord || !theta || !aligned(t_coord, 4) || !aligned(theta, 4)) return DKV_ERR_ARG;
+  if (layout != DKV_ROPE_INTERLEAVED && layout != DKV_ROPE_HALF) return DKV_ERR_ARG;
+  const RopeArgs ra{theta, t_coord, layout};
+  return admit_impl(bank, Kc, Vc, N, step, &ra, stream);
 }
 
 dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream) {
@@ -480,7 +495,7 @@ dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const v
   const Ws& w = bank->w;
   Timer* t = &bank->timer;
   const KParams& kp = bank->kp;
-  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, kp, s, t);
+  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, kp, nullptr, s, t);
   if (e == cudaSuccess && kp.order == DKV_ORDER_SCORE)
     e = bank->tc ? launch_score_tc(b, w, Kc, N, kp, s, t) : launch_score_fp32(b, w, Kc, N, kp, s, t);
   if (e == cudaSuccess) e = launch_sort(b, w, Kc, kp.order == DKV_ORDER_SOURCE, s, t);

@@ -40,7 +40,9 @@ struct Ws {
   float* rho_t;         // [H][M_max]     projected density rho~(r_h) (Eq. C.2)
   int32_t* evict_list;  // [H][n_max]     evicted slots, ascending
   int32_t* surv_list;   // [H][M_max]     surviving slots, ascending
-  void* kevict;         // [H][n_max][d]  keys of evicted states (gathered before commit)
+  void* kevict;         // [H][n_max][d]  keys of evicted states (written by commit, read by the
+                        //   survivor pass); during admit with temporal re-zeroing it holds
+                        //   the re-zeroed candidate keys, [H][N][d] like the caller's K_c
   float* kevict_norm;   // [H][n_max]
   void* ksurv;          // [H][M_max][d]  keys of surviving states
   float* ksurv_norm;    // [H][M_max]
@@ -60,6 +62,13 @@ struct Ws {
   int layer_heads;      // heads per layer (the handle's heads form H / layer_heads layers)
 };
 
+// Temporal rotary re-zeroing of the offered keys (App. A), device arrays of the caller.
+struct RopeArgs {
+  const float* theta;    // [d/2] angular frequency of rotation pair j (0: pair not rotated)
+  const int32_t* tpos;   // [N] temporal coordinate of each candidate (all heads)
+  int layout;            // 0: pair j = elements (2j, 2j + 1); 1: (j, j + d/2)
+};
+
 // Per-layer state of head h.
 __host__ __device__ inline DevLayer* layer_of(const Ws& w, int h) { return w.L + h / w.layer_heads; }
 
@@ -74,8 +83,9 @@ void timer_end(Timer* t, cudaStream_t s);
 // ---- launches (each returns cudaGetLastError() of its launch) ----
 // update front half (admit)
 // candidates' norms and extension rows, zeroed crossing histogram, update snapshot
+// (rope != nullptr: the keys re-zeroed into w.kevict first, norms of the stored keys)
 cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
-                              cudaStream_t s, Timer* t);
+                              const RopeArgs* rope, cudaStream_t s, Timer* t);
 cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t);
 cudaError_t launch_cross_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);

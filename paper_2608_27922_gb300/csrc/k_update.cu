@@ -1,7 +1,9 @@
 // Selection, ordering and compaction kernels of the bank update (no pair math).
 //
 //   cand_norms   ||k_x||^2 of the candidates (fp32) and their extension rows, plus (one
-//                extra block) the snapshot of occupancy, budgets and prefix range
+//                extra block) the snapshot of occupancy, budgets and prefix range; with
+//                temporal re-zeroing (App. A) the keys are first rotated back to temporal
+//                rotary coordinate 0 and stored, and the norms taken of the stored keys
 //   sort         stable ascending order of the Eq. 6 scores, ties by source index (Alg. 1),
 //                and the candidate keys copied into that order (operand of the prefix passes)
 //   rstar_*      violator counts c_r = #{cross <= r}, budgets e_r (Eq. 10), feasibility,
@@ -142,21 +144,12 @@ __device__ __forceinline__ float sq_sum(const T* p, int pl) {
 // with all loads issued before the reductions.
 constexpr int NR_ROWS = 4;
 
-template <typename T>
-__device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t head_stride, int rows_cap,
-                                               const int32_t* count, int count_is_occ, int N,
-                                               float* __restrict__ out, int64_t out_hs, int d,
-                                               __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
-  const int h = blockIdx.y;
-  const int row0 = (blockIdx.x * (blockDim.x / 32) + warp_id()) * NR_ROWS;
-  const int n = min(count_is_occ ? count[h] : N, rows_cap);
-  if (row0 >= n) return;
-  const int pl = d / 32;
+// Warp reduction of the lanes' partial squares a[q] of rows row0 + q (< n), then the
+// norm and (ext != nullptr) the extension row of each.
+__device__ __forceinline__ void norms_ext_tail(float* a, int h, int row0, int n, float* __restrict__ out,
+                                               int64_t out_hs, __nv_bfloat16* __restrict__ ext, int64_t ext_hs,
+                                               float goff) {
   const int l = lane_id();
-  float a[NR_ROWS];
-#pragma unroll
-  for (int q = 0; q < NR_ROWS; ++q)
-    a[q] = row0 + q < n ? sq_sum<T>(K + (int64_t)h * head_stride + (int64_t)(row0 + q) * d + l * pl, pl) : 0.f;
 #pragma unroll
   for (int q = 0; q < NR_ROWS; ++q)
 #pragma unroll
@@ -177,6 +170,150 @@ __device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t 
       else if (l >= 16 && l < 19) v = one;
       else if (l >= 19 && l < 22) v = hh[l - 19];
       ext[(int64_t)h * ext_hs + (int64_t)row * 32 + l] = v;
+    }
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t head_stride, int rows_cap,
+                                               const int32_t* count, int count_is_occ, int N,
+                                               float* __restrict__ out, int64_t out_hs, int d,
+                                               __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
+  const int h = blockIdx.y;
+  const int row0 = (blockIdx.x * (blockDim.x / 32) + warp_id()) * NR_ROWS;
+  const int n = min(count_is_occ ? count[h] : N, rows_cap);
+  if (row0 >= n) return;
+  const int pl = d / 32;
+  const int l = lane_id();
+  float a[NR_ROWS];
+#pragma unroll
+  for (int q = 0; q < NR_ROWS; ++q)
+    a[q] = row0 + q < n ? sq_sum<T>(K + (int64_t)h * head_stride + (int64_t)(row0 + q) * d + l * pl, pl) : 0.f;
+  norms_ext_tail(a, h, row0, n, out, out_hs, ext, ext_hs, goff);
+}
+
+// ---- temporal rotary re-zeroing (App. A: memory keys carry temporal coordinate 0) ----
+// A rotation pair (x, y) of a key rotated by a = t theta (t the token's temporal
+// coordinate) is moved back by -a:  x0 = x cos a + y sin a,  y0 = y cos a - x sin a,
+// i.e. rot(u, v) = u cos a + v sin a with (u, v) = (x, y) and (y, -x).  The stored value is
+// the nearest value of the key's type (ties to even) to the exact rotation.
+//
+// cos a and sin a come from a per-CTA table: float64 sincos of the exact float64 angle,
+// once per distinct coordinate among the CTA's rows and pair (not per element or head).
+// bf16 keys: r = u c + v s in fp32 with c, s the table values rounded to fp32
+// (|c - cos a|, |s - sin a| <= 2^-24.99), so |r - exact| <= 2^-24 (|u| + 2 |v| + |r|) < E.
+// Rounding is monotone: when both ends of [r - E, r + E] (rounded outwards) give the
+// same bf16 value, that is the rounding of the exact rotation; otherwise (about 1
+// element in 2,000) r is taken in float64 from the float64 table.  fp32 keys: float64.
+
+// float64 evaluation rounded once to the key type: bf16 through float32 rounded to odd
+// (exact for a later rounding to 8 significant bits).
+template <typename T>
+__device__ __forceinline__ float rot_f64(float u, float v, double c, double s) {
+  const double r = (double)u * c + (double)v * s;
+  if constexpr (sizeof(T) == 4) {
+    return __double2float_rn(r);
+  } else {
+    float f = __double2float_rz(r);
+    if ((double)f != r) f = __uint_as_float(__float_as_uint(f) | 1u);
+    return __bfloat162float(__float2bfloat16_rn(f));
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ float rot_tab(float u, float v, float c, float s, double cd, double sd) {
+  if constexpr (sizeof(T) == 2) {
+    const float r = fmaf(u, c, v * s);
+    const float E = 0x1p-23f * (fabsf(u) + fabsf(v) + fabsf(r)) + 0x1p-126f;
+    const __nv_bfloat16 lo = __float2bfloat16_rn(__fsub_rd(r, E));
+    const __nv_bfloat16 hi = __float2bfloat16_rn(__fadd_ru(r, E));
+    if (__bfloat16_as_ushort(lo) == __bfloat16_as_ushort(hi)) return __bfloat162float(lo);
+  }
+  return rot_f64<T>(u, v, cd, sd);
+}
+
+template <typename T>
+__device__ __forceinline__ void load_lane(const T* p, int pl, float* x) {
+  if constexpr (sizeof(T) == 2) {
+    if (pl == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(p);
+      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+      const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+      x[0] = __low2float(a); x[1] = __high2float(a); x[2] = __low2float(c); x[3] = __high2float(c);
+    } else {
+      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(p);
+      x[0] = __low2float(a); x[1] = __high2float(a); x[2] = 0.f; x[3] = 0.f;
+    }
+  } else {
+    if (pl == 4) {
+      const float4 f = *reinterpret_cast<const float4*>(p);
+      x[0] = f.x; x[1] = f.y; x[2] = f.z; x[3] = f.w;
+    } else {
+      const float2 f = *reinterpret_cast<const float2*>(p);
+      x[0] = f.x; x[1] = f.y; x[2] = 0.f; x[3] = 0.f;
+    }
+  }
+}
+
+// Stores values that are exactly representable in T.
+template <typename T>
+__device__ __forceinline__ void store_lane(T* p, int pl, const float* x) {
+  if constexpr (sizeof(T) == 2) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(x[0], x[1]);
+    if (pl == 4) {
+      const __nv_bfloat162 c = __floats2bfloat162_rn(x[2], x[3]);
+      uint2 u;
+      u.x = *reinterpret_cast<const uint32_t*>(&a);
+      u.y = *reinterpret_cast<const uint32_t*>(&c);
+      *reinterpret_cast<uint2*>(p) = u;
+    } else {
+      *reinterpret_cast<__nv_bfloat162*>(p) = a;
+    }
+  } else {
+    if (pl == 4) *reinterpret_cast<float4*>(p) = make_float4(x[0], x[1], x[2], x[3]);
+    else *reinterpret_cast<float2*>(p) = make_float2(x[0], x[1]);
+  }
+}
+
+constexpr int ROPE_ROWS = 8;   // candidate rows per CTA of the re-zeroing prepare (all heads)
+
+struct RopeTab {
+  float th[64];                    // theta_j
+  int t[ROPE_ROWS];                // temporal coordinate of each row
+  int lead[ROPE_ROWS];             // first row of the CTA with the same coordinate
+  float cf[ROPE_ROWS][64], sf[ROPE_ROWS][64];     // cos / sin rounded to fp32 (leader rows)
+  double cd[ROPE_ROWS][64], sd[ROPE_ROWS][64];    // cos / sin in float64
+};
+
+// The lane's pl elements (from element e0 of a row of the CTA's table row q) rotated back.
+// Interleaved layout: the lane holds whole pairs.  Half layout: the partner of element e
+// is e +- d/2, held by lane l ^ 16 at the same position (called by all 32 lanes).
+template <typename T>
+__device__ __forceinline__ void rope_lane(float* x, int pl, int e0, int d, int layout, const RopeTab& tb, int q) {
+  const int t = tb.t[q];
+  const int k = tb.lead[q];
+  if (layout == 0) {
+#pragma unroll
+    for (int i = 0; i < 4; i += 2) {
+      if (i >= pl) break;
+      const int j = (e0 + i) >> 1;
+      if (tb.th[j] == 0.f || t == 0) continue;
+      const float u = x[i], v = x[i + 1];
+      x[i] = rot_tab<T>(u, v, tb.cf[k][j], tb.sf[k][j], tb.cd[k][j], tb.sd[k][j]);
+      x[i + 1] = rot_tab<T>(v, -u, tb.cf[k][j], tb.sf[k][j], tb.cd[k][j], tb.sd[k][j]);
+    }
+  } else {
+    const int half = d / 2;
+    const bool first = e0 < half;
+    float o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = __shfl_xor_sync(0xffffffffu, x[i], 16);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (i >= pl) break;
+      const int j = (e0 + i) % half;
+      if (tb.th[j] == 0.f || t == 0) continue;
+      x[i] = rot_tab<T>(x[i], first ? o[i] : -o[i], tb.cf[k][j], tb.sf[k][j], tb.cd[k][j], tb.sd[k][j]);
     }
   }
 }
@@ -206,6 +343,70 @@ __global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, int N, in
   }
   row_norms_body<T>(Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm, b.n_max, b.d, (__nv_bfloat16*)w.cext,
                     (int64_t)b.n_max * 32, goff);
+}
+
+// k_cand_prepare with temporal re-zeroing: CTA x takes candidate rows [8x, 8x + 8) of every
+// head.  It builds the cos / sin table of its rows' distinct coordinates, then its warps
+// take batches of NR_ROWS rows of one head: rotated back into w.kevict ([H][N][d], the
+// layout of Kc), norms and extension rows of the stored keys.  Last CTA: prepare_body.
+template <typename T>
+__global__ void __launch_bounds__(256) k_cand_prepare_rope(Bank b, Ws w, const T* __restrict__ Kc, int N,
+                                                           int64_t step, float goff, const RopeArgs ra) {
+  if (blockIdx.x == gridDim.x - 1) {
+    prepare_body(b, w, N, step);
+    return;
+  }
+  {
+    const int64_t nh = (int64_t)b.H * w.hist_stride;
+    const int64_t nthr = (int64_t)(gridDim.x - 1) * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nh; i += nthr) w.hist[i] = 0;
+  }
+  __shared__ RopeTab tb;
+  const int d = b.d, P = d / 2;
+  const int x0 = blockIdx.x * ROPE_ROWS;
+  const int nr = min(ROPE_ROWS, N - x0);
+  if (threadIdx.x < P) tb.th[threadIdx.x] = __ldg(ra.theta + threadIdx.x);
+  if (threadIdx.x < nr) tb.t[threadIdx.x] = __ldg(ra.tpos + x0 + threadIdx.x);
+  __syncthreads();
+  if (threadIdx.x < nr) {
+    int k = threadIdx.x;
+    for (int q = 0; q < (int)threadIdx.x; ++q)
+      if (tb.t[q] == tb.t[threadIdx.x]) { k = q; break; }
+    tb.lead[threadIdx.x] = k;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < nr * P; i += blockDim.x) {
+    const int q = i / P, j = i % P;
+    if (tb.lead[q] != q) continue;
+    double sv = 0.0, cv = 1.0;
+    if (tb.th[j] != 0.f && tb.t[q] != 0) sincos((double)tb.t[q] * (double)tb.th[j], &sv, &cv);
+    tb.cd[q][j] = cv;
+    tb.sd[q][j] = sv;
+    tb.cf[q][j] = (float)cv;
+    tb.sf[q][j] = (float)sv;
+  }
+  __syncthreads();
+  T* __restrict__ Kout = (T*)w.kevict;
+  const int pl = d / 32, l = lane_id();
+  const int nw = blockDim.x / 32;
+  for (int base = warp_id() * NR_ROWS; base < b.H * ROPE_ROWS; base += nw * NR_ROWS) {
+    const int h = base / ROPE_ROWS, q0 = base % ROPE_ROWS;   // NR_ROWS divides ROPE_ROWS: one head
+    if (q0 >= nr) continue;                                    // warp-uniform
+    float x[NR_ROWS][4];
+#pragma unroll
+    for (int q = 0; q < NR_ROWS; ++q)
+      if (q0 + q < nr) load_lane<T>(Kc + ((int64_t)h * N + x0 + q0 + q) * d + l * pl, pl, x[q]);
+    float a[NR_ROWS];
+#pragma unroll
+    for (int q = 0; q < NR_ROWS; ++q) {
+      a[q] = 0.f;
+      if (q0 + q >= nr) continue;                              // warp-uniform
+      rope_lane<T>(x[q], pl, l * pl, d, ra.layout, tb, q0 + q);
+      store_lane<T>(Kout + ((int64_t)h * N + x0 + q0 + q) * d + l * pl, pl, x[q]);
+      a[q] = fmaf(x[q][3], x[q][3], fmaf(x[q][2], x[q][2], fmaf(x[q][1], x[q][1], x[q][0] * x[q][0])));
+    }
+    norms_ext_tail(a, h, x0 + q0, x0 + nr, w.cnorm, b.n_max, (__nv_bfloat16*)w.cext, (int64_t)b.n_max * 32, goff);
+  }
 }
 
 // Sort of the keys (fkey(score) << 32 | source index) per head: ascending score, equal
@@ -830,13 +1031,20 @@ __global__ void k_seq_gather(Bank b, Ws w, const char* __restrict__ Kc, const ch
 static float ext_goff(const KParams& kp) { return kp.eps * 0.5f / kp.inv_s2; }   // eps sigma^2 / 2
 
 cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
-                              cudaStream_t s, Timer* t) {
+                              const RopeArgs* rope, cudaStream_t s, Timer* t) {
   dim3 grid((N + 8 * NR_ROWS - 1) / (8 * NR_ROWS) + 1, b.H);   // + the prepare block
   timer_begin(t, "cand_norms", s);
-  if (b.bf16)
+  if (rope) {
+    const dim3 rgrid((N + ROPE_ROWS - 1) / ROPE_ROWS + 1);   // + the prepare block
+    if (b.bf16)
+      k_cand_prepare_rope<__nv_bfloat16><<<rgrid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, N, step, ext_goff(kp), *rope);
+    else
+      k_cand_prepare_rope<float><<<rgrid, 256, 0, s>>>(b, w, (const float*)Kc, N, step, ext_goff(kp), *rope);
+  } else if (b.bf16) {
     k_cand_prepare<__nv_bfloat16><<<grid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, N, step, ext_goff(kp));
-  else
+  } else {
     k_cand_prepare<float><<<grid, 256, 0, s>>>(b, w, (const float*)Kc, N, step, ext_goff(kp));
+  }
   timer_end(t, s);
   return cudaGetLastError();
 }

@@ -72,6 +72,7 @@ SIGNATURES = [
     ("dkv_bank_destroy", None, [_P]),
     ("dkv_bank_reset", _I, [_P, _P]),
     ("dkv_bank_admit", _I, [_P, _P, _P, _I, ctypes.c_int64, _P]),
+    ("dkv_bank_admit_rope", _I, [_P, _P, _P, _I, ctypes.c_int64, _P, _P, _I, _P]),
     ("dkv_bank_compress", _I, [_P, _P]),
     ("dkv_bank_evict", _I, [_P, _P]),
     ("dkv_bank_commit", _I, [_P, _P]),
@@ -176,6 +177,14 @@ def dkv_bank_reset(bank: int, stream=None) -> None:
 
 def dkv_bank_admit(bank: int, Kc, Vc, N: int, step: int, stream=None) -> None:
     _check(lib().dkv_bank_admit(bank, _ptr(Kc), _ptr(Vc), N, step, _stream(stream)), "dkv_bank_admit")
+
+
+DKV_ROPE_INTERLEAVED, DKV_ROPE_HALF = 0, 1
+
+
+def dkv_bank_admit_rope(bank: int, Kc, Vc, N: int, step: int, t_coord, theta, layout: int, stream=None) -> None:
+    _check(lib().dkv_bank_admit_rope(bank, _ptr(Kc), _ptr(Vc), N, step, _ptr(t_coord), _ptr(theta), layout,
+                                     _stream(stream)), "dkv_bank_admit_rope")
 
 
 def dkv_sequential_scratch_size(H: int, d: int, n_max: int, dtype: int) -> int:
@@ -347,12 +356,24 @@ class BankLayer:
     def reset(self, stream=None):
         dkv_bank_reset(self.handle, stream)
 
-    def admit(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):
+    def admit(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None, t_coord=None, theta=None,
+              rope_layout: int = DKV_ROPE_INTERLEAVED):
+        """Steps 1-2.  With t_coord (int32 [N]) and theta (fp32 [d/2]) on the device, the
+        keys are first rotated back to temporal rotary coordinate 0 (dkv_bank_admit_rope)."""
         N = Kc.shape[1]
         self._chk(Kc, (self.H, N, self.d), "Kc")
         self._chk(Vc, (self.H, N, self.d), "Vc")
-        self._pending = (Kc, Vc)   # keep the candidates alive until commit
-        dkv_bank_admit(self.handle, Kc, Vc, N, step, stream)
+        if (t_coord is None) != (theta is None):
+            raise ValueError("t_coord and theta go together")
+        if t_coord is None:
+            self._pending = (Kc, Vc)   # keep the candidates alive until commit
+            dkv_bank_admit(self.handle, Kc, Vc, N, step, stream)
+            return
+        for x, dt, shape, name in ((t_coord, torch.int32, (N,), "t_coord"), (theta, torch.float32, (self.d // 2,), "theta")):
+            if x.dtype != dt or tuple(x.shape) != shape or not x.is_contiguous() or x.device != self.device:
+                raise ValueError(f"{name}: expected contiguous {dt} {shape} on {self.device}")
+        self._pending = (Kc, Vc, t_coord, theta)
+        dkv_bank_admit_rope(self.handle, Kc, Vc, N, step, t_coord, theta, rope_layout, stream)
 
     def compress(self, stream=None):
         dkv_bank_compress(self.handle, stream)
@@ -365,8 +386,8 @@ class BankLayer:
         """Second half of compress; order every reader of the old bank before it."""
         dkv_bank_commit(self.handle, stream)
 
-    def update(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):
-        self.admit(Kc, Vc, step, stream)
+    def update(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None, **rope):
+        self.admit(Kc, Vc, step, stream, **rope)
         self.compress(stream)
 
     def update_sequential(self, Kc: torch.Tensor, Vc: torch.Tensor, step: int, stream=None):

@@ -51,12 +51,31 @@ __all__ = [
     "get_workload",
     "LayerRollout",
     "round_to_bf16",
+    "temporal_rope_theta",
     "sample_vmf",
     "make_workload",
 ]
 
 # stream ids inside a (layer, head, step) seed key
 _S_CENTRES, _S_ASSIGN, _S_KEYS, _S_VALUES, _S_QUERIES, _S_QASSIGN, _S_HEADPARAMS = range(7)
+
+
+def temporal_rope_theta(d: int, band_pairs: Optional[int] = None, base: float = 10000.0,
+                        layout_first: bool = True) -> np.ndarray:
+    """Angular frequencies [d/2] (float32) of a 3-D rotary layout whose temporal band is
+    band_pairs rotation pairs (default: a third of the pairs, rounded down, 21 of 64 at
+    d = 128) with RoFormer frequencies base^(-j / band_pairs); the spatial pairs get 0
+    (their rotations are not touched by temporal re-zeroing).  The band is the first
+    pairs (layout_first) or the last ones."""
+    P = d // 2
+    n = P // 3 if band_pairs is None else band_pairs
+    th = np.zeros(P, dtype=np.float32)
+    band = (base ** (-np.arange(n, dtype=np.float64) / n)).astype(np.float32)
+    if layout_first:
+        th[:n] = band
+    else:
+        th[P - n:] = band
+    return th
 
 
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
@@ -156,6 +175,14 @@ class Workload:
             # after step t the 5-frame window starts at frame 3t - 2: block t - 2 has left it
             return t - 2 if t >= 2 else None
         return t - 1 if t >= 1 else None
+
+    def frame_coords(self, b: int) -> np.ndarray:
+        """Temporal coordinate (latent frame index) of each token of block b, int32 [N]:
+        block b holds frames frames_per_block * b ... in raster order of N / frames_per_block
+        tokens each."""
+        per = self.N // self.frames_per_block
+        return (self.frames_per_block * b + np.minimum(np.arange(self.N) // per,
+                                                       self.frames_per_block - 1)).astype(np.int32)
 
     def window_block(self, t: int) -> int:
         """Index of the block whose K/V form the local window read at step t (whole-block

@@ -109,18 +109,27 @@ def _g_row(hb: oracle.HeadBank, i: int, Kpi: np.ndarray, r: int, prm: oracle.Par
 
 
 def update_and_compare(bank: dkv.BankLayer, ob: oracle.LayerBank, K: np.ndarray, V: np.ndarray, step: int,
-                       tol: float, dens_tol: float) -> Tuple[Report, oracle.UpdateRecord]:
+                       tol: float, dens_tol: float, rope=None) -> Tuple[Report, oracle.UpdateRecord]:
     """Teacher-forced update: the GPU starts from the oracle's bank; both apply one update.
 
     tol: relative window within which a decision may differ (near-tie of s, g vs tau,
     rho~ vs the fill cutoff).  dens_tol: relative tolerance of s, rho~, rho and b.
-    ``ob`` is advanced by the oracle's update.
+    ``ob`` is advanced by the oracle's update.  rope = (t_coord, theta, layout): K carries
+    the temporal rotation; the GPU re-zeroes it in admit, the oracle updates with
+    ``oracle.rope_rezero`` of it.
     """
     prm = oracle_params(bank)
     before = ob.copy()
     load_state(bank, before)
     Kd, Vd = to_dev(K, bank.dtype), to_dev(V, bank.dtype)
-    bank.admit(Kd, Vd, step)
+    if rope is not None:
+        t_coord, theta, layout = rope
+        bank.admit(Kd, Vd, step, t_coord=torch.from_numpy(np.asarray(t_coord, np.int32)).to(bank.device),
+                   theta=torch.from_numpy(np.asarray(theta, np.float32)).to(bank.device),
+                   rope_layout={"interleaved": 0, "half": 1}[layout])
+        K = oracle.rope_rezero(K, t_coord, theta, layout, "bf16" if bank.dtype == torch.bfloat16 else "fp32")
+    else:
+        bank.admit(Kd, Vd, step)
     bank.compress()
     bank.sync()
     rec = oracle.update_layer(ob, K, V, step, prm)

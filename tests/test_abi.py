@@ -106,6 +106,7 @@ def test_host_only_entry_points():
     h = ctypes.c_void_p()
     assert L.dkv_bank_create(ctypes.byref(h), 2, 64, None, 16, 1, None, None) == 1
     assert L.dkv_bank_admit(None, None, None, 1, 0, None) == 1
+    assert L.dkv_bank_admit_rope(None, None, None, 1, 0, None, None, 0, None) == 1
     assert L.dkv_bank_compress(None, None) == 1
     assert L.dkv_bank_evict(None, None) == 1
     assert L.dkv_bank_commit(None, None) == 1
