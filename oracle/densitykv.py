@@ -38,6 +38,8 @@ What each function follows (paper sections / equations):
                          their frame's temporal rotation are rotated back.
 * ``round_nearest_bf16`` the storage rounding of rotated bf16 keys (nearest,
                          ties to even), from its definition.
+* ``kv_descriptor``      App. E "Retention geometry": the [K; V] descriptor, run
+                         through the same update in place of the keys.
 
 Readings taken where the paper is silent or ambiguous (each is restated in
 the design notes of the repository):
@@ -84,7 +86,7 @@ __all__ = [
     "Params", "HeadBank", "LayerBank", "HeadRecord", "UpdateRecord",
     "soft_riesz", "sq_dist", "density", "potential_against",
     "update_layer", "update_layer_sequential", "block_order", "attend", "storage_bytes", "GIB",
-    "rope_rezero", "round_nearest_bf16",
+    "rope_rezero", "round_nearest_bf16", "kv_descriptor",
 ]
 
 GIB = float(1 << 30)
@@ -454,6 +456,18 @@ def attend(hb: HeadBank, Q: np.ndarray, Kw: np.ndarray, Vw: np.ndarray) -> np.nd
     P = np.exp(S)
     P /= P.sum(axis=1, keepdims=True)
     return P @ Vall
+
+
+def kv_descriptor(K: np.ndarray, V: np.ndarray) -> np.ndarray:
+    """App. E "Retention geometry": the [K; V] descriptor of each state, its key and value
+    concatenated (2 d_k values), float64.
+
+    The [K; V] policy is the same algorithm with these rows in place of the keys: a
+    LayerBank of dimension 2 d_k updated by ``update_layer(bank, kv_descriptor(Kc, Vc),
+    Vc, ...)``; sigma defaults to sqrt(2 d_k / 2) = sqrt(d_k) (the App. B rule for the
+    descriptor dimension), and a stored row's first d_k values are its key.
+    """
+    return np.concatenate([np.asarray(K, dtype=np.float64), np.asarray(V, dtype=np.float64)], axis=-1)
 
 
 def round_nearest_bf16(x: np.ndarray) -> np.ndarray:

@@ -702,6 +702,49 @@ def check_rope_rezero(O):
     assert np.array_equal(a, b)
 
 
+# --------------------------------------------------------------------------- App. E: [K; V] descriptor
+def check_kv_descriptor(O):
+    rng = np.random.default_rng(47)
+    H, d, N, M, steps = 2, 3, 6, 9, 4
+    prm = _prm(O, sigma=2.0)
+
+    def rollout(make):
+        bank = O.LayerBank.empty([M] * H, 2 * d)
+        out = []
+        for t in range(steps):
+            K = rng_k[t]
+            V = rng_v[t]
+            rec = O.update_layer(bank, make(K, V), V, t, prm)
+            out.append((rec.r_star, [sorted(zip(hb.step.tolist(), hb.src.tolist())) for hb in bank.heads],
+                        [np.sort(hb.rho) for hb in bank.heads]))
+        return bank, out
+
+    rng_k = [rng.normal(size=(H, N, d)) for _ in range(steps)]
+    rng_v = [rng.normal(size=(H, N, d)) for _ in range(steps)]
+    # the descriptor is the key followed by the value; stored rows keep both
+    D = O.kv_descriptor(rng_k[0], rng_v[0])
+    assert D.shape == (H, N, 2 * d) and np.array_equal(D[..., :d], rng_k[0]) and np.array_equal(D[..., d:], rng_v[0])
+    # distances are permutation-invariant over coordinates: [V; K] decides exactly as [K; V]
+    _, a = rollout(O.kv_descriptor)
+    _, b = rollout(lambda K, V: O.kv_descriptor(V, K))
+    for (ra, pa, qa), (rb, pb, qb) in zip(a, b):
+        assert ra == rb and pa == pb
+        assert all(np.allclose(x, y, rtol=1e-12, atol=0) for x, y in zip(qa, qb))
+    # with all values equal the descriptor geometry is that of the keys (same sigma)
+    bank_k = O.LayerBank.empty([M] * H, d)
+    bank_kv = O.LayerBank.empty([M] * H, 2 * d)
+    for t in range(steps):
+        V1 = np.ones((H, N, d))
+        rk = O.update_layer(bank_k, rng_k[t], V1, t, prm)
+        rkv = O.update_layer(bank_kv, O.kv_descriptor(rng_k[t], V1), V1, t, prm)
+        assert rk.r_star == rkv.r_star
+        for hk, hkv in zip(bank_k.heads, bank_kv.heads):
+            assert np.array_equal(hk.step, hkv.step) and np.array_equal(hk.src, hkv.src)
+            assert np.allclose(hk.rho, hkv.rho, rtol=1e-12) and np.array_equal(hk.K, hkv.K[:, :d])
+    # the descriptor default bandwidth is sqrt(2 d / 2) = sqrt(d) (App. B rule at dimension 2 d)
+    assert abs(O.Params().sigma_for(2 * 64) - 8.0) < 1e-15
+
+
 ALL_CHECKS = [
     check_kernel_closed_forms,
     check_distance_identities,
@@ -718,4 +761,5 @@ ALL_CHECKS = [
     check_sequential_admission,
     check_round_nearest_bf16,
     check_rope_rezero,
+    check_kv_descriptor,
 ]

@@ -81,6 +81,10 @@ MUTANTS = [
     ("rope_first_token_time", "a = t[:, None] * th[None, :]", "a = t[:1, None] * th[None, :]"),
     ("bf16_ties_up", "out = np.ldexp(np.rint(m * 256.0), e - 8)", "out = np.ldexp(np.floor(m * 256.0 + 0.5), e - 8)"),
     ("bf16_through_fp32", "m, e = np.frexp(x)", "m, e = np.frexp(x.astype(np.float32).astype(np.float64))"),
+    ("kv_keys_only", "    return np.concatenate([np.asarray(K, dtype=np.float64), np.asarray(V, dtype=np.float64)], axis=-1)",
+     "    return np.concatenate([np.asarray(K, dtype=np.float64), 0.0 * np.asarray(V, dtype=np.float64)], axis=-1)"),
+    ("kv_value_twice", "    return np.concatenate([np.asarray(K, dtype=np.float64), np.asarray(V, dtype=np.float64)], axis=-1)",
+     "    return np.concatenate([np.asarray(V, dtype=np.float64), np.asarray(V, dtype=np.float64)], axis=-1)"),
 ]
 
 
