@@ -83,6 +83,8 @@ def parse_args():
                     help="run attention and the update on one stream instead of overlapping them")
     ap.add_argument("--no-graphs", action="store_true",
                     help="launch every step directly instead of replaying a captured CUDA graph")
+    ap.add_argument("--descriptor", choices=["k", "kv"], default="k",
+                    help="retention descriptor: keys, or [K; V] (App. E ablation; fp32 score mode)")
     ap.add_argument("--rope", choices=["off", "interleaved", "half"], default="off",
                     help="blocks arrive rotated to their frames' temporal RoPE coordinates and admit "
                          "rotates them back to coordinate 0 (dkv_bank_admit_rope)")
@@ -92,6 +94,8 @@ def parse_args():
         args.no_graphs = args.no_overlap = args.no_e2e = True
         if args.rope != "off":
             ap.error("--rope applies to the batch admission path")
+    if args.descriptor == "kv" and args.score_mode != "fp32":
+        ap.error("--descriptor kv runs in the fp32 score mode (--score-mode fp32)")
     if args.rope != "off" and args.layers > 1:
         ap.error("--rope is measured on the single-layer step")
     return args
@@ -314,6 +318,8 @@ def run_ours(args):
                   eviction={"mandatory_densest": dkv.DKV_EVICT_MANDATORY_DENSEST, "densest": dkv.DKV_EVICT_DENSEST,
                             "mandatory_source": dkv.DKV_EVICT_MANDATORY_SOURCE}[args.eviction],
                   refresh_baselines=int(args.refresh_baselines))
+    if args.descriptor == "kv":   # [K; V] rows, sigma = sqrt(2d / 2)
+        policy.update(descriptor=dkv.DKV_DESC_KV, sigma=float(wl.d) ** 0.5)
     bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(layer), wl.N, bf, score_mode=mode, device=dev,
                          **policy)
     bank.reset()
@@ -619,7 +625,7 @@ def run_ours(args):
                        "policy": {"order": args.order, "eviction": args.eviction,
                                   "refresh_baselines": bool(args.refresh_baselines),
                                   "within_block": args.within_block,
-                                  "rope_rezero": args.rope},
+                                  "rope_rezero": args.rope, "descriptor": args.descriptor},
                        "streams": (("admit, then attention || evict" if P == 1 else "attention || admit + evict") + ", then commit")
                        if not args.no_overlap else "one stream",
                        "cuda_graphs": graphs is not None,

@@ -94,6 +94,13 @@ typedef enum {
   DKV_EVICT_MANDATORY_SOURCE = 2
 } dkv_evict_t;
 
+/* Retention descriptor (App. E "Retention geometry").  DKV_DESC_K: the post-RoPE key
+ * (Sec. 3, default).  DKV_DESC_KV: the concatenation [k; v] of key and value, so every
+ * interaction of Eqs. 2-12 uses ||k - k'||^2 + ||v - v'||^2 and, when sigma <= 0,
+ * sigma = sqrt(2d / 2) = sqrt(d) (App. B's rule for the descriptor dimension 2d).
+ * Attention still reads the keys and values as they are.                          */
+typedef enum { DKV_DESC_K = 0, DKV_DESC_KV = 1 } dkv_descriptor_t;
+
 /* Method parameters.  Defaults (dkv_params_default): tau = 2, sigma = sqrt(d/2),
  * p = 2, eps = 1, delta = 1e-6, shared cross-head prefix (Sec. 4.1; App. B
  * "Parameterization"; App. D "Default DensityKV configuration").           */
@@ -117,6 +124,9 @@ typedef struct {
                            layer_heads) of every [H][..] buffer): each layer has its own
                            shared prefix r* (Eq. 11) and prefix range, and one call
                            updates or reads all layers with single kernel launches      */
+  int32_t descriptor;   /* dkv_descriptor_t: the vectors whose geometry the density uses
+                           (Eqs. 2-3).  DKV_DESC_KV needs DKV_SCORE_FP32 and the
+                           workspace of dkv_bank_workspace_size_ex                      */
 } dkv_params_t;
 
 /* Caller-owned device buffers of the handle's H per-head banks (one layer, or
@@ -171,13 +181,21 @@ dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d);
 size_t dkv_bank_workspace_size(int32_t H, int32_t d, const int32_t* budgets,
                                int32_t n_max, int32_t dtype);
 
+/* As dkv_bank_workspace_size for a handle created with *params (host pointer; NULL:
+ * the defaults).  The [K; V] descriptor needs the values of the candidates in score
+ * order and of the survivors and evicted states as well: H (n_max + M_max + n_max) d
+ * elements more.  Returns 0 if the arguments are invalid.                        */
+size_t dkv_bank_workspace_size_ex(int32_t H, int32_t d, const int32_t* budgets,
+                                  int32_t n_max, int32_t dtype, const dkv_params_t* params);
+
 /* Creates a handle over caller-owned buffers (see dkv_buffers_t).  budgets is a
  * host array of H per-head budgets M_h >= 1.  Create writes the workspace
  * header once, synchronously (budgets, a cleared error word); it does not
  * touch the bank buffers, so the caller must zero `occupancy` (or call
  * dkv_bank_reset) before the first admit.  Limits: 1 <= H <= 4096,
  * d in {64, 128}, 1 <= M_h <= 262144, 1 <= n_max <= 16384.
- * DKV_SCORE_TENSOR requires dtype bf16 and d = 128.                          */
+ * DKV_SCORE_TENSOR requires dtype bf16 and d = 128; DKV_DESC_KV requires
+ * DKV_SCORE_FP32 (else DKV_ERR_UNSUPPORTED).                                  */
 dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_t* budgets,
                              int32_t n_max, int32_t dtype, const dkv_params_t* params,
                              const dkv_buffers_t* buffers);

@@ -99,7 +99,7 @@ void timer_end(Timer* t, cudaStream_t s) {
 // ------------------------------------------------------------------ workspace
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* base) {
+size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, char* base) {
   const size_t es = bf16 ? 2 : 4;
   const int hist_stride = ((n_max + 2) + 3) & ~3;
   const int snap_stride = n_max / SNAP + 2;
@@ -137,6 +137,11 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* ba
   w.bext = take(Hh * Mm * 64);
   w.ksurv_ext = take(Hh * Mm * 64);
   w.kevict_ext = take(Hh * Nm * 64);
+  if (kv) {
+    w.vperm = take(Hh * Nm * d * es);
+    w.vsurv = take(Hh * Mm * d * es);
+    w.vevict = take(Hh * Nm * d * es);
+  }
   const int sort_stride = (n_max + 255) / 256 * 256;
   w.sortbuf = (unsigned long long*)take(Hh * (size_t)sort_stride * 8);
   const int invb_stride = (M_max + 3) & ~3;   // 16-byte rows for the bulk copies
@@ -235,18 +240,26 @@ dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   out->eviction = DKV_EVICT_MANDATORY_DENSEST;
   out->refresh_baselines = 0;
   out->layer_heads = 0;
+  out->descriptor = DKV_DESC_K;
   return DKV_OK;
 }
 
-size_t dkv_bank_workspace_size(int32_t H, int32_t d, const int32_t* budgets, int32_t n_max, int32_t dtype) {
+size_t dkv_bank_workspace_size_ex(int32_t H, int32_t d, const int32_t* budgets, int32_t n_max, int32_t dtype,
+                                  const dkv_params_t* params) {
   if (H < 1 || H > kMaxH || (d != 64 && d != 128) || !budgets || n_max < 1 || n_max > kMaxN) return 0;
   if (dtype != DKV_DTYPE_BF16 && dtype != DKV_DTYPE_FP32) return 0;
+  const int kv = params ? params->descriptor : DKV_DESC_K;
+  if (kv != DKV_DESC_K && kv != DKV_DESC_KV) return 0;
   int M_max = 0;
   for (int h = 0; h < H; ++h) {
     if (budgets[h] < 1 || budgets[h] > kMaxM) return 0;
     M_max = budgets[h] > M_max ? budgets[h] : M_max;
   }
-  return ws_layout(H, d, M_max, n_max, dtype == DKV_DTYPE_BF16, nullptr, nullptr);
+  return ws_layout(H, d, M_max, n_max, dtype == DKV_DTYPE_BF16, kv, nullptr, nullptr);
+}
+
+size_t dkv_bank_workspace_size(int32_t H, int32_t d, const int32_t* budgets, int32_t n_max, int32_t dtype) {
+  return dkv_bank_workspace_size_ex(H, d, budgets, n_max, dtype, nullptr);
 }
 
 dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_t* budgets, int32_t n_max,
@@ -264,6 +277,7 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
       (p.eviction != DKV_EVICT_MANDATORY_DENSEST && p.eviction != DKV_EVICT_DENSEST &&
        p.eviction != DKV_EVICT_MANDATORY_SOURCE) ||
       (p.refresh_baselines != 0 && p.refresh_baselines != 1) ||
+      (p.descriptor != DKV_DESC_K && p.descriptor != DKV_DESC_KV) ||
       !std::isfinite(p.tau) || !std::isfinite(p.sigma) || !std::isfinite(p.eps) || !std::isfinite(p.delta))
     return DKV_ERR_ARG;
   int M_max = 0;
@@ -276,7 +290,8 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
     return DKV_ERR_ARG;
   if (!aligned(buf->k, 16) || !aligned(buf->v, 16) || !aligned(buf->workspace, 256)) return DKV_ERR_ARG;
   const int bf16 = dtype == DKV_DTYPE_BF16;
-  const size_t need = ws_layout(H, d, M_max, n_max, bf16, nullptr, nullptr);
+  const int kv = p.descriptor == DKV_DESC_KV;
+  const size_t need = ws_layout(H, d, M_max, n_max, bf16, kv, nullptr, nullptr);
   if (buf->workspace_bytes < need) return DKV_ERR_NOMEM;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return DKV_ERR_CUDA;
@@ -285,6 +300,7 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   if (prop.major != 10 || prop.minor != 3) return DKV_ERR_UNSUPPORTED;   // built for sm_103a only
   const bool want_tc = p.score_mode == DKV_SCORE_TENSOR;
   if (want_tc && !tc_supported(d, bf16)) return DKV_ERR_UNSUPPORTED;
+  if (want_tc && kv) return DKV_ERR_UNSUPPORTED;   // [K; V] geometry: fp32 score mode only
   std::call_once(g_smem_once, [] {
     cudaError_t e = simt_set_smem_limits();
     if (e == cudaSuccess) e = update_set_smem_limits();
@@ -297,14 +313,14 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   if (!bk) return DKV_ERR_ARG;
   bk->device = dev;
   bk->params = p;
-  if (!(bk->params.sigma > 0.0f)) bk->params.sigma = std::sqrt((float)d / 2.0f);
+  if (!(bk->params.sigma > 0.0f)) bk->params.sigma = std::sqrt((float)(kv ? 2 * d : d) / 2.0f);
   bk->budgets.assign(budgets, budgets + H);
   bk->tc = want_tc;
   Bank& b = bk->b;
   b.k = buf->k; b.v = buf->v; b.rho = buf->rho; b.base = buf->base; b.knorm = buf->knorm;
   b.prov_step = buf->prov_step; b.prov_src = buf->prov_src; b.occ = buf->occupancy;
   b.H = H; b.d = d; b.M_max = M_max; b.n_max = n_max; b.bf16 = bf16;
-  ws_layout(H, d, M_max, n_max, bf16, &bk->w, (char*)buf->workspace);
+  ws_layout(H, d, M_max, n_max, bf16, kv, &bk->w, (char*)buf->workspace);
   bk->w.layer_heads = p.layer_heads > 0 ? p.layer_heads : H;
   bk->n_layers = H / bk->w.layer_heads;
   const float sg = bk->params.sigma;
@@ -362,8 +378,8 @@ static dkv_status_t admit_impl(dkv_bank_t bank, const void* Kc, const void* Vc, 
   if (rope) Kc = w.kevict;   // the re-zeroed keys, same [H][N][d] layout
   if (e == cudaSuccess)
     if (bank->kp.order == DKV_ORDER_SCORE)   // source order needs no scores (App. E)
-      e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, N, bank->kp, s, t);
-  if (e == cudaSuccess) e = launch_sort(b, w, Kc, bank->kp.order == DKV_ORDER_SOURCE, s, t);
+      e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, bank->kp, s, t);
+  if (e == cudaSuccess) e = launch_sort(b, w, Kc, Vc, bank->kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_cross_tc(b, w, bank->kp, s, t) : launch_cross_fp32(b, w, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_rstar(b, w, bank->kp, s, t);
   if (e != cudaSuccess) return DKV_ERR_CUDA;
@@ -497,8 +513,8 @@ dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const v
   const KParams& kp = bank->kp;
   cudaError_t e = launch_cand_norms(b, w, Kc, N, step, kp, nullptr, s, t);
   if (e == cudaSuccess && kp.order == DKV_ORDER_SCORE)
-    e = bank->tc ? launch_score_tc(b, w, Kc, N, kp, s, t) : launch_score_fp32(b, w, Kc, N, kp, s, t);
-  if (e == cudaSuccess) e = launch_sort(b, w, Kc, kp.order == DKV_ORDER_SOURCE, s, t);
+    e = bank->tc ? launch_score_tc(b, w, Kc, N, kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, kp, s, t);
+  if (e == cudaSuccess) e = launch_sort(b, w, Kc, Vc, kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = launch_seq_gather(b, w, Kc, Vc, N, sc.kseq, sc.vseq, sc.srcseq, s);
   if (e != cudaSuccess) return DKV_ERR_CUDA;
   // one one-candidate update per position j: the j-th candidate of every head

@@ -53,6 +53,10 @@ struct Ws {
   void* bext;           // [H][M_max][32] bank (derived from the bank keys, kept in step)
   void* ksurv_ext;      // [H][M_max][32]
   void* kevict_ext;     // [H][n_max][32]
+  // values beside the key copies, [K; V] descriptor only (nullptr otherwise)
+  void* vperm;          // [H][n_max][d]  candidate values in pi order
+  void* vsurv;          // [H][M_max][d]  values of surviving states
+  void* vevict;         // [H][n_max][d]  values of evicted states
   unsigned long long* sortbuf;   // [H][sort_stride] sorted runs of 256 sort keys
   float* invb;          // [H][invb_stride] 1 / b of the bank states (derived from the
                         //   baselines, kept in step; 128 floats of padding at the end)
@@ -73,7 +77,7 @@ struct RopeArgs {
 __host__ __device__ inline DevLayer* layer_of(const Ws& w, int h) { return w.L + h / w.layer_heads; }
 
 // Computes the sub-buffer offsets of the workspace; returns the total bytes.
-size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, Ws* out, char* base);
+size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, char* base);
 
 // Kernel timing hook (dkv_api.cu): brackets a launch with events when enabled.
 struct Timer;
@@ -86,8 +90,11 @@ void timer_end(Timer* t, cudaStream_t s);
 // (rope != nullptr: the keys re-zeroed into w.kevict first, norms of the stored keys)
 cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
                               const RopeArgs* rope, cudaStream_t s, Timer* t);
-cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
-cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t);
+// (Vc: the candidates' values, read with the [K; V] descriptor)
+cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
+                              cudaStream_t s, Timer* t);
+cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int identity, cudaStream_t s,
+                        Timer* t);
 cudaError_t launch_cross_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_rstar(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // update back half (compress)

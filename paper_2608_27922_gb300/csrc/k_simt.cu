@@ -7,6 +7,9 @@
 // One thread owns one row and walks the columns in increasing order, so the
 // running sums of Eq. C.2 are formed in the same order by the crossing pass
 // and by the projection pass that later resumes them from a snapshot.
+// With the [K; V] descriptor (App. E "Retention geometry") two neighbouring threads
+// own a row, one its key and one its value; d2 = d2_key + d2_value after one shuffle,
+// identical in both, and the even thread writes.
 #include "dkv_internal.h"
 
 #include <climits>
@@ -25,6 +28,8 @@ struct PairJob {
   int64_t rk_hs;     // row-key head stride (elements)
   const void* ck;    // column keys of head 0
   int64_t ck_hs;     // column-key head stride (elements)
+  const void* rv;    // row values ([K; V] descriptor; same layout as rk)
+  const void* cv;    // column values (same layout as ck)
   Bank b;
   Ws w;
   KParams kp;
@@ -35,11 +40,13 @@ __device__ __forceinline__ const T* ptr(const void* p, int64_t off) {
   return reinterpret_cast<const T*>(p) + off;
 }
 
-template <typename T, int D, int MODE>
+template <typename T, int D, int MODE, bool KV>
 __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
+  constexpr int DC = KV ? 2 * D : D;   // staged floats per column: key (| value)
+  constexpr int RPB = KV ? ROWS / 2 : ROWS;   // rows per block
   extern __shared__ float smem[];
-  float* cs = smem;              // [CT][D] staged column keys
-  float* cmeta = smem + CT * D;  // [CT]    per-column factor (SCORE: 1 / b_j)
+  float* cs = smem;               // [CT][DC] staged column keys (| values)
+  float* cmeta = smem + CT * DC;  // [CT]     per-column factor (SCORE: 1 / b_j)
 
   const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
@@ -51,16 +58,18 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
   if (MODE == PM_PROJECT) { nrows = hd.empty ? 0 : hd.m_old;        c0 = (hd.r / SNAP) * SNAP; c1 = hd.r; }
   if (MODE == PM_SUB) { nrows = hd.empty ? 0 : hd.m_old - hd.e;     c1 = hd.e; }
   if (MODE == PM_NEWBASE) { nrows = hd.r;                           c1 = hd.m_new; }
-  const int row0 = blockIdx.x * ROWS;
+  const int row0 = blockIdx.x * RPB;
   if (row0 >= nrows) return;
-  const int row = row0 + threadIdx.x;
+  const int half = KV ? (threadIdx.x & 1) : 0;        // KV: 0 key, 1 value
+  const int row = row0 + (KV ? (threadIdx.x >> 1) : threadIdx.x);
   const bool active = row < nrows;
+  const bool writer = active && half == 0;
   const int64_t bh = (int64_t)h * j.b.M_max;   // bank head offset (rows)
 
-  // this thread's row key, in registers
+  // this thread's row key (or value), in registers
   float rr[D];
   {
-    const T* rp = ptr<T>(j.rk, (int64_t)h * j.rk_hs + (int64_t)(active ? row : 0) * D);
+    const T* rp = ptr<T>(half ? j.rv : j.rk, (int64_t)h * j.rk_hs + (int64_t)(active ? row : 0) * D);
 #pragma unroll
     for (int k = 0; k < D; ++k) rr[k] = active ? to_f<T>(rp[k]) : 0.f;
   }
@@ -75,7 +84,7 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
       thr = __fmul_rn(j.kp.tau, j.b.base[bh + row]);
       if (S >= thr) cross = 0;
       snap_row = j.w.snap + ((int64_t)h * j.b.M_max + row) * j.w.snap_stride;
-      snap_row[0] = S;
+      if (writer) snap_row[0] = S;
     } else if (MODE == PM_PROJECT) {
       S = j.w.snap[((int64_t)h * j.b.M_max + row) * j.w.snap_stride + c0 / SNAP];
     } else if (MODE == PM_SUB) {
@@ -90,18 +99,30 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
     const int nc = min(CT, c1 - t0);
     __syncthreads();
     const T* cp = ptr<T>(j.ck, (int64_t)h * j.ck_hs + (int64_t)t0 * D);
-    for (int e = threadIdx.x; e < nc * D; e += ROWS) cs[e] = to_f<T>(cp[e]);
+    if (KV) {
+      const T* cvp = ptr<T>(j.cv, (int64_t)h * j.ck_hs + (int64_t)t0 * D);
+      for (int e = threadIdx.x; e < nc * DC; e += ROWS) {
+        const int c = e / DC, k = e - c * DC;
+        cs[e] = to_f<T>(k < D ? cp[c * D + k] : cvp[c * D + k - D]);
+      }
+    } else {
+      for (int e = threadIdx.x; e < nc * D; e += ROWS) cs[e] = to_f<T>(cp[e]);
+    }
     if (MODE == PM_SCORE)
       for (int c = threadIdx.x; c < nc; c += ROWS) cmeta[c] = __frcp_rn(j.b.base[bh + t0 + c]);
     __syncthreads();
-    if (!active) continue;
+    if (!KV && !active) continue;   // KV: both threads of a row pair take part in the shuffle
     for (int c = 0; c < nc; ++c) {
-      const float* col = cs + c * D;
+      const float* col = cs + c * DC + half * D;
       float d2 = 0.f;
 #pragma unroll
       for (int k = 0; k < D; ++k) {
         float df = __fsub_rn(rr[k], col[k]);
         d2 = __fmaf_rn(df, df, d2);
+      }
+      if (KV) {
+        const float other = __shfl_xor_sync(0xffffffffu, d2, 1);
+        d2 = half ? __fadd_rn(other, d2) : __fadd_rn(d2, other);   // key part + value part
       }
       const float w = riesz_w(d2, j.kp);
       const int jc = t0 + c;
@@ -110,7 +131,7 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
       } else if (MODE == PM_CROSS) {
         S = __fadd_rn(S, w);
         if (cross == INT_MAX && S >= thr) cross = jc + 1;
-        if (((jc + 1) % SNAP) == 0) snap_row[(jc + 1) / SNAP] = S;
+        if (writer && ((jc + 1) % SNAP) == 0) snap_row[(jc + 1) / SNAP] = S;
       } else if (MODE == PM_PROJECT) {
         S = __fadd_rn(S, w);
       } else if (MODE == PM_SUB) {
@@ -120,7 +141,7 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
       }
     }
   }
-  if (!active) return;
+  if (!writer) return;
   if ((MODE == PM_SUB && (slot < 0 || slot >= hd.m_old)) || (MODE == PM_NEWBASE && (self < 0 || self >= hd.M))) {
     dev_fail(j.w.L, DEV_INCONSISTENT, 6000 + MODE);   // a list entry out of range: skip the write
     return;
@@ -149,22 +170,31 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
   }
 }
 
+template <int MODE, bool KV>
+void launch_pairs_t(dim3 grid, size_t sm, cudaStream_t s, const Bank& b, const PairJob& j) {
+  if (b.bf16) {
+    if (b.d == 128) simt_pairs<__nv_bfloat16, 128, MODE, KV><<<grid, ROWS, sm, s>>>(j);
+    else simt_pairs<__nv_bfloat16, 64, MODE, KV><<<grid, ROWS, sm, s>>>(j);
+  } else {
+    if (b.d == 128) simt_pairs<float, 128, MODE, KV><<<grid, ROWS, sm, s>>>(j);
+    else simt_pairs<float, 64, MODE, KV><<<grid, ROWS, sm, s>>>(j);
+  }
+}
+
+// rv / cv: the row and column values, non-null only with the [K; V] descriptor.
 template <int MODE>
 cudaError_t launch_pairs(const Bank& b, const Ws& w, const KParams& kp, const void* rk, int64_t rk_hs,
-                         const void* ck, int64_t ck_hs, int max_rows, cudaStream_t s, Timer* t,
-                         const char* name) {
-  PairJob j{rk, rk_hs, ck, ck_hs, b, w, kp};
-  dim3 grid((max_rows + ROWS - 1) / ROWS, b.H);
+                         const void* ck, int64_t ck_hs, const void* rv, const void* cv, int max_rows,
+                         cudaStream_t s, Timer* t, const char* name) {
+  const bool kv = rv != nullptr;
+  PairJob j{rk, rk_hs, ck, ck_hs, rv, cv, b, w, kp};
+  const int rpb = kv ? ROWS / 2 : ROWS;
+  dim3 grid((max_rows + rpb - 1) / rpb, b.H);
   if (grid.x == 0) return cudaSuccess;
-  const size_t sm = (size_t)(CT * b.d + CT) * sizeof(float);
+  const size_t sm = (size_t)(CT * b.d * (kv ? 2 : 1) + CT) * sizeof(float);
   timer_begin(t, name, s);
-  if (b.bf16) {
-    if (b.d == 128) simt_pairs<__nv_bfloat16, 128, MODE><<<grid, ROWS, sm, s>>>(j);
-    else simt_pairs<__nv_bfloat16, 64, MODE><<<grid, ROWS, sm, s>>>(j);
-  } else {
-    if (b.d == 128) simt_pairs<float, 128, MODE><<<grid, ROWS, sm, s>>>(j);
-    else simt_pairs<float, 64, MODE><<<grid, ROWS, sm, s>>>(j);
-  }
+  if (kv) launch_pairs_t<MODE, true>(grid, sm, s, b, j);
+  else launch_pairs_t<MODE, false>(grid, sm, s, b, j);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -239,31 +269,38 @@ __global__ void __launch_bounds__(AQ) simt_attend(const T* __restrict__ Q, int N
 
 }  // namespace
 
-cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp,
+// With the [K; V] descriptor every pass also reads the values beside its keys: the
+// candidates' (source order; pi order: vperm), the bank's, and the survivors' and evicted
+// states' copies (vsurv, vevict) taken by commit.
+cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
                               cudaStream_t s, Timer* t) {
   // rows: candidates in source order; columns: bank keys [0, m)
-  return launch_pairs<PM_SCORE>(b, w, kp, Kc, (int64_t)N * b.d, b.k, (int64_t)b.M_max * b.d, N, s, t,
-                                "score_fp32");
+  const bool kv = w.vperm != nullptr;
+  return launch_pairs<PM_SCORE>(b, w, kp, Kc, (int64_t)N * b.d, b.k, (int64_t)b.M_max * b.d, kv ? Vc : nullptr,
+                                kv ? b.v : nullptr, N, s, t, "score_fp32");
 }
 
 cudaError_t launch_cross_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
-  return launch_pairs<PM_CROSS>(b, w, kp, b.k, (int64_t)b.M_max * b.d, w.kperm, (int64_t)b.n_max * b.d, b.M_max,
-                                s, t, "cross_fp32");
+  const bool kv = w.vperm != nullptr;
+  return launch_pairs<PM_CROSS>(b, w, kp, b.k, (int64_t)b.M_max * b.d, w.kperm, (int64_t)b.n_max * b.d,
+                                kv ? b.v : nullptr, w.vperm, b.M_max, s, t, "cross_fp32");
 }
 
 cudaError_t launch_project_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
   return launch_pairs<PM_PROJECT>(b, w, kp, b.k, (int64_t)b.M_max * b.d, w.kperm, (int64_t)b.n_max * b.d,
-                                  b.M_max, s, t, "project_fp32");
+                                  kv ? b.v : nullptr, w.vperm, b.M_max, s, t, "project_fp32");
 }
 
 cudaError_t launch_subtract_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   return launch_pairs<PM_SUB>(b, w, kp, w.ksurv, (int64_t)b.M_max * b.d, w.kevict, (int64_t)b.n_max * b.d,
-                              b.M_max, s, t, "subtract_fp32");
+                              w.vsurv, w.vevict, b.M_max, s, t, "subtract_fp32");
 }
 
 cudaError_t launch_newbase_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
   return launch_pairs<PM_NEWBASE>(b, w, kp, w.kperm, (int64_t)b.n_max * b.d, b.k, (int64_t)b.M_max * b.d,
-                                  b.n_max, s, t, "newbase_fp32");
+                                  w.vperm, kv ? b.v : nullptr, b.n_max, s, t, "newbase_fp32");
 }
 
 cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void* Kw, const void* Vw, int W,

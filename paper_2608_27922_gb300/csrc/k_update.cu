@@ -500,8 +500,8 @@ __device__ __forceinline__ int run_rank(const unsigned long long* r, unsigned lo
 // distinct and cover [0, N)).  The block then copies its candidates' keys, norms and
 // extension rows to their positions (the operand of the prefix passes in pi order).
 // Source order (empty bank, or the source-order policy): position = source index.
-__global__ void __launch_bounds__(RUN) k_sort_rank(Bank bk, Ws w, const char* __restrict__ Kc, int esize,
-                                                   int identity) {
+__global__ void __launch_bounds__(RUN) k_sort_rank(Bank bk, Ws w, const char* __restrict__ Kc,
+                                                   const char* __restrict__ Vc, int esize, int identity) {
   extern __shared__ unsigned long long runs[];
   __shared__ int s_pos[RUN], s_src[RUN];
   const int h = blockIdx.y;
@@ -546,14 +546,19 @@ __global__ void __launch_bounds__(RUN) k_sort_rank(Bank bk, Ws w, const char* __
   }
   __syncthreads();
   const int rb = bk.d * esize;
-  const int kg = rb / 64;                         // key groups; then one extension group
-  for (int c = t; c < nvalid * (kg + 1); c += RUN) {
-    const int row = c / (kg + 1), grp = c - row * (kg + 1);
+  const int kg = rb / 64;                         // key groups, one extension group, then
+  const int vg = w.vperm ? kg : 0;                // value groups ([K; V] descriptor)
+  const int per_row = kg + 1 + vg;
+  for (int c = t; c < nvalid * per_row; c += RUN) {
+    const int row = c / per_row, grp = c - row * per_row;
     const int pos = s_pos[row], src = s_src[row];
     if (pos < 0 || src < 0 || src >= N) continue;   // reported above
     if (grp < kg) {
       copy64(reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb) + 4 * grp,
              reinterpret_cast<uint4*>((char*)w.kperm + (hn + pos) * rb) + 4 * grp);
+    } else if (grp > kg) {
+      copy64(reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg - 1),
+             reinterpret_cast<uint4*>((char*)w.vperm + (hn + pos) * rb) + 4 * (grp - kg - 1));
     } else {
       w.kperm_norm[hn + pos] = w.cnorm[hn + src];
       copy64(reinterpret_cast<const uint4*>((const char*)w.cext + (hn + src) * 64),
@@ -959,7 +964,8 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
   for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < total; c += gridDim.x * blockDim.x) {
     const int row = c / per_row, grp = c - row * per_row;
     if (row < ng) {
-      // surviving state: key and its derived rows to the workspace (no values)
+      // surviving state: key and its derived rows to the workspace (its value too with
+      // the [K; V] descriptor)
       const int slot = w.surv_list[bh + row];
       if (slot < 0 || slot >= hd.m_old) {
         if (grp == 0) dev_fail(w.L, DEV_INCONSISTENT, 7000 + h);
@@ -968,7 +974,11 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
       if (grp < kg) {
         copy64(reinterpret_cast<const uint4*>((const char*)b.k + (bh + slot) * rb) + 4 * grp,
                reinterpret_cast<uint4*>((char*)w.ksurv + (bh + row) * rb) + 4 * grp);
-      } else if (grp == 2 * kg) {
+      } else if (grp < 2 * kg) {
+        if (w.vsurv)   // [K; V] descriptor: the survivors' values too
+          copy64(reinterpret_cast<const uint4*>((const char*)b.v + (bh + slot) * rb) + 4 * (grp - kg),
+                 reinterpret_cast<uint4*>((char*)w.vsurv + (bh + row) * rb) + 4 * (grp - kg));
+      } else {
         w.ksurv_norm[bh + row] = b.knorm[bh + slot];
         copy64(reinterpret_cast<const uint4*>((const char*)w.bext + (bh + slot) * 64),
                reinterpret_cast<uint4*>((char*)w.ksurv_ext + (bh + row) * 64));
@@ -987,8 +997,9 @@ __global__ void k_commit(Bank b, Ws w, const char* __restrict__ Vc, int N, int e
       if (j < hd.e) copy64(dst, reinterpret_cast<uint4*>((char*)w.kevict + (hn + j) * rb) + 4 * grp);
       copy64(reinterpret_cast<const uint4*>((const char*)w.kperm + (hn + j) * rb) + 4 * grp, dst);
     } else if (grp < 2 * kg) {
-      copy64(reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg),
-             reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb) + 4 * (grp - kg));
+      uint4* dst = reinterpret_cast<uint4*>((char*)b.v + (bh + slot) * rb) + 4 * (grp - kg);
+      if (w.vevict && j < hd.e) copy64(dst, reinterpret_cast<uint4*>((char*)w.vevict + (hn + j) * rb) + 4 * (grp - kg));
+      copy64(reinterpret_cast<const uint4*>(Vc + ((int64_t)h * N + src) * rb) + 4 * (grp - kg), dst);
     } else {
       uint4* dx = reinterpret_cast<uint4*>((char*)w.bext + (bh + slot) * 64);
       if (j < hd.e) {
@@ -1070,13 +1081,14 @@ cudaError_t launch_inv_base(const Bank& b, const Ws& w, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, int identity, cudaStream_t s, Timer* t) {
+cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int identity, cudaStream_t s,
+                        Timer* t) {
   const int max_runs = (b.n_max + RUN - 1) / RUN;
   timer_begin(t, "sort_runs", s);
   k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max, identity);
   timer_end(t, s);
   timer_begin(t, "sort_rank", s);
-  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(b, w, (const char*)Kc,
+  k_sort_rank<<<dim3(max_runs, b.H), RUN, (size_t)max_runs * RUN * 8, s>>>(b, w, (const char*)Kc, (const char*)Vc,
                                                                            b.bf16 ? 2 : 4, identity);
   timer_end(t, s);
   return cudaGetLastError();

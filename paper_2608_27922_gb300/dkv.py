@@ -23,6 +23,7 @@ DKV_OK = 0
 DKV_DTYPE_BF16, DKV_DTYPE_FP32 = 0, 1
 DKV_SCORE_TENSOR, DKV_SCORE_FP32 = 0, 1
 DKV_ORDER_SCORE, DKV_ORDER_SOURCE = 0, 1
+DKV_DESC_K, DKV_DESC_KV = 0, 1
 DKV_EVICT_MANDATORY_DENSEST, DKV_EVICT_DENSEST, DKV_EVICT_MANDATORY_SOURCE = 0, 1, 2
 STATUS = {0: "DKV_OK", 1: "DKV_ERR_ARG", 2: "DKV_ERR_SHAPE", 3: "DKV_ERR_STATE", 4: "DKV_ERR_CUDA",
           5: "DKV_ERR_NOMEM", 6: "DKV_ERR_TIMEOUT", 7: "DKV_ERR_UNSUPPORTED", 8: "DKV_ERR_DEVICE"}
@@ -32,7 +33,8 @@ class dkv_params_t(ctypes.Structure):
     _fields_ = [("tau", ctypes.c_float), ("sigma", ctypes.c_float), ("p", ctypes.c_float),
                 ("eps", ctypes.c_float), ("delta", ctypes.c_float), ("sync_heads", ctypes.c_int32),
                 ("score_mode", ctypes.c_int32), ("order", ctypes.c_int32), ("eviction", ctypes.c_int32),
-                ("refresh_baselines", ctypes.c_int32), ("layer_heads", ctypes.c_int32)]
+                ("refresh_baselines", ctypes.c_int32), ("layer_heads", ctypes.c_int32),
+                ("descriptor", ctypes.c_int32)]
 
 
 class dkv_buffers_t(ctypes.Structure):
@@ -67,6 +69,8 @@ SIGNATURES = [
     ("dkv_version", _I, []),
     ("dkv_params_default", _I, [ctypes.POINTER(dkv_params_t), _I]),
     ("dkv_bank_workspace_size", ctypes.c_size_t, [_I, _I, ctypes.POINTER(ctypes.c_int32), _I, _I]),
+    ("dkv_bank_workspace_size_ex", ctypes.c_size_t, [_I, _I, ctypes.POINTER(ctypes.c_int32), _I, _I,
+                                                     ctypes.POINTER(dkv_params_t)]),
     ("dkv_bank_create", _I, [ctypes.POINTER(_P), _I, _I, ctypes.POINTER(ctypes.c_int32), _I, _I,
                              ctypes.POINTER(dkv_params_t), ctypes.POINTER(dkv_buffers_t)]),
     ("dkv_bank_destroy", None, [_P]),
@@ -155,8 +159,11 @@ def dkv_params_default(d: int) -> dkv_params_t:
     return p
 
 
-def dkv_bank_workspace_size(H: int, d: int, budgets: Sequence[int], n_max: int, dtype: int) -> int:
-    return int(lib().dkv_bank_workspace_size(H, d, _i32(budgets), n_max, dtype))
+def dkv_bank_workspace_size(H: int, d: int, budgets: Sequence[int], n_max: int, dtype: int,
+                            params: Optional[dkv_params_t] = None) -> int:
+    if params is None:
+        return int(lib().dkv_bank_workspace_size(H, d, _i32(budgets), n_max, dtype))
+    return int(lib().dkv_bank_workspace_size_ex(H, d, _i32(budgets), n_max, dtype, ctypes.byref(params)))
 
 
 def dkv_bank_create(H: int, d: int, budgets: Sequence[int], n_max: int, dtype: int, params: dkv_params_t,
@@ -328,7 +335,7 @@ class BankLayer:
         self.prov_step = torch.full((H, self.M_max), -1, dtype=torch.int64, device=dev)
         self.prov_src = torch.full((H, self.M_max), -1, dtype=torch.int32, device=dev)
         self.occupancy = torch.zeros(H, dtype=torch.int32, device=dev)
-        ws = dkv_bank_workspace_size(H, d, self.budgets, n_max, self.dtype_code)
+        ws = dkv_bank_workspace_size(H, d, self.budgets, n_max, self.dtype_code, p)
         if ws == 0:
             raise ValueError("invalid bank shape")
         self.workspace = torch.empty(ws, dtype=torch.uint8, device=dev)

@@ -41,7 +41,7 @@ def load_state(bank: dkv.BankLayer, ob: oracle.LayerBank) -> None:
     for h, hb in enumerate(ob.heads):
         m = hb.m
         if m:
-            bank.k[h, :m] = to_dev(hb.K, bank.dtype)
+            bank.k[h, :m] = to_dev(hb.K[:, :bank.d], bank.dtype)   # a [K; V] bank: its key part
             bank.v[h, :m] = to_dev(hb.V, bank.dtype)
             bank.rho[h, :m] = torch.from_numpy(hb.rho.astype(np.float32)).cuda()
             bank.base[h, :m] = torch.from_numpy(hb.base.astype(np.float32)).cuda()
@@ -130,6 +130,8 @@ def update_and_compare(bank: dkv.BankLayer, ob: oracle.LayerBank, K: np.ndarray,
         K = oracle.rope_rezero(K, t_coord, theta, layout, "bf16" if bank.dtype == torch.bfloat16 else "fp32")
     else:
         bank.admit(Kd, Vd, step)
+    if bank.params.descriptor == dkv.DKV_DESC_KV:   # the oracle bank holds [K; V] rows (App. E)
+        K = oracle.kv_descriptor(K, V)
     bank.compress()
     bank.sync()
     rec = oracle.update_layer(ob, K, V, step, prm)
@@ -213,7 +215,7 @@ def update_and_compare(bank: dkv.BankLayer, ob: oracle.LayerBank, K: np.ndarray,
         for key in set(g) & set(o):
             kg, vg, rg, bg, kn, _ = g[key]
             ko, vo, ro, bo = o[key]
-            if not (np.array_equal(kg, ko.astype(np.float32)) and np.array_equal(vg, vo.astype(np.float32))):
+            if not (np.array_equal(kg, ko[:kg.shape[0]].astype(np.float32)) and np.array_equal(vg, vo.astype(np.float32))):
                 rep.kv_bit_exact = False
             rep.rho_max_rel = max(rep.rho_max_rel, abs(rg - ro) / max(abs(ro), 1e-30))
             rep.base_max_rel = max(rep.base_max_rel, abs(bg - bo) / max(abs(bo), 1e-30))

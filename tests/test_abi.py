@@ -62,10 +62,11 @@ def test_struct_layouts_match_c():
 #include <stddef.h>
 #include "dkv.h"
 int main(void) {
-  printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t),
+  printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(dkv_params_t), sizeof(dkv_buffers_t),
          sizeof(dkv_layer_stats_t), sizeof(dkv_head_stats_t), sizeof(dkv_intermediates_t),
          offsetof(dkv_buffers_t, workspace_bytes), offsetof(dkv_params_t, order), offsetof(dkv_params_t, eviction),
-         offsetof(dkv_params_t, refresh_baselines), offsetof(dkv_params_t, layer_heads));
+         offsetof(dkv_params_t, refresh_baselines), offsetof(dkv_params_t, layer_heads),
+         offsetof(dkv_params_t, descriptor));
   return 0;
 }
 """
@@ -84,7 +85,8 @@ int main(void) {
                      ctypes.sizeof(dkv.dkv_layer_stats_t), ctypes.sizeof(dkv.dkv_head_stats_t),
                      ctypes.sizeof(dkv.dkv_intermediates_t), dkv.dkv_buffers_t.workspace_bytes.offset,
                      dkv.dkv_params_t.order.offset, dkv.dkv_params_t.eviction.offset,
-                     dkv.dkv_params_t.refresh_baselines.offset, dkv.dkv_params_t.layer_heads.offset]
+                     dkv.dkv_params_t.refresh_baselines.offset, dkv.dkv_params_t.layer_heads.offset,
+                     dkv.dkv_params_t.descriptor.offset]
 
 
 def test_host_only_entry_points():
@@ -102,6 +104,15 @@ def test_host_only_entry_points():
     assert dkv.dkv_bank_workspace_size(12, 96, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16) == 0
     assert dkv.dkv_bank_workspace_size(2, 64, [0, 5], 16, dkv.DKV_DTYPE_FP32) == 0
     assert dkv.dkv_bank_workspace_size(2, 64, [5, 5], 1 << 20, dkv.DKV_DTYPE_FP32) == 0
+    # the [K; V] descriptor adds the value copies: H (n_max + M_max + n_max) d elements
+    p = dkv.dkv_params_default(128)
+    base = dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16, p)
+    assert base == dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16)
+    p.descriptor = dkv.DKV_DESC_KV
+    kv = dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16, p)
+    assert 0 <= kv - base - 12 * (4680 + 9360 + 4680) * 128 * 2 < 3 * 256
+    p.descriptor = 2
+    assert dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680, dkv.DKV_DTYPE_BF16, p) == 0
     # argument errors are reported before any CUDA call
     h = ctypes.c_void_p()
     assert L.dkv_bank_create(ctypes.byref(h), 2, 64, None, 16, 1, None, None) == 1
