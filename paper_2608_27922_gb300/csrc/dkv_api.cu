@@ -225,7 +225,7 @@ const char* dkv_status_str(dkv_status_t s) {
   return "unknown status";
 }
 
-int32_t dkv_version(void) { return 120; }
+int32_t dkv_version(void) { return 200; }   // 0.2.0: dkv_params_t.descriptor, admit_rope
 
 dkv_status_t dkv_params_default(dkv_params_t* out, int32_t d) {
   if (!out || d <= 0) return DKV_ERR_ARG;
