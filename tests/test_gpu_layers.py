@@ -86,6 +86,43 @@ def test_grouped_layers_match_one_handle_per_layer(dkv, mode, sync):
         bk.close()
 
 
+def test_grouped_layers_rope(dkv):
+    """Temporal re-zeroing (dkv_bank_admit_rope) in a three-layer handle: one coordinate
+    array for all layers' heads, bit-identical to one handle per layer."""
+    L, H = 3, 2
+    wl = synth.get_workload("wan13b_layer_h12", L=L, H=H, N=96, W=96, Nq=64, budgets=[300, 190, 420] * 2, steps=6)
+    dt = torch.bfloat16
+    sep = [dkv.BankLayer(H, wl.d, wl.budgets_of_layer(l), wl.N, dt) for l in range(L)]
+    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, dt, layer_heads=H)
+    for b in sep + [grp]:
+        b.reset()
+    theta = torch.from_numpy(synth.temporal_rope_theta(wl.d)).cuda()
+    ro = [synth.LayerRollout(wl, l) for l in range(L)]
+    for t in range(wl.steps):
+        b = wl.admitted_block(t)
+        if b is None:
+            continue
+        tc = torch.from_numpy(wl.frame_coords(b) + 500).cuda()
+        blocks = [ro[l].block(b) for l in range(L)]
+        for l in range(L):
+            sep[l].update(to_dev(blocks[l][0], dt), to_dev(blocks[l][1], dt), b, t_coord=tc, theta=theta)
+        grp.update(_cat_heads([x[0] for x in blocks], dt), _cat_heads([x[1] for x in blocks], dt), b,
+                   t_coord=tc, theta=theta)
+        torch.cuda.synchronize()
+        for bk in sep + [grp]:
+            bk.sync()
+        for name in BUFFERS:
+            g = getattr(grp, name)
+            for l in range(L):
+                want = getattr(sep[l], name)
+                got = g[l * H:(l + 1) * H]
+                if want.dim() > 1:
+                    got = got[:, :want.shape[1]]
+                assert torch.equal(want, got), (t, name, l)
+    for bk in sep + [grp]:
+        bk.close()
+
+
 def test_layer_heads_must_divide_heads(dkv):
     wl = synth.get_workload("wan13b_layer_h12", H=6, N=16, budgets=32)
     for bad in (4, 7, -1):
