@@ -65,7 +65,7 @@ typedef enum {
   DKV_ERR_SHAPE = 2,        /* size outside what the handle / library supports           */
   DKV_ERR_STATE = 3,        /* call out of order (admit twice, compress without admit)   */
   DKV_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed                      */
-  DKV_ERR_NOMEM = 5,        /* workspace smaller than dkv_bank_workspace_size()          */
+  DKV_ERR_NOMEM = 5,        /* workspace smaller than dkv_bank_workspace_size_ex()       */
   DKV_ERR_TIMEOUT = 6,      /* a bounded device-side wait gave up (sticky, see sync)     */
   DKV_ERR_UNSUPPORTED = 7,  /* feature not available for this dtype / d / device         */
   DKV_ERR_DEVICE = 8        /* device-side consistency check failed (sticky, see sync)   */
@@ -143,8 +143,10 @@ typedef struct {
   int64_t* prov_step;   /* device [H][M_max] update step that admitted the state    */
   int32_t* prov_src;    /* device [H][M_max] source index within its block          */
   int32_t* occupancy;   /* device [H] number of retained states per head            */
-  void* workspace;      /* device scratch, >= dkv_bank_workspace_size() bytes,
-                           256-byte aligned; contents are private to the handle    */
+  void* workspace;      /* device scratch, >= dkv_bank_workspace_size_ex() bytes for
+                           the handle's parameters (= dkv_bank_workspace_size() with
+                           the key descriptor), 256-byte aligned; contents are
+                           private to the handle                                    */
   size_t workspace_bytes;
 } dkv_buffers_t;
 
