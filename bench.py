@@ -85,7 +85,7 @@ def parse_args():
     ap.add_argument("--no-graphs", action="store_true",
                     help="launch every step directly instead of replaying a captured CUDA graph")
     ap.add_argument("--descriptor", choices=["k", "kv"], default="k",
-                    help="retention descriptor: keys, or [K; V] (App. E ablation; fp32 score mode)")
+                    help="retention descriptor: keys, or [K; V] (App. E ablation)")
     ap.add_argument("--rope", choices=["off", "interleaved", "half"], default="off",
                     help="blocks arrive rotated to their frames' temporal RoPE coordinates and admit "
                          "rotates them back to coordinate 0 (dkv_bank_admit_rope)")
@@ -95,8 +95,6 @@ def parse_args():
         args.no_graphs = args.no_overlap = args.no_e2e = True
         if args.rope != "off":
             ap.error("--rope applies to the batch admission path")
-    if args.descriptor == "kv" and args.score_mode != "fp32":
-        ap.error("--descriptor kv runs in the fp32 score mode (--score-mode fp32)")
     if args.rope != "off" and args.layers > 1:
         ap.error("--rope is measured on the single-layer step")
     return args

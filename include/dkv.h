@@ -125,8 +125,8 @@ typedef struct {
                            shared prefix r* (Eq. 11) and prefix range, and one call
                            updates or reads all layers with single kernel launches      */
   int32_t descriptor;   /* dkv_descriptor_t: the vectors whose geometry the density uses
-                           (Eqs. 2-3).  DKV_DESC_KV needs DKV_SCORE_FP32 and the
-                           workspace of dkv_bank_workspace_size_ex                      */
+                           (Eqs. 2-3).  DKV_DESC_KV needs the workspace of
+                           dkv_bank_workspace_size_ex; knorm then holds ||k||^2 + ||v||^2 */
 } dkv_params_t;
 
 /* Caller-owned device buffers of the handle's H per-head banks (one layer, or
@@ -196,8 +196,7 @@ size_t dkv_bank_workspace_size_ex(int32_t H, int32_t d, const int32_t* budgets,
  * touch the bank buffers, so the caller must zero `occupancy` (or call
  * dkv_bank_reset) before the first admit.  Limits: 1 <= H <= 4096,
  * d in {64, 128}, 1 <= M_h <= 262144, 1 <= n_max <= 16384.
- * DKV_SCORE_TENSOR requires dtype bf16 and d = 128; DKV_DESC_KV requires
- * DKV_SCORE_FP32 (else DKV_ERR_UNSUPPORTED).                                  */
+ * DKV_SCORE_TENSOR requires dtype bf16 and d = 128.                          */
 dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_t* budgets,
                              int32_t n_max, int32_t dtype, const dkv_params_t* params,
                              const dkv_buffers_t* buffers);

@@ -300,7 +300,6 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   if (prop.major != 10 || prop.minor != 3) return DKV_ERR_UNSUPPORTED;   // built for sm_103a only
   const bool want_tc = p.score_mode == DKV_SCORE_TENSOR;
   if (want_tc && !tc_supported(d, bf16)) return DKV_ERR_UNSUPPORTED;
-  if (want_tc && kv) return DKV_ERR_UNSUPPORTED;   // [K; V] geometry: fp32 score mode only
   std::call_once(g_smem_once, [] {
     cudaError_t e = simt_set_smem_limits();
     if (e == cudaSuccess) e = update_set_smem_limits();
@@ -374,11 +373,11 @@ static dkv_status_t admit_impl(dkv_bank_t bank, const void* Kc, const void* Vc, 
   const Ws& w = bank->w;
   Timer* t = &bank->timer;
   bank->last = s;
-  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, bank->kp, rope, s, t);
+  cudaError_t e = launch_cand_norms(b, w, Kc, Vc, N, step, bank->kp, rope, s, t);
   if (rope) Kc = w.kevict;   // the re-zeroed keys, same [H][N][d] layout
   if (e == cudaSuccess)
     if (bank->kp.order == DKV_ORDER_SCORE)   // source order needs no scores (App. E)
-      e = bank->tc ? launch_score_tc(b, w, Kc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, bank->kp, s, t);
+      e = bank->tc ? launch_score_tc(b, w, Kc, Vc, N, bank->kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_sort(b, w, Kc, Vc, bank->kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = bank->tc ? launch_cross_tc(b, w, bank->kp, s, t) : launch_cross_fp32(b, w, bank->kp, s, t);
   if (e == cudaSuccess) e = launch_rstar(b, w, bank->kp, s, t);
@@ -511,9 +510,9 @@ dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const v
   const Ws& w = bank->w;
   Timer* t = &bank->timer;
   const KParams& kp = bank->kp;
-  cudaError_t e = launch_cand_norms(b, w, Kc, N, step, kp, nullptr, s, t);
+  cudaError_t e = launch_cand_norms(b, w, Kc, Vc, N, step, kp, nullptr, s, t);
   if (e == cudaSuccess && kp.order == DKV_ORDER_SCORE)
-    e = bank->tc ? launch_score_tc(b, w, Kc, N, kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, kp, s, t);
+    e = bank->tc ? launch_score_tc(b, w, Kc, Vc, N, kp, s, t) : launch_score_fp32(b, w, Kc, Vc, N, kp, s, t);
   if (e == cudaSuccess) e = launch_sort(b, w, Kc, Vc, kp.order == DKV_ORDER_SOURCE, s, t);
   if (e == cudaSuccess) e = launch_seq_gather(b, w, Kc, Vc, N, sc.kseq, sc.vseq, sc.srcseq, s);
   if (e != cudaSuccess) return DKV_ERR_CUDA;

@@ -87,9 +87,10 @@ void timer_end(Timer* t, cudaStream_t s);
 // ---- launches (each returns cudaGetLastError() of its launch) ----
 // update front half (admit)
 // candidates' norms and extension rows, zeroed crossing histogram, update snapshot
-// (rope != nullptr: the keys re-zeroed into w.kevict first, norms of the stored keys)
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
-                              const RopeArgs* rope, cudaStream_t s, Timer* t);
+// (rope != nullptr: the keys re-zeroed into w.kevict first, norms of the stored keys;
+// [K; V] descriptor: the norms and extension rows are those of [k; v], Vc read too)
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, int64_t step,
+                              const KParams& kp, const RopeArgs* rope, cudaStream_t s, Timer* t);
 // (Vc: the candidates' values, read with the [K; V] descriptor)
 cudaError_t launch_score_fp32(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
                               cudaStream_t s, Timer* t);
@@ -108,7 +109,8 @@ cudaError_t launch_seq_gather(const Bank& b, const Ws& w, const void* Kc, const 
 cudaError_t launch_subtract_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_newbase_fp32(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 // tensor-core (tcgen05) versions of the pair passes, bf16 and d = 128 only
-cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s, Timer* t);
+cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
+                            cudaStream_t s, Timer* t);
 cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t);

@@ -50,27 +50,37 @@ enum TMode { TM_SCORE = 0, TM_CROSS = 1, TM_PROJECT = 2, TM_SUB = 3, TM_NEWBASE 
 
 constexpr int BM = 128;                     // rows per CTA (TMEM lanes)
 constexpr int BN = 128;                     // columns per tile
-constexpr int TILE_BYTES = BM * 128 * 2;    // 128 rows x 128 bf16
-constexpr int HALF_BYTES = TILE_BYTES / 2;  // one 64-column 128-byte-swizzle panel
+constexpr int HALF_BYTES = BM * 64 * 2;    // one 64-column 128-byte-swizzle panel (16 KiB)
 constexpr int EXT_BYTES = BM * 16 * 2;      // 128 rows x 16 bf16 (32-byte swizzle)
 constexpr int STAGES = 2;
 constexpr int EPI_WARPS = 8;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 256;         // two 128-column accumulators
-constexpr int OFF_A = 0;
-constexpr int OFF_AX = TILE_BYTES;
-constexpr int OFF_B = OFF_AX + EXT_BYTES;                 // [STAGES] tiles
-constexpr int OFF_BX = OFF_B + STAGES * TILE_BYTES;       // [STAGES] extension tiles
 // score weights of tiles t .. t+4: buffer t % 5 is refilled for tile t + 5 once the MMA
 // of tile t + 3 has completed, which needs every epilogue warp's release of tile t + 1,
 // given only after that warp finished tile t (the release can precede a tile's arithmetic)
 constexpr int META_BUFS = 5;
-constexpr int OFF_META = OFF_BX + STAGES * EXT_BYTES;     // float [META_BUFS][BN]
-constexpr int OFF_XCH = OFF_META + META_BUFS * BN * 4;    // float [2][2][BM]
-constexpr int OFF_FLAG = OFF_XCH + 2 * 2 * BM * 4;      // int: last-arrival flag of split tiles
-constexpr int OFF_BAR = OFF_FLAG + 16;
-constexpr size_t SMEM_BYTES = OFF_BAR + 128;              // base 1024-aligned (checked)
-constexpr uint32_t LOAD_BYTES = TILE_BYTES + EXT_BYTES;
+
+// Shared-memory layout.  A tile row is the state's descriptor: its key (two 64-column
+// panels) or, with the [K; V] descriptor (App. E), its key and value (four panels); one
+// CTA per SM then (209 KiB), two otherwise (2 x 110 KiB).
+template <bool KV>
+struct Lay {
+  static constexpr int NP = KV ? 4 : 2;                        // 64-column panels per row
+  static constexpr int TILE = NP * HALF_BYTES;
+  static constexpr int A = 0;
+  static constexpr int AX = TILE;
+  static constexpr int B = AX + EXT_BYTES;                     // [STAGES] tiles
+  static constexpr int BX = B + STAGES * TILE;                 // [STAGES] extension tiles
+  static constexpr int META = BX + STAGES * EXT_BYTES;         // float [META_BUFS][BN]
+  static constexpr int XCH = META + META_BUFS * BN * 4;        // float [2][2][BM]
+  static constexpr int FLAG = XCH + 2 * 2 * BM * 4;            // int: last-arrival flag of split tiles
+  static constexpr int BAR = FLAG + 16;
+  static constexpr size_t SMEM = BAR + 128;                    // base 1024-aligned (checked)
+  static constexpr uint32_t LOAD = TILE + EXT_BYTES;
+  static_assert(B % 1024 == 0 && TILE % 1024 == 0, "128-byte-swizzled panels need 1024-byte alignment");
+  static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+};
 
 struct TcJob {
   Bank b;
@@ -178,19 +188,21 @@ __device__ __forceinline__ float chunk_sum_skip(const float (&v)[32], int lim, i
   return s;
 }
 
-template <int MODE, int P>
-__global__ void __launch_bounds__(THREADS, 2)
+template <int MODE, int P, bool KV>
+__global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
     tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
-             const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx, TcJob j) {
+             const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx,
+             const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j) {
+  using LY = Lay<KV>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if ((smem_u32(smem_raw) & 1023u) != 0u) {   // 128-byte-swizzled tiles need 1024-byte alignment
     if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9900);
     return;
   }
   uint8_t* smem = smem_raw;
-  float* meta = reinterpret_cast<float*>(smem + OFF_META);
-  float* xch = reinterpret_cast<float*>(smem + OFF_XCH);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  float* meta = reinterpret_cast<float*>(smem + LY::META);
+  float* xch = reinterpret_cast<float*>(smem + LY::XCH);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + LY::BAR);
   uint64_t* bar_a = bars + 0;
   // ready[b]: column tile t (b = t & 1) has landed AND the epilogue has released
   // accumulator b (tile t - 2): the MMA issuer's only wait per tile
@@ -238,22 +250,25 @@ __global__ void __launch_bounds__(THREADS, 2)
     if (lane == 0 && ntiles > 0) {
       // ---------------- TMA producer: row tile (+ row-form extension) once, column tiles
       prefetch_map(&tmA); prefetch_map(&tmAx); prefetch_map(&tmB); prefetch_map(&tmBx);
-      mbar_arrive_expect_tx(bar_a, LOAD_BYTES);
-      tma_load_3d(smem + OFF_A, &tmA, bar_a, 0, row0, h);
-      tma_load_3d(smem + OFF_A + HALF_BYTES, &tmA, bar_a, 64, row0, h);
-      tma_load_3d(smem + OFF_AX, &tmAx, bar_a, 0, row0, h);
+      if (KV) { prefetch_map(&tmAv); prefetch_map(&tmBv); }
+      mbar_arrive_expect_tx(bar_a, LY::LOAD);
+#pragma unroll
+      for (int pn = 0; pn < LY::NP; ++pn)   // key panels, then value panels ([K; V])
+        tma_load_3d(smem + LY::A + pn * HALF_BYTES, pn < 2 ? &tmA : &tmAv, bar_a, (pn & 1) * 64, row0, h);
+      tma_load_3d(smem + LY::AX, &tmAx, bar_a, 0, row0, h);
       int issued = 0;
       for (int t = 0; t < ntiles; ++t) {
         const int s = t % STAGES;   // == t & 1, the accumulator of tile t
         // MMA(t - 2) complete: stage s is free, and (it waited for ready) the epilogue of
         // tile t - 4 has finished with meta buffer t % 4
         if (!mbar_wait(bar_empty + s, ((t / STAGES) & 1) ^ 1, abort_flag)) break;
-        mbar_arrive_expect_tx(bar_rdy + s, LOAD_BYTES);
+        mbar_arrive_expect_tx(bar_rdy + s, LY::LOAD);
         const int col = c0 + t * BN;
-        uint8_t* dst = smem + OFF_B + s * TILE_BYTES;
-        tma_load_3d(dst, &tmB, bar_rdy + s, 0, col, h);
-        tma_load_3d(dst + HALF_BYTES, &tmB, bar_rdy + s, 64, col, h);
-        tma_load_3d(smem + OFF_BX + s * EXT_BYTES, &tmBx, bar_rdy + s, 16, col, h);
+        uint8_t* dst = smem + LY::B + s * LY::TILE;
+#pragma unroll
+        for (int pn = 0; pn < LY::NP; ++pn)
+          tma_load_3d(dst + pn * HALF_BYTES, pn < 2 ? &tmB : &tmBv, bar_rdy + s, (pn & 1) * 64, col, h);
+        tma_load_3d(smem + LY::BX + s * EXT_BYTES, &tmBx, bar_rdy + s, 16, col, h);
         if (MODE == TM_SCORE) {
           // 1 / b_j of the tile's columns (a whole 128-float row; values past the last
           // column are not used)
@@ -286,11 +301,11 @@ __global__ void __launch_bounds__(THREADS, 2)
     }
   } else if (warp == 1) {
     if (lane == 0 && ntiles > 0) {
-      // ---------------- MMA issuer: 8 k-steps of the keys + 1 of the extension
+      // ---------------- MMA issuer: 8 k-steps per key (16 per [key; value]) + 1 of the extension
       constexpr uint32_t idesc = idesc_bf16(BM, BN);
       bool ok = mbar_wait(bar_a, 0, abort_flag);
-      const uint32_t a_base = smem_u32(smem + OFF_A);
-      const uint32_t ax_base = smem_u32(smem + OFF_AX);
+      const uint32_t a_base = smem_u32(smem + LY::A);
+      const uint32_t ax_base = smem_u32(smem + LY::AX);
       int done = 0;
       for (int t = 0; ok && t < ntiles; ++t) {
         const int s = t % STAGES;
@@ -298,10 +313,10 @@ __global__ void __launch_bounds__(THREADS, 2)
         // one wait per tile: every other wait in this thread stalls the tensor pipe
         if (!(ok = mbar_wait(bar_rdy + b, (t >> 1) & 1, abort_flag))) break;
         fence_after_sync();
-        const uint32_t b_base = smem_u32(smem + OFF_B + s * TILE_BYTES);
-        const uint32_t bx_base = smem_u32(smem + OFF_BX + s * EXT_BYTES);
+        const uint32_t b_base = smem_u32(smem + LY::B + s * LY::TILE);
+        const uint32_t bx_base = smem_u32(smem + LY::BX + s * EXT_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
+        for (int kk = 0; kk < 4 * LY::NP; ++kk) {
           const uint32_t koff = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
           mma_bf16(tmem + b * BN, desc_sw128(a_base + koff), desc_sw128(b_base + koff), idesc, kk > 0);
         }
@@ -477,7 +492,7 @@ __global__ void __launch_bounds__(THREADS, 2)
         if (half == 0 && active) part[blockIdx.z * zstride + row] = acc;
         __threadfence();
         named_bar(6, 32 * EPI_WARPS);
-        int* flag = reinterpret_cast<int*>(smem + OFF_FLAG);
+        int* flag = reinterpret_cast<int*>(smem + LY::FLAG);
         if (et == 0) {
           int32_t* cnt = j.w.cnt + (int64_t)h * j.w.cnt_stride + blockIdx.x;
           const int prev = atomicAdd(cnt, 1);
@@ -597,24 +612,35 @@ namespace {
 
 template <int MODE, int P>
 void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap& ax, const CUtensorMap& b,
-              const CUtensorMap& bx, const TcJob& job) {
-  tc_pairs<MODE, P><<<grid, THREADS, SMEM_BYTES, s>>>(a, ax, b, bx, job);
+              const CUtensorMap& bx, const CUtensorMap& av, const CUtensorMap& bv, bool kv, const TcJob& job) {
+  if (kv) tc_pairs<MODE, P, true><<<grid, THREADS, Lay<true>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
+  else tc_pairs<MODE, P, false><<<grid, THREADS, Lay<false>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
 }
 
+// rv / cv: the row and column values (same layouts as rk / ck), non-null only with the
+// [K; V] descriptor; the extension rows rx / cx then carry the descriptors' norms.
 template <int MODE>
 cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void* rk, const void* rx, int64_t rk_rows,
                       const void* ck, const void* cx, int64_t ck_rows, int max_rows, cudaStream_t s, Timer* t,
-                      const char* name, int split = 1) {
-  CUtensorMap ma, max_, mb, mbx;
+                      const char* name, int split = 1, const void* rv = nullptr, const void* cv = nullptr) {
+  const bool kv = rv != nullptr;
+  CUtensorMap ma, max_, mb, mbx, mav, mbv;
   if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_ext(&max_, rx, rk_rows, b.H, BM) ||
       !make_map_rows(&mb, ck, ck_rows, b.H, BN) || !make_map_ext(&mbx, cx, ck_rows, b.H, BN))
     return cudaErrorInvalidValue;
+  if (kv) {
+    if (!cv || !make_map_rows(&mav, rv, rk_rows, b.H, BM) || !make_map_rows(&mbv, cv, ck_rows, b.H, BN))
+      return cudaErrorInvalidValue;
+  } else {
+    mav = ma;   // never read
+    mbv = mb;
+  }
   TcJob job{b, w, kp};
   dim3 grid((max_rows + BM - 1) / BM, b.H, split);
   timer_begin(t, name, s);
-  if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, job);
-  else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, job);
-  else launch_p<MODE, 2>(grid, s, ma, max_, mb, mbx, job);
+  if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
+  else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
+  else launch_p<MODE, 2>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -627,46 +653,53 @@ cudaError_t tc_attn_set_smem_limits();
 
 cudaError_t tc_set_smem_limits() {
   cudaError_t e = cudaSuccess;
+#define DKV_OPT1(M, P, KV)                                                                                     \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_pairs<M, P, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Lay<KV>::SMEM);
 #define DKV_OPT(M)                                                                                             \
-  if (e == cudaSuccess)                                                                                        \
-    e = cudaFuncSetAttribute(tc_pairs<M, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);    \
-  if (e == cudaSuccess)                                                                                        \
-    e = cudaFuncSetAttribute(tc_pairs<M, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);    \
-  if (e == cudaSuccess)                                                                                        \
-    e = cudaFuncSetAttribute(tc_pairs<M, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  DKV_OPT1(M, 1, false) DKV_OPT1(M, 2, false) DKV_OPT1(M, 4, false)                                            \
+  DKV_OPT1(M, 1, true) DKV_OPT1(M, 2, true) DKV_OPT1(M, 4, true)
   DKV_OPT(TM_SCORE)
   DKV_OPT(TM_CROSS)
   DKV_OPT(TM_PROJECT)
   DKV_OPT(TM_SUB)
   DKV_OPT(TM_NEWBASE)
 #undef DKV_OPT
+#undef DKV_OPT1
   if (e == cudaSuccess) e = tc_attn_set_smem_limits();
   return e;
 }
 
-cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, int N, const KParams& kp, cudaStream_t s,
-                            Timer* t) {
-  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", 2);
+// With the [K; V] descriptor every pass also reads the values beside its keys (same
+// sources as the fp32 passes: the candidates' values, vperm, the bank's, vsurv, vevict).
+cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
+                            cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
+  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", 2,
+                             kv ? Vc : nullptr, kv ? b.v : nullptr);
 }
 
 cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
   return launch_tc<TM_CROSS>(b, w, kp, b.k, w.bext, b.M_max, w.kperm, w.kperm_ext, b.n_max, b.M_max, s, t,
-                             "cross_tc");
+                             "cross_tc", 1, kv ? b.v : nullptr, w.vperm);
 }
 
 cudaError_t launch_project_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
   return launch_tc<TM_PROJECT>(b, w, kp, b.k, w.bext, b.M_max, w.kperm, w.kperm_ext, b.n_max, b.M_max, s, t,
-                               "project_tc");
+                               "project_tc", 1, kv ? b.v : nullptr, w.vperm);
 }
 
 cudaError_t launch_subtract_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
   return launch_tc<TM_SUB>(b, w, kp, w.ksurv, w.ksurv_ext, b.M_max, w.kevict, w.kevict_ext, b.n_max, b.M_max, s,
-                           t, "subtract_tc");
+                           t, "subtract_tc", 1, w.vsurv, w.vevict);
 }
 
 cudaError_t launch_newbase_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {
+  const bool kv = w.vperm != nullptr;
   return launch_tc<TM_NEWBASE>(b, w, kp, w.kperm, w.kperm_ext, b.n_max, b.k, w.bext, b.M_max, b.n_max, s, t,
-                               "newbase_tc", 2);
+                               "newbase_tc", 2, w.vperm, kv ? b.v : nullptr);
 }
 
 }  // namespace dkv

@@ -174,9 +174,10 @@ __device__ __forceinline__ void norms_ext_tail(float* a, int h, int row0, int n,
   }
 }
 
+// V != nullptr ([K; V] descriptor): the norms are those of [k; v], V laid out like K.
 template <typename T>
-__device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t head_stride, int rows_cap,
-                                               const int32_t* count, int count_is_occ, int N,
+__device__ __forceinline__ void row_norms_body(const T* __restrict__ K, const T* __restrict__ V, int64_t head_stride,
+                                               int rows_cap, const int32_t* count, int count_is_occ, int N,
                                                float* __restrict__ out, int64_t out_hs, int d,
                                                __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
   const int h = blockIdx.y;
@@ -187,8 +188,11 @@ __device__ __forceinline__ void row_norms_body(const T* __restrict__ K, int64_t 
   const int l = lane_id();
   float a[NR_ROWS];
 #pragma unroll
-  for (int q = 0; q < NR_ROWS; ++q)
-    a[q] = row0 + q < n ? sq_sum<T>(K + (int64_t)h * head_stride + (int64_t)(row0 + q) * d + l * pl, pl) : 0.f;
+  for (int q = 0; q < NR_ROWS; ++q) {
+    const int64_t off = (int64_t)h * head_stride + (int64_t)(row0 + q) * d + l * pl;
+    a[q] = row0 + q < n ? sq_sum<T>(K + off, pl) : 0.f;
+    if (V && row0 + q < n) a[q] += sq_sum<T>(V + off, pl);
+  }
   norms_ext_tail(a, h, row0, n, out, out_hs, ext, ext_hs, goff);
 }
 
@@ -319,17 +323,18 @@ __device__ __forceinline__ void rope_lane(float* x, int pl, int e0, int d, int l
 }
 
 template <typename T>
-__global__ void k_row_norms(const T* __restrict__ K, int64_t head_stride, int rows_cap, const int32_t* count,
-                            int count_is_occ, int N, float* __restrict__ out, int64_t out_hs, int d,
-                            __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
-  row_norms_body<T>(K, head_stride, rows_cap, count, count_is_occ, N, out, out_hs, d, ext, ext_hs, goff);
+__global__ void k_row_norms(const T* __restrict__ K, const T* __restrict__ V, int64_t head_stride, int rows_cap,
+                            const int32_t* count, int count_is_occ, int N, float* __restrict__ out, int64_t out_hs,
+                            int d, __nv_bfloat16* __restrict__ ext, int64_t ext_hs, float goff) {
+  row_norms_body<T>(K, V, head_stride, rows_cap, count, count_is_occ, N, out, out_hs, d, ext, ext_hs, goff);
 }
 
 // First kernel of an update: the candidates' norms and extension rows, the zeroed
 // crossing histogram, and the update snapshot (prepare_body) in one extra block (last x,
 // head 0); the three share no data.
 template <typename T>
-__global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, int N, int64_t step, float goff) {
+__global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, const T* __restrict__ Vc, int N, int64_t step,
+                               float goff) {
   if (blockIdx.x == gridDim.x - 1) {
     if (blockIdx.y == 0) prepare_body(b, w, N, step);
     return;
@@ -341,7 +346,7 @@ __global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, int N, in
          i += nthr)
       w.hist[i] = 0;
   }
-  row_norms_body<T>(Kc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm, b.n_max, b.d, (__nv_bfloat16*)w.cext,
+  row_norms_body<T>(Kc, Vc, (int64_t)N * b.d, N, nullptr, 0, N, w.cnorm, b.n_max, b.d, (__nv_bfloat16*)w.cext,
                     (int64_t)b.n_max * 32, goff);
 }
 
@@ -350,8 +355,9 @@ __global__ void k_cand_prepare(Bank b, Ws w, const T* __restrict__ Kc, int N, in
 // take batches of NR_ROWS rows of one head: rotated back into w.kevict ([H][N][d], the
 // layout of Kc), norms and extension rows of the stored keys.  Last CTA: prepare_body.
 template <typename T>
-__global__ void __launch_bounds__(256) k_cand_prepare_rope(Bank b, Ws w, const T* __restrict__ Kc, int N,
-                                                           int64_t step, float goff, const RopeArgs ra) {
+__global__ void __launch_bounds__(256) k_cand_prepare_rope(Bank b, Ws w, const T* __restrict__ Kc,
+                                                           const T* __restrict__ Vc, int N, int64_t step, float goff,
+                                                           const RopeArgs ra) {
   if (blockIdx.x == gridDim.x - 1) {
     prepare_body(b, w, N, step);
     return;
@@ -404,6 +410,7 @@ __global__ void __launch_bounds__(256) k_cand_prepare_rope(Bank b, Ws w, const T
       rope_lane<T>(x[q], pl, l * pl, d, ra.layout, tb, q0 + q);
       store_lane<T>(Kout + ((int64_t)h * N + x0 + q0 + q) * d + l * pl, pl, x[q]);
       a[q] = fmaf(x[q][3], x[q][3], fmaf(x[q][2], x[q][2], fmaf(x[q][1], x[q][1], x[q][0] * x[q][0])));
+      if (Vc) a[q] += sq_sum<T>(Vc + ((int64_t)h * N + x0 + q0 + q) * d + l * pl, pl);   // [K; V] descriptor
     }
     norms_ext_tail(a, h, x0 + q0, x0 + nr, w.cnorm, b.n_max, (__nv_bfloat16*)w.cext, (int64_t)b.n_max * 32, goff);
   }
@@ -1041,20 +1048,24 @@ __global__ void k_seq_gather(Bank b, Ws w, const char* __restrict__ Kc, const ch
 
 static float ext_goff(const KParams& kp) { return kp.eps * 0.5f / kp.inv_s2; }   // eps sigma^2 / 2
 
-cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, int N, int64_t step, const KParams& kp,
-                              const RopeArgs* rope, cudaStream_t s, Timer* t) {
+cudaError_t launch_cand_norms(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, int64_t step,
+                              const KParams& kp, const RopeArgs* rope, cudaStream_t s, Timer* t) {
+  if (!w.vperm) Vc = nullptr;   // values enter the norms with the [K; V] descriptor only
   dim3 grid((N + 8 * NR_ROWS - 1) / (8 * NR_ROWS) + 1, b.H);   // + the prepare block
   timer_begin(t, "cand_norms", s);
   if (rope) {
     const dim3 rgrid((N + ROPE_ROWS - 1) / ROPE_ROWS + 1);   // + the prepare block
     if (b.bf16)
-      k_cand_prepare_rope<__nv_bfloat16><<<rgrid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, N, step, ext_goff(kp), *rope);
+      k_cand_prepare_rope<__nv_bfloat16><<<rgrid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc,
+                                                               (const __nv_bfloat16*)Vc, N, step, ext_goff(kp), *rope);
     else
-      k_cand_prepare_rope<float><<<rgrid, 256, 0, s>>>(b, w, (const float*)Kc, N, step, ext_goff(kp), *rope);
+      k_cand_prepare_rope<float><<<rgrid, 256, 0, s>>>(b, w, (const float*)Kc, (const float*)Vc, N, step,
+                                                       ext_goff(kp), *rope);
   } else if (b.bf16) {
-    k_cand_prepare<__nv_bfloat16><<<grid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, N, step, ext_goff(kp));
+    k_cand_prepare<__nv_bfloat16><<<grid, 256, 0, s>>>(b, w, (const __nv_bfloat16*)Kc, (const __nv_bfloat16*)Vc, N,
+                                                       step, ext_goff(kp));
   } else {
-    k_cand_prepare<float><<<grid, 256, 0, s>>>(b, w, (const float*)Kc, N, step, ext_goff(kp));
+    k_cand_prepare<float><<<grid, 256, 0, s>>>(b, w, (const float*)Kc, (const float*)Vc, N, step, ext_goff(kp));
   }
   timer_end(t, s);
   return cudaGetLastError();
@@ -1064,13 +1075,15 @@ cudaError_t launch_bank_norms(const Bank& b, const Ws& w, const KParams& kp, cud
   dim3 grid((b.M_max + 8 * NR_ROWS - 1) / (8 * NR_ROWS), b.H);
   __nv_bfloat16* ext = (__nv_bfloat16*)w.bext;
   timer_begin(t, "bank_norms", s);
+  const void* V = w.vperm ? b.v : nullptr;   // [K; V] descriptor: norms of [k; v]
   if (b.bf16)
-    k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)b.k, (int64_t)b.M_max * b.d, b.M_max,
-                                                    b.occ, 1, 0, b.knorm, b.M_max, b.d, ext,
-                                                    (int64_t)b.M_max * 32, ext_goff(kp));
+    k_row_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)b.k, (const __nv_bfloat16*)V,
+                                                    (int64_t)b.M_max * b.d, b.M_max, b.occ, 1, 0, b.knorm, b.M_max,
+                                                    b.d, ext, (int64_t)b.M_max * 32, ext_goff(kp));
   else
-    k_row_norms<float><<<grid, 256, 0, s>>>((const float*)b.k, (int64_t)b.M_max * b.d, b.M_max, b.occ, 1, 0,
-                                            b.knorm, b.M_max, b.d, ext, (int64_t)b.M_max * 32, ext_goff(kp));
+    k_row_norms<float><<<grid, 256, 0, s>>>((const float*)b.k, (const float*)V, (int64_t)b.M_max * b.d, b.M_max,
+                                            b.occ, 1, 0, b.knorm, b.M_max, b.d, ext, (int64_t)b.M_max * 32,
+                                            ext_goff(kp));
   timer_end(t, s);
   return cudaGetLastError();
 }
