@@ -32,18 +32,19 @@ def _cat_heads(parts, dtype):
     return torch.cat([to_dev(p, dtype) for p in parts], dim=0).contiguous()
 
 
-@pytest.mark.parametrize("mode", ["tc", "fp32"])
-@pytest.mark.parametrize("sync", [1, 0])
-def test_grouped_layers_match_one_handle_per_layer(dkv, mode, sync):
+@pytest.mark.parametrize("mode,sync,desc", [("tc", 1, 0), ("tc", 0, 0), ("fp32", 1, 0), ("fp32", 0, 0),
+                                             ("tc", 1, 1), ("fp32", 1, 1)])
+def test_grouped_layers_match_one_handle_per_layer(dkv, mode, sync, desc):
+    """desc = 1: the [K; V] descriptor (App. E)."""
     L, H = 3, 2
     # per-layer budgets differ, so the layers fill, saturate and freeze at different steps
     budgets = [300, 300, 190, 250, 420, 420]
     wl = synth.get_workload("wan13b_layer_h12", L=L, H=H, N=96, W=96, Nq=64, budgets=budgets, steps=9)
     sm = dkv.DKV_SCORE_TENSOR if mode == "tc" else dkv.DKV_SCORE_FP32
     dt = torch.bfloat16
-    sep = [dkv.BankLayer(H, wl.d, wl.budgets_of_layer(l), wl.N, dt, score_mode=sm, sync_heads=sync)
-           for l in range(L)]
-    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, dt, score_mode=sm, sync_heads=sync, layer_heads=H)
+    kw = dict(score_mode=sm, sync_heads=sync, descriptor=desc)
+    sep = [dkv.BankLayer(H, wl.d, wl.budgets_of_layer(l), wl.N, dt, **kw) for l in range(L)]
+    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, dt, layer_heads=H, **kw)
     assert grp.n_layers == L
     for b in sep + [grp]:
         b.reset()

@@ -118,19 +118,21 @@ def test_rezeroed_keys_wide_angles(dkv, dtype, layout):
     bank.close()
 
 
-@pytest.mark.parametrize("mode", ["fp32", "tc"])
-@pytest.mark.parametrize("layout", sorted(LAYOUTS))
-def test_rope_rollout_matches_oracle(dkv, mode, layout):
+@pytest.mark.parametrize("mode,layout,desc", [("fp32", "interleaved", 0), ("fp32", "half", 0),
+                                              ("tc", "interleaved", 0), ("tc", "half", 0), ("tc", "interleaved", 1)])
+def test_rope_rollout_matches_oracle(dkv, mode, layout, desc):
     """Teacher-forced rollout (d = 128 bf16, N = 300, M = 700, 3 heads) whose blocks arrive
     rotated to their frames' coordinates: decisions, r*, retained sets, K/V bits and
-    densities against the oracle updating with rope_rezero of the same keys."""
+    densities against the oracle updating with rope_rezero of the same keys (desc = 1:
+    with the [K; V] descriptor, re-zeroed key then value)."""
     wl = synth.get_workload("wan13b_layer_h12", H=3, N=300, W=200, Nq=130, budgets=700, steps=7)
     sm = dkv.DKV_SCORE_TENSOR if mode == "tc" else dkv.DKV_SCORE_FP32
     tol, dens = (1e-3, 1e-2) if mode == "tc" else (2e-4, 2e-4)
-    bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(0), wl.N, torch.bfloat16, score_mode=sm)
+    kw = dict(descriptor=desc, sigma=float(np.sqrt(wl.d))) if desc else {}
+    bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(0), wl.N, torch.bfloat16, score_mode=sm, **kw)
     bank.reset()
     ro = synth.LayerRollout(wl, 0)
-    ob = oracle.LayerBank.empty(wl.budgets_of_layer(0), wl.d)
+    ob = oracle.LayerBank.empty(wl.budgets_of_layer(0), wl.d * (2 if desc else 1))
     theta = synth.temporal_rope_theta(wl.d, layout_first=(layout == "interleaved"))
     for t in range(wl.steps):
         b = wl.admitted_block(t)
