@@ -100,6 +100,21 @@ def parse_args():
     return args
 
 
+def update_pairs(hs, N, rmax):
+    """Key-pair interactions the update's pair passes evaluate, summed over heads: scores
+    m N (Eq. 6), crossings m rmax (Eqs. 8-9), the projection resumed from the last
+    128-column snapshot m (r* mod 128) (Eq. C.2), survivor maintenance (m - e) e
+    (Eq. C.4) and new baselines r* m' (Eq. 5); an empty bank only the last."""
+    tot = 0
+    for h in hs:
+        m, r, e, m2 = h.occupancy_before, h.admitted, h.evicted, h.occupancy_after
+        if m == 0:
+            tot += r * m2
+        else:
+            tot += m * N + m * rmax + m * (r % 128) + (m - e) * e + r * m2
+    return tot
+
+
 def rotate_to_frames(K, t, theta, layout):
     """Input synthesis for --rope: keys as a backbone's local window holds them, each
     rotation pair turned by its token's temporal coordinate (z -> z e^{i t theta}),
@@ -403,6 +418,7 @@ def run_ours(args):
         bank.set_timing(True)   # with graphs, the timing events were captured into them
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     keys = 0
+    pairs = 0
     stats = []
     wall0 = time.perf_counter()
     for i in range(K):
@@ -419,6 +435,7 @@ def run_ours(args):
         L, hs = bank.stats()
         if wl.admitted_block(t) is not None:
             keys += sum(h.occupancy_before + wl.N for h in hs)
+            pairs += update_pairs(hs, wl.N, L.rmax)
         # occupancy_before is the bank this step's attention read
         stats.append((L.r_star, sum(h.evicted for h in hs), sum(h.mandatory for h in hs),
                       sum(h.occupancy_before for h in hs)))
@@ -431,6 +448,7 @@ def run_ours(args):
     bank.sync()
     total_ms = sum(step_ms)
     total_ms_max, keys_all = reduce_over_ranks(total_ms, keys, world, dev)
+    _, pairs_all = reduce_over_ranks(total_ms, pairs, world, dev)
     value = keys_all / (total_ms_max / 1e3)
 
     # ---- end to end through the C ABI with host buffers: H2D inputs, compute, D2H output.
@@ -632,7 +650,7 @@ def run_ours(args):
                        "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
                        "parallelism": f"{world} independent layers, no collective" if world > 1 else "single layer"},
             "blocks_per_s": world * K / (total_ms_max / 1e3),
-            "interaction_pairs_per_s": None,
+            "interaction_pairs_per_s": pairs_all / (total_ms_max / 1e3),
             "wall_s_timed": wall,
             "e2e": e2e, "gpu_launches": launches * world, "roofline": roof, "cpu_baseline": cpu,
             "clocks": clk, "per_kernel": per_kernel,
