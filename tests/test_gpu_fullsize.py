@@ -88,10 +88,14 @@ def _rstar_from_cross(cross_all, occ, budgets, rmax, sync):
     return None, [None if f is None else int(np.nonzero(f)[0].max()) for f in per_head]
 
 
-def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0):
+def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0, kv=False):
+    """kv: the [K; V] descriptor (App. E); every interaction below is then taken between
+    [k; v] rows."""
     rng = np.random.default_rng(seed)
+    extra = dict(descriptor=dkv.DKV_DESC_KV, sigma=float(np.sqrt(wl.d))) if kv else {}
     bank = dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(0), wl.N, torch.bfloat16,
-                         score_mode=dkv.DKV_SCORE_TENSOR, sync_heads=sync_heads)
+                         score_mode=dkv.DKV_SCORE_TENSOR, sync_heads=sync_heads, **extra)
+    desc = (lambda K, V: oracle.kv_descriptor(K, V)) if kv else (lambda K, V: np.asarray(K, dtype=np.float64))
     bank.reset()
     prm = oracle.Params(tau=float(bank.params.tau), sigma=float(bank.params.sigma), p=float(bank.params.p),
                         eps=float(bank.params.eps), delta=float(np.float32(bank.params.delta)),
@@ -136,7 +140,7 @@ def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0):
                 assert r == min(N, M)
                 assert sorted(after["src"][h, :r].tolist()) == list(range(r))
                 continue
-            Kb = snap["K"][h, :m]
+            Kb = desc(snap["K"][h, :m], snap["V"][h, :m])
             rho0, b0 = snap["rho"][h, :m].astype(np.float64), snap["base"][h, :m].astype(np.float64)
             s_gpu = inter["score"][h, :N]
             pi = inter["perm"][h, :N]
@@ -146,10 +150,10 @@ def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0):
             assert np.all((sp[1:] > sp[:-1]) | ((sp[1:] == sp[:-1]) & (pi[1:] > pi[:-1])))
             # Eq. 6 on sampled candidates
             xs = rng.choice(N, size=min(cands, N), replace=False)
-            s_ref = (_w(prm, d, Kc[h][xs].astype(np.float64), Kb) / b0[None, :]).sum(1) / m
+            s_ref = (_w(prm, d, desc(Kc[h][xs], Vc[h][xs]), Kb) / b0[None, :]).sum(1) / m
             assert np.max(np.abs(s_gpu[xs] - s_ref) / s_ref) < TOL_DENS, (t, h)
             # crossing and rho~(r) of sampled rows under the GPU's pi
-            Kpi = Kc[h][pi].astype(np.float64)
+            Kpi = desc(Kc[h][pi], Vc[h][pi])
             rowsel = rng.choice(m, size=min(rows, m), replace=False)
             rmax = L.rmax
             Wr = _w(prm, d, Kb[rowsel], Kpi[:rmax])                       # [rows, rmax]
@@ -198,7 +202,7 @@ def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0):
                     assert np.array_equal(after["K"][h, i], Kc[h][k_[1]]) and \
                         np.array_equal(after["V"][h, i], Vc[h][k_[1]])
             # cached densities vs Phi over the final bank (sampled)
-            Kf = after["K"][h, :mnew]
+            Kf = desc(after["K"][h, :mnew], after["V"][h, :mnew])
             sel = rng.choice(mnew, size=min(rows, mnew), replace=False)
             phi = _w(prm, d, Kf[sel], Kf).sum(1) - prm.eps ** (-prm.p)     # Eq. 3: self excluded by index
             rho_f = after["rho"][h, sel]
@@ -209,6 +213,14 @@ def _run(dkv, wl, steps, sync_heads=1, rows=40, cands=40, seed=0):
     occ_final = bank.occupancy_host()
     bank.close()
     return evicted_total, occ_final
+
+
+def test_fullsize_wan13b_layer_kv_descriptor(dkv):
+    """The [K; V] descriptor at the bench size (12 heads, N = 4,680, M = 9,360), tensor
+    mode, the first four steps (fill, saturation, eviction)."""
+    wl = synth.get_workload("wan13b_layer_h12")
+    evicted, _ = _run(dkv, wl, steps=4, kv=True)
+    assert evicted > 0
 
 
 def test_fullsize_wan13b_layer(dkv):
