@@ -94,13 +94,15 @@ def test_rezeroed_keys_bit_exact_fullsize(dkv, layout):
     bank.close()
 
 
+@pytest.mark.parametrize("d", [128, 64])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("layout", sorted(LAYOUTS))
-def test_rezeroed_keys_wide_angles(dkv, dtype, layout):
+def test_rezeroed_keys_wide_angles(dkv, dtype, layout, d):
     """Random coordinates in [-70,000, 70,000] (negative too, many distinct ones per row
-    strip), random frequencies up to 3 in most pairs: angles from 0 to 2e5 rad."""
+    strip), random frequencies up to 3 in most pairs: angles from 0 to 2e5 rad; both
+    head dimensions (at d = 64 a lane holds one pair, or half a split pair)."""
     rng = np.random.default_rng(7)
-    H, N, d = 3, 1000, 128
+    H, N = 3, 1000
     K = synth.round_to_bf16(rng.normal(size=(H, N, d)).astype(np.float32) * 4.0)
     V = synth.round_to_bf16(rng.normal(size=(H, N, d)).astype(np.float32))
     t = rng.integers(-70000, 70000, size=N).astype(np.int32)
@@ -109,7 +111,7 @@ def test_rezeroed_keys_wide_angles(dkv, dtype, layout):
     theta = (rng.uniform(0, 3, size=d // 2) * (rng.uniform(size=d // 2) < 0.9)).astype(np.float32)
     theta[:4] = np.float32([1e-6, 1.0, 2.5e-3, 0.0])
     bank = _admit_empty(dkv, K, V, t, theta, layout, dtype,
-                        score_mode=dkv.DKV_SCORE_FP32 if dtype == torch.float32 else None)
+                        score_mode=dkv.DKV_SCORE_FP32 if dtype == torch.float32 or d != 128 else None)
     Ks, _ = _stored_in_source_order(bank, N)
     want = oracle.rope_rezero(K, t, theta, layout, "bf16" if dtype == torch.bfloat16 else "fp32")
     bad = np.argwhere(Ks != want)

@@ -322,19 +322,21 @@ def test_bounded_wait_gives_up_and_context_stays_usable(dkv):
     _rollout(dkv, wl, "fp32", check_attn=False)
 
 
-@pytest.mark.parametrize("mode", ["fp32", "tc"])
-def test_sequential_admission_matches_oracle(dkv, mode):
+@pytest.mark.parametrize("mode,desc", [("fp32", 0), ("tc", 0), ("fp32", 1)])
+def test_sequential_admission_matches_oracle(dkv, mode, desc):
     """Within-block competition (App. E): teacher-forced blocks, each offered one candidate
     per head at a time in the order fixed at block start; the retained sets (keyed by
     provenance) must match the oracle exactly, K/V bit for bit, rho and b within the
-    mode's density tolerance.  The first block (all heads empty) takes the whole block."""
+    mode's density tolerance.  The first block (all heads empty) takes the whole block.
+    desc = 1: with the [K; V] descriptor (the oracle offers [k; v] rows)."""
     import gpu_util
     wl = synth.get_workload("wan13b_layer_h12", H=2, N=24, W=24, Nq=16, budgets=[56, 72], steps=6)
-    bank = _bank(dkv, wl, _mode(dkv, mode))
+    kw = dict(descriptor=desc, sigma=float(np.sqrt(wl.d))) if desc else {}
+    bank = _bank(dkv, wl, _mode(dkv, mode), **kw)
     prm = gpu_util.oracle_params(bank)
     _, dens = _tols(mode)
     ro = synth.LayerRollout(wl, 0)
-    ob = oracle.LayerBank.empty(wl.budgets_of_layer(0), wl.d)
+    ob = oracle.LayerBank.empty(wl.budgets_of_layer(0), wl.d * (2 if desc else 1))
     gated = 0
     for t in range(wl.steps):
         b = wl.admitted_block(t)
@@ -344,14 +346,15 @@ def test_sequential_admission_matches_oracle(dkv, mode):
         load_state(bank, ob)
         bank.update_sequential(to_dev(K, bank.dtype), to_dev(V, bank.dtype), b)
         bank.sync()
-        recs = oracle.update_layer_sequential(ob, K, V, b, prm)
+        recs = oracle.update_layer_sequential(ob, oracle.kv_descriptor(K, V) if desc else K, V, b, prm)
         gated += sum(1 for r in recs if r.r_star == 0)
         got, want = gpu_util.gpu_heads(bank), gpu_util.oracle_heads(ob)
         for h in range(wl.H):
             assert set(got[h]) == set(want[h]), (t, h, sorted(set(got[h]) ^ set(want[h]))[:6])
             for key, (k, v, rho, base, _, _) in got[h].items():
                 wk, wv, wrho, wbase = want[h][key]
-                assert np.array_equal(k, wk.astype(np.float32)) and np.array_equal(v, wv.astype(np.float32)), key
+                assert np.array_equal(k, wk[:k.shape[0]].astype(np.float32)) and \
+                    np.array_equal(v, wv.astype(np.float32)), key
                 assert abs(rho - wrho) <= dens * max(abs(wrho), 1e-30), (t, h, key, rho, wrho)
                 assert abs(base - wbase) <= dens * max(abs(wbase), 1e-30), (t, h, key, base, wbase)
     assert gated > 0   # some offers were gated out: the candidates did compete
