@@ -1,5 +1,6 @@
 // Host implementation of the C ABI declared in include/dkv.h.
 #include "../../include/dkv.h"
+#include <nvtx3/nvToolsExt.h>
 #include "dkv_internal.h"
 
 #include <cmath>
@@ -71,7 +72,17 @@ static void record(cudaEvent_t e, cudaStream_t s) {
     cudaEventRecord(e, s);
 }
 
+// NVTX: every kernel launch sits in a range named after it, every ABI call in one named
+// after the call (host-side ranges; free unless a profiler is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 void timer_begin(Timer* t, const char* name, cudaStream_t s) {
+  nvtxRangePushA(name);   // popped by timer_end
   if (!t || !t->on) return;
   if (t->attend_only && std::strncmp(name, "attend", 6) != 0) {   // counted, not timed
     auto it = t->acc.find(name);
@@ -89,6 +100,7 @@ void timer_begin(Timer* t, const char* name, cudaStream_t s) {
 }
 
 void timer_end(Timer* t, cudaStream_t s) {
+  nvtxRangePop();
   if (!t || !t->on || !t->cur_a) return;
   cudaEvent_t b = t->get();
   record(b, s);
@@ -363,6 +375,7 @@ dkv_status_t dkv_bank_reset(dkv_bank_t bank, void* stream) {
 
 static dkv_status_t admit_impl(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
                                const RopeArgs* rope, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_admit");
   if (!bank || !Kc || !Vc) return DKV_ERR_ARG;
   if (bank->state != 0) return DKV_ERR_STATE;
   if (N < 1 || N > bank->b.n_max) return DKV_ERR_SHAPE;
@@ -405,6 +418,7 @@ dkv_status_t dkv_bank_admit_rope(dkv_bank_t bank, const void* Kc, const void* Vc
 }
 
 dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_evict");
   if (!bank) return DKV_ERR_ARG;
   if (bank->state != 1) return DKV_ERR_STATE;
   cudaStream_t s = (cudaStream_t)stream;
@@ -420,6 +434,7 @@ dkv_status_t dkv_bank_evict(dkv_bank_t bank, void* stream) {
 }
 
 dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_commit");
   if (!bank) return DKV_ERR_ARG;
   if (bank->state != 2) return DKV_ERR_STATE;
   cudaStream_t s = (cudaStream_t)stream;
@@ -483,6 +498,7 @@ size_t dkv_sequential_scratch_size(int32_t H, int32_t d, int32_t n_max, int32_t 
 
 dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const void* Vc, int32_t N, int64_t step,
                                         void* scratch, size_t scratch_bytes, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_update_sequential");
   if (!bank || !Kc || !Vc || !scratch) return DKV_ERR_ARG;
   if (bank->state != 0) return DKV_ERR_STATE;
   if (N < 1 || N > bank->b.n_max) return DKV_ERR_SHAPE;
@@ -537,6 +553,7 @@ dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const v
 
 dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const void* Kw, const void* Vw,
                              int32_t W, void* O, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_attend");
   if (!bank || !Q || !O) return DKV_ERR_ARG;
   if (Nq < 1 || Nq > (1 << 20) || W < 0 || W > (1 << 20)) return DKV_ERR_SHAPE;
   if (W > 0 && (!Kw || !Vw)) return DKV_ERR_ARG;
@@ -549,6 +566,7 @@ dkv_status_t dkv_bank_attend(dkv_bank_t bank, const void* Q, int32_t Nq, const v
 }
 
 dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* stream) {
+  NvtxRange nvtx_range("dkv_bank_import");
   if (!bank || !occupancy) return DKV_ERR_ARG;
   if (bank->state != 0) return DKV_ERR_STATE;
   for (int h = 0; h < bank->b.H; ++h)
