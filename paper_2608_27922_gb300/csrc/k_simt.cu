@@ -4,11 +4,15 @@
 // then w = (eps + d2 / sigma^2)^(-p) (Eq. 2).  These kernels serve fp32 banks
 // and the DKV_SCORE_FP32 mode of bf16 banks.
 //
-// One thread owns one row and walks the columns in increasing order, so the
-// running sums of Eq. C.2 are formed in the same order by the crossing pass
-// and by the projection pass that later resumes them from a snapshot.
+// Two neighbouring threads share two rows: each holds one half of the dimensions of
+// both rows, forms the two half sums (sequential fused multiply-adds), and one shuffle
+// gives each thread d2 = first half + second half of its own row (same order in every
+// pass).  Each thread walks the columns in increasing order, so the running sums of
+// Eq. C.2 are formed in the same order by the crossing pass and by the projection pass
+// that later resumes them from a snapshot.  Every staged column element thus serves
+// two rows (half the shared-memory reads of a one-row-per-thread layout).
 // With the [K; V] descriptor (App. E "Retention geometry") two neighbouring threads
-// own a row, one its key and one its value; d2 = d2_key + d2_value after one shuffle,
+// own one row, one its key and one its value; d2 = d2_key + d2_value after one shuffle,
 // identical in both, and the even thread writes.
 #include "dkv_internal.h"
 
@@ -44,6 +48,7 @@ template <typename T, int D, int MODE, bool KV>
 __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
   constexpr int DC = KV ? 2 * D : D;   // staged floats per column: key (| value)
   constexpr int RPB = KV ? ROWS / 2 : ROWS;   // rows per block
+  constexpr int DH = D / 2;
   extern __shared__ float smem[];
   float* cs = smem;               // [CT][DC] staged column keys (| values)
   float* cmeta = smem + CT * DC;  // [CT]     per-column factor (SCORE: 1 / b_j)
@@ -60,18 +65,29 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
   if (MODE == PM_NEWBASE) { nrows = hd.r;                           c1 = hd.m_new; }
   const int row0 = blockIdx.x * RPB;
   if (row0 >= nrows) return;
-  const int half = KV ? (threadIdx.x & 1) : 0;        // KV: 0 key, 1 value
-  const int row = row0 + (KV ? (threadIdx.x >> 1) : threadIdx.x);
+  const int half = threadIdx.x & 1;   // KV: 0 key, 1 value; else: dimensions [half D/2, +D/2)
+  const int pr = threadIdx.x >> 1;
+  const int row = KV ? row0 + pr : row0 + 2 * pr + half;
   const bool active = row < nrows;
-  const bool writer = active && half == 0;
+  const bool writer = KV ? active && half == 0 : active;
   const int64_t bh = (int64_t)h * j.b.M_max;   // bank head offset (rows)
 
-  // this thread's row key (or value), in registers
+  // KV: this thread's row key (or value); else halves of the pair's two rows:
+  // rr[0, D/2) = row 2 pr, rr[D/2, D) = row 2 pr + 1, dimensions [half D/2, half D/2 + D/2)
   float rr[D];
-  {
+  if (KV) {
     const T* rp = ptr<T>(half ? j.rv : j.rk, (int64_t)h * j.rk_hs + (int64_t)(active ? row : 0) * D);
 #pragma unroll
     for (int k = 0; k < D; ++k) rr[k] = active ? to_f<T>(rp[k]) : 0.f;
+  } else {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int rq = row0 + 2 * pr + q;
+      const bool aq = rq < nrows;
+      const T* rp = ptr<T>(j.rk, (int64_t)h * j.rk_hs + (int64_t)(aq ? rq : 0) * D + half * DH);
+#pragma unroll
+      for (int k = 0; k < DH; ++k) rr[q * DH + k] = aq ? to_f<T>(rp[k]) : 0.f;
+    }
   }
 
   // per-row state
@@ -111,18 +127,32 @@ __global__ void __launch_bounds__(ROWS) simt_pairs(PairJob j) {
     if (MODE == PM_SCORE)
       for (int c = threadIdx.x; c < nc; c += ROWS) cmeta[c] = __frcp_rn(j.b.base[bh + t0 + c]);
     __syncthreads();
-    if (!KV && !active) continue;   // KV: both threads of a row pair take part in the shuffle
+    // every thread takes part in the shuffles (a thread whose row is past the end too)
     for (int c = 0; c < nc; ++c) {
-      const float* col = cs + c * DC + half * D;
-      float d2 = 0.f;
-#pragma unroll
-      for (int k = 0; k < D; ++k) {
-        float df = __fsub_rn(rr[k], col[k]);
-        d2 = __fmaf_rn(df, df, d2);
-      }
+      float d2;
       if (KV) {
+        const float* col = cs + c * DC + half * D;
+        d2 = 0.f;
+#pragma unroll
+        for (int k = 0; k < D; ++k) {
+          float df = __fsub_rn(rr[k], col[k]);
+          d2 = __fmaf_rn(df, df, d2);
+        }
         const float other = __shfl_xor_sync(0xffffffffu, d2, 1);
         d2 = half ? __fadd_rn(other, d2) : __fadd_rn(d2, other);   // key part + value part
+      } else {
+        const float* col = cs + c * DC + half * DH;
+        float q0 = 0.f, q1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < DH; ++k) {
+          const float x = col[k];
+          const float d0 = __fsub_rn(rr[k], x), d1 = __fsub_rn(rr[DH + k], x);
+          q0 = __fmaf_rn(d0, d0, q0);
+          q1 = __fmaf_rn(d1, d1, q1);
+        }
+        // the partner needs this thread's half of its row: row 2 pr + 1 - half
+        const float other = __shfl_xor_sync(0xffffffffu, half ? q0 : q1, 1);
+        d2 = half ? __fadd_rn(other, q1) : __fadd_rn(q0, other);    // first half + second half
       }
       const float w = riesz_w(d2, j.kp);
       const int jc = t0 + c;
