@@ -1,0 +1,48 @@
+"""Host-side helpers of bench.py on the CPU: the interaction-pair count behind
+`interaction_pairs_per_s` and the input synthesis of `--rope`."""
+import os
+import sys
+import types
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+import oracle  # noqa: E402
+import synth  # noqa: E402
+
+
+def _head(m, r, e, m2):
+    return types.SimpleNamespace(occupancy_before=m, admitted=r, evicted=e, occupancy_after=m2)
+
+
+def test_update_pairs_counts_each_pass():
+    N = 4680
+    # steady state of the single-layer workload: m = M = 9,360, r* = e = N
+    steady = _head(9360, N, N, 9360)
+    want = 9360 * N + 9360 * N + 9360 * (N % 128) + (9360 - N) * N + N * 9360
+    assert bench.update_pairs([steady], N, N) == want == 153990720
+    # an empty bank only computes the new baselines of the admitted block
+    assert bench.update_pairs([_head(0, N, 0, N)], N, N) == N * N
+    # no eviction: no survivor pass; r* a multiple of 128: no projection columns
+    assert bench.update_pairs([_head(1000, 256, 0, 1256)], N, 300) == 1000 * N + 1000 * 300 + 0 + 0 + 256 * 1256
+    # heads add up
+    assert bench.update_pairs([steady, steady], N, N) == 2 * want
+
+
+def test_rope_input_synthesis_is_undone_by_the_oracle():
+    """Keys rotated to their frames by bench.rotate_to_frames come back to the generated
+    keys (up to the storage rounding) under the oracle's re-zeroing, in both layouts."""
+    rng = np.random.default_rng(5)
+    K = synth.round_to_bf16(rng.normal(size=(2, 40, 128)).astype(np.float32) * 3.0)
+    t = (np.arange(40) // 8 + 11).astype(np.int32)
+    for layout in ("interleaved", "half"):
+        theta = synth.temporal_rope_theta(128, layout_first=layout == "interleaved")
+        Kt = bench.rotate_to_frames(torch.from_numpy(K).to(torch.bfloat16), t, theta, layout).float().numpy()
+        assert not np.allclose(Kt, K)
+        back = oracle.rope_rezero(Kt, t, theta, layout, storage=None)
+        assert np.max(np.abs(back - K)) <= 2.0 ** -7 * np.max(np.abs(K))
