@@ -132,3 +132,52 @@ def test_binding_has_no_fallback(monkeypatch):
     monkeypatch.setattr(dkv, "_LIB", None)
     with pytest.raises(RuntimeError):
         dkv.lib()
+
+
+def test_plain_c_program_links_and_calls_the_library():
+    """A C program that includes dkv.h and links libdkv.so: the host-only calls and the
+    argument errors behave as documented, with no Python in between."""
+    dkv = _built_lib()
+    if not shutil.which("gcc"):
+        pytest.skip("gcc unavailable")
+    from paper_2608_27922_gb300 import build as B
+    src = r"""
+#include <stdio.h>
+#include <string.h>
+#include "dkv.h"
+int main(void) {
+  dkv_params_t p;
+  if (dkv_params_default(&p, 128) != DKV_OK || p.tau != 2.0f || p.sigma != 8.0f || p.descriptor != DKV_DESC_K)
+    return 1;
+  int32_t budgets[12];
+  for (int h = 0; h < 12; ++h) budgets[h] = 9360;
+  size_t a = dkv_bank_workspace_size(12, 128, budgets, 4680, DKV_DTYPE_BF16);
+  size_t b = dkv_bank_workspace_size_ex(12, 128, budgets, 4680, DKV_DTYPE_BF16, &p);
+  p.descriptor = DKV_DESC_KV;
+  size_t c = dkv_bank_workspace_size_ex(12, 128, budgets, 4680, DKV_DTYPE_BF16, &p);
+  if (a == 0 || a != b || c <= a) return 2;
+  if (dkv_bank_workspace_size(12, 96, budgets, 4680, DKV_DTYPE_BF16) != 0) return 3;
+  if (dkv_bank_admit(NULL, NULL, NULL, 1, 0, NULL) != DKV_ERR_ARG) return 4;
+  if (dkv_bank_admit_rope(NULL, NULL, NULL, 1, 0, NULL, NULL, DKV_ROPE_HALF, NULL) != DKV_ERR_ARG) return 5;
+  if (dkv_bank_compress(NULL, NULL) != DKV_ERR_ARG || dkv_bank_sync(NULL) != DKV_ERR_ARG) return 6;
+  if (strlen(dkv_status_str(DKV_ERR_TIMEOUT)) == 0 || dkv_version() < 100) return 7;
+  dkv_bank_destroy(NULL);
+  printf("%d %zu\n", dkv_version(), a);
+  return 0;
+}
+"""
+    tmp = os.path.join(ROOT, "tests", "_abi_c_probe")
+    with open(tmp + ".c", "w") as f:
+        f.write(src)
+    try:
+        subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), tmp + ".c", "-o", tmp,
+                               "-L", B.LIBDIR, "-ldkv", "-Wl,-rpath," + B.LIBDIR])
+        out = subprocess.run([tmp], capture_output=True, text=True)
+    finally:
+        for p in (tmp + ".c", tmp):
+            if os.path.exists(p):
+                os.remove(p)
+    assert out.returncode == 0, (out.returncode, out.stderr)
+    ver, ws = out.stdout.split()
+    assert int(ver) == dkv.dkv_version() and int(ws) == dkv.dkv_bank_workspace_size(12, 128, [9360] * 12, 4680,
+                                                                                       dkv.DKV_DTYPE_BF16)
