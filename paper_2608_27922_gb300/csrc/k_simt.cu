@@ -269,8 +269,42 @@ __global__ void __launch_bounds__(AQ) simt_attend(const T* __restrict__ Q, int N
       vs[e] = c < m ? to_f<T>(vb[(int64_t)c * D + k]) : to_f<T>(vw[(int64_t)(c - m) * D + k]);
     }
     __syncthreads();
+    // four keys at a time: each staged query element serves four dot products and the
+    // running maximum is raised at most once per four keys
+    int c = 0;
 #pragma unroll 1
-    for (int c = 0; c < nc; ++c) {
+    for (; c + 4 <= nc; c += 4) {
+      float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+      for (int k = 0; k < D; ++k) {
+        const float q = qs[k * AQ + threadIdx.x];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a[u] = fmaf(q, ks[(c + u) * D + k], a[u]);
+      }
+      const float amax = fmaxf(fmaxf(a[0], a[1]), fmaxf(a[2], a[3]));
+      if (amax > mrun) {   // online softmax: rescale the running sums to the new maximum
+        const float alpha = exp2f(mrun - amax);
+        l *= alpha;
+#pragma unroll
+        for (int k = 0; k < D; ++k) acc[k] *= alpha;
+        mrun = amax;
+      }
+      float pu[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        pu[u] = exp2f(a[u] - mrun);
+        l += pu[u];
+      }
+#pragma unroll
+      for (int k = 0; k < D; ++k) {
+        float x = acc[k];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x = fmaf(pu[u], vs[(c + u) * D + k], x);
+        acc[k] = x;
+      }
+    }
+#pragma unroll 1
+    for (; c < nc; ++c) {
       float a = 0.f;
 #pragma unroll 8
       for (int k = 0; k < D; ++k) a = fmaf(qs[k * AQ + threadIdx.x], ks[c * D + k], a);
