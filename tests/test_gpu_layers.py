@@ -10,8 +10,9 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import synth
-from gpu_util import to_dev
+from gpu_util import check_report, to_dev, tols, update_and_compare_layers
 
 pytestmark = pytest.mark.gpu
 
@@ -85,6 +86,38 @@ def test_grouped_layers_match_one_handle_per_layer(dkv, mode, sync, desc):
     assert any(len(set(r)) > 1 for r in rstars), rstars
     for bk in sep + [grp]:
         bk.close()
+
+
+@pytest.mark.parametrize("mode,sync", [("tc", 1), ("tc", 0), ("fp32", 1), ("fp32", 0)])
+def test_grouped_layers_match_oracle(dkv, mode, sync):
+    """A three-layer handle (ragged sizes, per-layer budgets) teacher-forced against
+    oracle.update_layer run on every layer by itself: each layer's r* (Eq. 11 per layer),
+    scores, order, crossings, retained set, K/V bits and densities at the mode's bar."""
+    L, H = 3, 3
+    budgets = [700, 700, 700, 420, 520, 600, 900, 900, 650]
+    wl = synth.get_workload("wan13b_layer_h12", L=L, H=H, N=300, W=64, Nq=64, budgets=budgets, steps=7)
+    sm = dkv.DKV_SCORE_TENSOR if mode == "tc" else dkv.DKV_SCORE_FP32
+    grp = dkv.BankLayer(L * H, wl.d, list(wl.budgets), wl.N, torch.bfloat16, layer_heads=H, score_mode=sm,
+                        sync_heads=sync)
+    grp.reset()
+    tol, dens = tols(mode)
+    ro = [synth.LayerRollout(wl, l) for l in range(L)]
+    obs = [oracle.LayerBank.empty(wl.budgets_of_layer(l), wl.d) for l in range(L)]
+    rstars, evicted = [], 0
+    for t in range(wl.steps):
+        b = wl.admitted_block(t)
+        if b is None:
+            continue
+        blocks = [ro[l].block(b) for l in range(L)]
+        reps, recs = update_and_compare_layers(grp, obs, [x[0] for x in blocks], [x[1] for x in blocks], b,
+                                               tol, dens)
+        for l, rep in enumerate(reps):
+            check_report(rep, mode, (t, l))
+        rstars.append(tuple(r.rstar_oracle for r in reps))
+        evicted += sum(len(hr.evicted) for rec in recs for hr in rec.heads)
+    assert evicted > 0
+    assert any(len(set(r)) > 1 for r in rstars), rstars   # the layers took different prefixes
+    grp.close()
 
 
 def test_grouped_layers_rope(dkv):
