@@ -382,14 +382,18 @@ dkv_status_t dkv_selftest_wait_timeout(int32_t limit_us, int64_t* elapsed_ns);
  *
  * Limits: 1 <= N <= DKV_NOALLOC_MAX_N (else DKV_ERR_SHAPE, nothing is launched),
  * 0 <= m <= 262144, d in {64, 128}.
+ * Arithmetic: that of the fp32 score mode of dkv_bank_admit, in the same order, so
+ * the scores and the order are bit-identical to admit's in that mode.
  * Memory: the scores live in a fixed 64 KiB device array inside the library (one
  * per GPU that loads it, kept until the process exits); the call allocates nothing,
- * on the device or through any library.  The first call on each device looks up
- * that array's device address and sets a kernel attribute, once; make that first
- * call before any stream capture.  Nothing in the array needs clearing: every
- * entry a call reads is written earlier in the same call.  All calls on a device
- * share the array, so calls whose work overlaps on the GPU (different streams
- * without ordering between them) race; order them on one stream.               */
+ * on the device or through any library.  The first successful call on each device
+ * (made with that device current) looks up that array's device address and sets a
+ * kernel attribute; make that first call before any stream capture.  If that set-up
+ * fails the call returns DKV_ERR_CUDA and the next call on the device tries again.
+ * Nothing in the array needs clearing: every entry a call reads is written earlier
+ * in the same call.  All calls on a device share the array, so calls whose work
+ * overlaps on the GPU (different streams without ordering between them) race;
+ * order them on one stream.                                                      */
 dkv_status_t dkv_candidate_order_noalloc(const void* K_bank, const float* base, int32_t m, const void* Kc,
                                          int32_t N, int32_t d, int32_t dtype, const dkv_params_t* params,
                                          float* scores_out, int32_t* perm_out, void* stream);

@@ -11,9 +11,12 @@
 // file-scope device array below, of a fixed size.
 //
 // The scoring kernel is the fp32 direct-difference variant of the Eq. 6 pass for
-// one head (same arithmetic, same column order as the fp32 score mode of
-// dkv_bank_admit); the ordering kernel is the stable ascending sort with ties in
-// source order.
+// one head, with the arithmetic of the fp32 score mode of dkv_bank_admit in the same
+// order: d2 = (sequential fused multiply-adds over the first half of the dimensions)
+// + (the same over the second half), one rounded add joining them; w by the shared
+// Eq. 2 helper; the weighted sum over bank columns in increasing order; one division
+// by m.  Its scores are therefore bit-identical to admit's in that mode.  The ordering
+// kernel is the stable ascending sort with ties in source order.
 #include "../../include/dkv.h"
 #include "dkv_device.cuh"
 
@@ -52,13 +55,14 @@ __global__ void __launch_bounds__(ROWS) noalloc_score(const T* __restrict__ Kb, 
     if (!active) continue;
     for (int c = 0; c < nc; ++c) {
       const float* col = cs + c * D;
-      float d2 = 0.f;
+      float q0 = 0.f, q1 = 0.f;   // first and second half of the dimensions
 #pragma unroll
-      for (int k = 0; k < D; ++k) {
-        const float df = __fsub_rn(rr[k], col[k]);
-        d2 = __fmaf_rn(df, df, d2);
+      for (int k = 0; k < D / 2; ++k) {
+        const float d0 = __fsub_rn(rr[k], col[k]), d1 = __fsub_rn(rr[D / 2 + k], col[D / 2 + k]);
+        q0 = __fmaf_rn(d0, d0, q0);
+        q1 = __fmaf_rn(d1, d1, q1);
       }
-      acc = __fmaf_rn(riesz_w(d2, kp), cinv[c], acc);
+      acc = __fmaf_rn(riesz_w(__fadd_rn(q0, q1), kp), cinv[c], acc);
     }
   }
   if (active) scratch[x] = __fdiv_rn(acc, (float)m);
@@ -97,31 +101,37 @@ __global__ void __launch_bounds__(SORT_THREADS) noalloc_order(const float* __res
   }
 }
 
-// One-time set-up per device: the device address of the scratch array (host code
-// may not use the array's name as an address) and the shared-memory opt-in of the
-// ordering kernel.
+// Set-up per device, with that device current: the device address of the scratch
+// array (in host code the array's name is only a host-side stand-in) and the
+// shared-memory opt-in of the ordering kernel.  Only a complete success is kept; a
+// failed attempt leaves nothing behind, so the next call on that device tries again.
 constexpr int kMaxDevices = 64;
 struct DeviceSetup {
-  std::once_flag once;
-  cudaError_t err = cudaSuccess;
+  bool ready = false;
   float* scratch = nullptr;
 };
 DeviceSetup g_setup[kMaxDevices];
+std::mutex g_setup_mu;
 
 cudaError_t setup_device(int dev, float** scratch) {
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
   DeviceSetup& s = g_setup[dev];
-  std::call_once(s.once, [&s] {
+  if (!s.ready) {
     void* p = nullptr;
-    s.err = cudaGetSymbolAddress(&p, g_noalloc_scores);
-    if (s.err == cudaSuccess) {
-      s.scratch = static_cast<float*>(p);
-      s.err = cudaFuncSetAttribute(noalloc_order, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   DKV_NOALLOC_MAX_N * (int)sizeof(unsigned long long));
+    cudaError_t err = cudaGetSymbolAddress(&p, g_noalloc_scores);
+    if (err == cudaSuccess)
+      err = cudaFuncSetAttribute(noalloc_order, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 DKV_NOALLOC_MAX_N * (int)sizeof(unsigned long long));
+    if (err != cudaSuccess) {
+      (void)cudaGetLastError();   // do not leave the failure to the next unrelated check
+      return err;
     }
-  });
+    s.scratch = static_cast<float*>(p);
+    s.ready = true;
+  }
   *scratch = s.scratch;
-  return s.err;
+  return cudaSuccess;
 }
 
 }  // namespace
