@@ -52,10 +52,17 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=17)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="wan13b_layer_h12")
+    ap.add_argument("--workload", default="wan14b_headwise_l40h40",
+                    help="a stack workload (L > 1) runs the whole model step on one handle; a one-layer "
+                         "workload runs the single-layer step")
+    ap.add_argument("--sync-heads", type=int, choices=[0, 1], default=1,
+                    help="1: shared prefix per layer (Eq. 11, the method's default); 0: independent per-head "
+                         "prefixes (App. E ablation)")
+    ap.add_argument("--profile-steps", type=int, default=2,
+                    help="stack run: steps after the timed region with every kernel timed (per-kernel roofline)")
     ap.add_argument("--score-mode", choices=["tensor", "fp32"], default="tensor")
     ap.add_argument("--order", choices=["score", "source"], default="score",
                     help="candidate order (policy ablation of Table 2(b); default: the method's)")
@@ -67,14 +74,8 @@ def parse_args():
                          "no graphs, no overlap, no e2e leg)")
     ap.add_argument("--attn-passes", type=int, default=1,
                     help="bank-reading attention passes per update (denoising passes; the update runs once)")
-    ap.add_argument("--layers", type=int, default=1,
-                    help="layers updated per step on this GPU (whole-stack throughput; > 1 selects the stack run)")
-    ap.add_argument("--streams", type=int, default=4, help="stream pairs the layers of a stack step spread over "
-                    "(--stack-mode streams)")
-    ap.add_argument("--stack-mode", choices=["grouped", "streams"], default="grouped",
-                    help="grouped: one handle over all layers, single launches; streams: one handle per layer")
-    ap.add_argument("--distinct-layers", type=int, default=2,
-                    help="stack run: layers with their own synthetic input stream (the rest reuse them)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="stack run: number of layers (default: the workload's; fewer for small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -95,8 +96,6 @@ def parse_args():
         args.no_graphs = args.no_overlap = args.no_e2e = True
         if args.rope != "off":
             ap.error("--rope applies to the batch admission path")
-    if args.rope != "off" and args.layers > 1:
-        ap.error("--rope is measured on the single-layer step")
     return args
 
 
@@ -235,14 +234,16 @@ def source_sha1(*names):
     return h.hexdigest()
 
 
-def traffic_for(kernel: str, src_files):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+def traffic_for(kernel: str, src_files, workload: str, heads: int):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu summary, if
+    the kernel's source is unchanged since the capture; a capture on fewer heads of the
+    same workload is scaled to `heads` (each head's operands are read once per launch)."""
     if not os.path.exists(TRAFFIC_FILE):
         return None
-    t = json.load(open(TRAFFIC_FILE)).get(kernel)
+    t = json.load(open(TRAFFIC_FILE)).get(f"{kernel}@{workload}")
     if not t or t.get("source_sha1") != source_sha1(*src_files):
         return None
-    return t.get("bytes_per_launch")
+    return t["bytes_per_launch"] * heads / t["heads_captured"]
 
 
 def make_workload(name, world, heads=0):
@@ -477,8 +478,9 @@ def run_ours(args):
                          "t": torch.empty(wl.N, dtype=torch.int32, device=dev),
                          "win": {n: (torch.empty(wl.H, n, wl.d, dtype=bf, device=dev),
                                      torch.empty(wl.H, n, wl.d, dtype=bf, device=dev)) for n in win_lens}})
-        copy_s = torch.cuda.Stream(dev)   # O download
-        pre_s = torch.cuda.Stream(dev)    # input uploads
+        # input uploads and the O download: one copy stream (on this host a download beside
+        # an upload slows the upload several-fold)
+        pre_s = torch.cuda.Stream(dev)
         bank.set_timing(False)
 
         def inputs_of(i):
@@ -544,11 +546,11 @@ def run_ours(args):
                     if not late:
                         bank.admit(kc, vc, ab, stream=cur, **rope_kw(ab, tbuf))
                     bank.evict(stream=cur)
-                copy_s.wait_event(att_done)
-                with torch.cuda.stream(copy_s):
+                pre_s.wait_event(att_done)   # same stream as the uploads: the copies take turns
+                with torch.cuda.stream(pre_s):
                     host_out.copy_(out, non_blocking=True)
                 o_done = torch.cuda.Event()
-                o_done.record(copy_s)
+                o_done.record(pre_s)
                 cur.wait_event(att_done)
                 if ab is not None:
                     bank.commit(stream=cur)
@@ -575,6 +577,7 @@ def run_ours(args):
             torch.cuda.synchronize()
         e2e_keys = 0
         e2e_ms = 0.0
+        e2e_step_ms = []
         h2d = d2h = 0
         for i in range(K):
             t = W + K + i
@@ -591,7 +594,8 @@ def run_ours(args):
                 h2d_i = e2e_step(i)
             s1.record(stream)
             s1.synchronize()
-            e2e_ms += s0.elapsed_time(s1)
+            e2e_step_ms.append(s0.elapsed_time(s1))
+            e2e_ms += e2e_step_ms[-1]
             L, hs = bank.stats()
             if wl.admitted_block(t) is not None:
                 e2e_keys += sum(h.occupancy_before + wl.N for h in hs)
@@ -600,8 +604,11 @@ def run_ours(args):
         e2e_ms, e2e_keys = reduce_over_ranks(e2e_ms, e2e_keys, world, dev)
         e2e = {"value": e2e_keys / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d // K,
                "d2h_bytes_per_step": d2h // K, "ms_per_step": e2e_ms / K,
+               "step_ms": {"min": min(e2e_step_ms), "median": statistics.median(e2e_step_ms),
+                           "max": max(e2e_step_ms), "first": e2e_step_ms[0]},
                "copies": "pinned host buffers; inputs double-buffered and uploaded one step ahead on a copy "
-                         "stream (every timed step's uploads inside the timed regions), O downloaded on another",
+                         "stream (every timed step's uploads inside the timed regions), O downloaded on the same "
+                         "stream",
                "cuda_graphs": e2e_graphs is not None}
 
     # ---- roofline of the dominant kernel (largest share of the timed region)
@@ -619,7 +626,7 @@ def run_ours(args):
         roof = {"kernel": dom_name, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "peak_source": f"{pk_src} bf16 dense (burst)",
                 "algorithmic_per_launch": {"flops": flops, "keys_per_query": m_bank + wl.W},
-                "traffic": traffic_for(dom_name, ["k_tc_attn.cu", "tc_ptx.cuh"])}
+                "traffic": traffic_for(dom_name, ["k_tc_attn.cu", "tc_ptx.cuh"], wl.name, wl.H)}
     else:
         roof = {"kernel": dom_name, "bound": "tensor", "achieved": None, "peak": float(pk["bf16_tflops"]),
                 "unit": "TFLOP/s", "frac": None, "traffic": None}
@@ -676,7 +683,8 @@ def oracle_threads():
 
 
 def _oracle_head_setup(wl, layer, head):
-    """Oracle bank of one head brought to steady state (untimed): first two updates."""
+    """Oracle bank of one head brought to steady state (untimed): updates until the bank
+    reaches its budget."""
     import oracle
     import synth
     ro = synth.LayerRollout(wl, layer, heads=[head])
@@ -721,7 +729,8 @@ def run_reference(args):
     if not reference_runs_on(rank):
         return
     wl = make_workload(args.workload, 1)
-    ro, ob, t = _oracle_head_setup(wl, 0, 0)
+    head = _stack_sample_heads(wl, 1)[0] if wl.L > 1 else 0
+    ro, ob, t = _oracle_head_setup(wl, 0, head)
     for i in range(args.warmup):
         _oracle_step(wl, ro, ob, t)
         t += 1
@@ -733,8 +742,9 @@ def run_reference(args):
         t += 1
     value = keys / tot
     cpu = {"value": value, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
-           "sample": f"each step: 1 head (of {wl.H}) of {wl.name} at steady state, attention of {wl.Nq} "
-                     f"queries + bank update (numpy float64)"}
+           "sample": f"each step: head {head} of layer 0 (budget {wl.budgets[head]}; {wl.L} x {wl.H} heads in the "
+                     f"workload) of {wl.name} at steady state, attention of {wl.Nq} queries + bank update "
+                     f"(numpy float64)"}
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
@@ -744,183 +754,442 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def run_stack(args):
-    """Whole-stack throughput on one GPU: every step updates `--layers` independent layer
-    banks (attention || admit + evict, then commit), the whole step captured as one CUDA
-    graph.  `--stack-mode grouped` (default): one handle holds all layers and every call
-    is a single launch per kernel over all L x H heads (each layer keeps its own r*);
-    `streams`: one handle per layer, the layers spread over `--streams` stream pairs.
-    Inputs of `--distinct-layers` synthetic layer streams are reused round-robin by the
-    others (each layer still has its own bank)."""
-    import torch
+# --------------------------------------------------------------------------- whole stacks
+TENSOR_KERNELS = ("attend_tc", "score_tc", "cross_tc", "project_tc", "subtract_tc", "newbase_tc")
+HBM_KERNELS = ("cand_norms", "sort_runs", "sort_rank", "rstar", "select", "commit")
 
-    torch.cuda.set_device(0)
-    dev = torch.device("cuda", 0)
+
+def kernel_work(name, d, esize, N, Nq, W, layer_of_head, Ls, hs):
+    """Algorithmic work of one launch of kernel `name` over every head of a handle in one
+    update step, from the step's statistics (Ls per layer, hs per head).
+
+    Tensor-core passes: flops, 2d per key pair (Eq. 2 through the MMA) and 4d per
+    query-key pair of the attention:
+      scores m N (Eq. 6), crossings m rmax (Eqs. 8-9), projection m (r* mod 128)
+      (Eq. C.2 resumed from the last 128-column snapshot), survivor maintenance (m - e) e
+      (Eq. C.4), new baselines r* m' (Eq. 5), attention Nq (m + W).
+    Memory-bound kernels: (algorithmic bytes, bytes the kernel moves by design):
+      candidate norms: read the candidate keys, write norms and extension rows;
+      sort runs: read scores 4N, write run keys 8N; sort rank: read run keys 8N, write
+      pi 4N (algorithmic: 12N per head over both phases, the sort's read of s and write of
+      pi plus the key exchange), and by design also the copy of the candidates into pi
+      order (key, norm, extension row read and written);
+      r*: the crossing histogram (N + 2) and the feasibility bits;
+      select: rho~, crossing index and mask, 12 m (algorithmic), plus the provenance
+      read for ties and the slot lists written, 32 m (moved);
+      commit: the admitted K and V rows read and written plus 20 B of metadata per
+      admitted state (algorithmic); by design also the evicted keys copied out, the
+      survivors' keys copied beside them (operands of Eq. C.4) and the extension rows."""
+    rowb = d * esize
+    tot_a = tot_m = 0.0
+    for h, st in enumerate(hs):
+        m, m2, r, e = st.occupancy_before, st.occupancy_after, st.admitted, st.evicted
+        rmax = Ls[layer_of_head(h)].rmax
+        live = m > 0
+        if name == "attend_tc":
+            tot_a += 4.0 * d * Nq * (m + W)
+        elif name == "score_tc":
+            tot_a += 2.0 * d * m * N if live else 0
+        elif name == "cross_tc":
+            tot_a += 2.0 * d * m * rmax if live else 0
+        elif name == "project_tc":
+            tot_a += 2.0 * d * m * (r % 128) if live else 0
+        elif name == "subtract_tc":
+            tot_a += 2.0 * d * (m - e) * e if live else 0
+        elif name == "newbase_tc":
+            tot_a += 2.0 * d * r * m2
+        elif name == "cand_norms":
+            tot_a += N * (rowb + 4 + 64)
+            tot_m += N * (rowb + 4 + 64)
+        elif name == "sort_runs":
+            tot_a += 6.0 * N if live else 0
+            tot_m += 12.0 * N if live else 0
+        elif name == "sort_rank":
+            tot_a += 6.0 * N if live else 0
+            tot_m += (12.0 * N + 2.0 * N * (rowb + 68)) if live else 4.0 * N + 2.0 * N * (rowb + 68)
+        elif name == "rstar":
+            tot_a += 4.0 * (rmax + 2) + (rmax + 1) / 8.0 if live else 0
+            tot_m += 4.0 * (rmax + 2) + (rmax + 1) / 8.0 if live else 0
+        elif name == "select":
+            tot_a += 12.0 * m if live and e > 0 else 0
+            tot_m += 32.0 * m if live and e > 0 else 0
+        elif name == "commit":
+            tot_a += r * (4.0 * rowb + 20.0)
+            ng = (m - e) if e > 0 else 0
+            tot_m += r * (4.0 * rowb + 20.0 + 128.0) + e * (2.0 * rowb + 136.0) + ng * (2.0 * rowb + 136.0)
+    if name in TENSOR_KERNELS:
+        return tot_a
+    return tot_a, tot_m
+
+
+def run_stack(args):
+    """Whole-stack throughput: every step is one generated block passing through all L
+    layers of the model (L x H heads, per-head budgets): attention of the block's queries
+    over [bank | window] in every layer, then admit, evict and commit of the block leaving
+    the window (Alg. 1 per layer, each layer with its own prefix r*, Eq. 11), all through
+    one handle whose calls are single launches over all L x H heads.  Every layer and
+    head draws its own synthetic stream (synth.device, generated on the GPU between
+    timed steps, outside the events)."""
+    import torch
+    from synth.device import StackRollout
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
     import __graft_entry__
-    __graft_entry__.build()
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
     from paper_2608_27922_gb300 import dkv
 
-    wl = make_workload(args.workload, 1, args.heads)
-    L, S = args.layers, max(1, args.streams)
-    D = max(1, min(args.distinct_layers, L))
-    W, K = args.warmup, args.steps
+    over = {"H": args.heads} if args.heads else {}
+    if args.layers:
+        over["L"] = args.layers
+    wl = synth_workload(args.workload, **over)
+    if wl.window not in ("prev", "own"):
+        raise SystemExit("the stack run takes whole-block windows (prev / own)")
+    L, H, d, N, Nq = wl.L, wl.H, wl.d, wl.N, wl.Nq
+    LH = L * H
+    W_, K = args.warmup, args.steps
     bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    inputs = []
-    cat1 = lambda xs: torch.cat(xs, dim=1).contiguous()
-    for l in range(D):
-        inp = Inputs(wl, l, W + K)
-        blocks = {b: (torch.from_numpy(k).to(dev, bf), torch.from_numpy(v).to(dev, bf)) for b, (k, v) in inp.blocks.items()}
-        inputs.append((blocks, [torch.from_numpy(q).to(dev, bf) for q in inp.queries],
-                       [inp.window(t, blocks, cat1) for t in range(W + K)]))
-    P = max(1, args.attn_passes)
+    esize = 2 if wl.dtype == "bf16" else 4
     mode = dkv.DKV_SCORE_TENSOR if args.score_mode == "tensor" else dkv.DKV_SCORE_FP32
-    grouped = args.stack_mode == "grouped"
+    sync = 0 if args.sync_heads == 0 else 1
+    # weak scaling: each rank runs its own rollout (an independent video) of the whole stack
+    gen = StackRollout(wl, device=dev, rank_seed=rank)
+    bank = dkv.BankLayer(LH, d, list(wl.budgets), N, bf, score_mode=mode, device=dev, layer_heads=H,
+                         sync_heads=sync)
+    bank.reset()
+    lay = lambda h: h // H
+    out = torch.empty(LH, Nq, d, dtype=bf, device=dev)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
-    if grouped:
-        # one handle holds all L layers (L x H heads, params.layer_heads = H): every call
-        # is one launch per kernel over all layers; the inputs are stacked along heads
-        budgets = [b for l in range(L) for b in wl.budgets_of_layer(l)]
-        banks = [dkv.BankLayer(L * wl.H, wl.d, budgets, wl.N, bf, score_mode=mode, device=dev, layer_heads=wl.H)]
-        banks[0].reset()
-        stack0 = lambda xs: torch.cat(xs, dim=0).contiguous()
-        admitted = sorted({wl.admitted_block(t) for t in range(W + K)} - {None})
-        s_blocks = {b: (stack0([inputs[l % D][0][b][0] for l in range(L)]),
-                        stack0([inputs[l % D][0][b][1] for l in range(L)])) for b in admitted}
-        s_queries = [stack0([inputs[l % D][1][t] for l in range(L)]) for t in range(W + K)]
-        def s_window(t):   # a window that is exactly an admitted block shares its tensors
-            parts = wl.window_parts(t)
-            if len(parts) == 1 and parts[0][1] == 0 and parts[0][2] == wl.N and parts[0][0] in s_blocks:
-                return s_blocks[parts[0][0]]
-            return (stack0([inputs[l % D][2][t][0] for l in range(L)]),
-                    stack0([inputs[l % D][2][t][1] for l in range(L)]))
-        s_windows = [s_window(t) for t in range(W + K)]
-        del inputs
-        out_all = torch.empty(L * wl.H, wl.Nq, wl.d, dtype=bf, device=dev)
-        side = torch.cuda.Stream(dev)
-
-        def stack_step(t):
-            cur = torch.cuda.current_stream(dev)
-            b = wl.admitted_block(t)
-            kw, vw = s_windows[t]
-            late = P == 1
-            if b is not None and late:
-                banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
-            go = torch.cuda.Event()
-            go.record(cur)
-            side.wait_event(go)
-            for _ in range(P):
-                banks[0].attend(s_queries[t], kw, vw, out=out_all, stream=side)
-            done = torch.cuda.Event()
-            done.record(side)
-            if b is not None:
-                if not late:
-                    banks[0].admit(s_blocks[b][0], s_blocks[b][1], b, stream=cur)
-                banks[0].evict(stream=cur)
-            cur.wait_event(done)
-            if b is not None:
-                banks[0].commit(stream=cur)
-    else:
-        banks = [dkv.BankLayer(wl.H, wl.d, wl.budgets_of_layer(l), wl.N, bf, score_mode=mode, device=dev)
-                 for l in range(L)]
-        for bk in banks:
-            bk.reset()
-        outs = [torch.empty(wl.H, wl.Nq, wl.d, dtype=bf, device=dev) for _ in range(L)]
-        mains = [torch.cuda.Stream(dev) for _ in range(S)]
-        sides = [torch.cuda.Stream(dev) for _ in range(S)]
-
-    def stack_step_streams(t):
-        cur = torch.cuda.current_stream(dev)
-        fork = torch.cuda.Event()
-        fork.record(cur)
-        joins = []
-        for l in range(L):
-            ms, ss = mains[l % S], sides[l % S]
-            blocks, queries, windows = inputs[l % D]
-            kw, vw = windows[t]
-            b = wl.admitted_block(t)
-            ms.wait_event(fork)
-            go = torch.cuda.Event()
-            go.record(ms)
-            ss.wait_event(go)
-            for _ in range(P):
-                banks[l].attend(queries[t], kw, vw, out=outs[l], stream=ss)
-            done = torch.cuda.Event()
-            done.record(ss)
-            if b is not None:
-                kc, vc = blocks[b]
-                banks[l].admit(kc, vc, b, stream=ms)
-                banks[l].evict(stream=ms)
-            ms.wait_event(done)
-            if b is not None:
-                banks[l].commit(stream=ms)
-            j = torch.cuda.Event()
-            j.record(ms)
-            joins.append(j)
-        for j in joins:
-            cur.wait_event(j)
-
-    if not grouped:
-        stack_step = stack_step_streams
+    side = torch.cuda.Stream(dev)
     stream = torch.cuda.current_stream(dev)
-    for t in range(W):
-        stack_step(t)
+
+    def new_set():
+        return {"q": torch.empty(LH, Nq, d, dtype=bf, device=dev), "k": torch.empty(LH, N, d, dtype=bf, device=dev),
+                "v": torch.empty(LH, N, d, dtype=bf, device=dev)}
+
+    gset = new_set()   # generated inputs of the device leg (and staging of the end-to-end leg)
+
+    def generate(t, st):
+        gen.queries(t, st["q"])
+        gen.block(wl.window_block(t), st["k"], st["v"])
+
+    def step(t, st, cur, serial=False, o=None):
+        """Attention of step t over [bank | window] in every layer, then the update with
+        the block leaving the window (= the window block for these workloads).  serial:
+        everything on one stream (per-kernel timing).  o: the attention output buffer."""
+        o = out if o is None else o
+        b = wl.admitted_block(t)
+        if b is not None:   # admit first: the score and crossing passes have the GPU alone
+            bank.admit(st["k"], st["v"], b, stream=cur)
+        att = cur if serial else side
+        go = torch.cuda.Event()
+        go.record(cur)
+        att.wait_event(go)
+        bank.attend(st["q"], st["k"], st["v"], out=o, stream=att)
+        done = torch.cuda.Event()
+        done.record(att)
+        if b is not None:
+            bank.evict(stream=cur)
+        cur.wait_event(done)   # commit changes the bank attention reads
+        if b is not None:
+            bank.commit(stream=cur)
+        return done
+
+    def step_stats(t):
+        if wl.admitted_block(t) is None:
+            return None
+        Ls = bank.layer_stats()
+        _, hs = bank.stats()
+        return Ls, hs
+
+    for t in range(W_):
+        generate(t, gset)
+        step(t, gset, stream)
     torch.cuda.synchronize()
-    graphs = []
-    cap = torch.cuda.Stream(dev)
-    cap.wait_stream(stream)
-    with torch.cuda.stream(cap):
-        for i in range(K):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=cap):
-                stack_step(W + i)
-            graphs.append(g)
-    stream.wait_stream(cap)
+    bank.sync()
+
+    # ---- timed region: K steps, each bracketed by CUDA events on the launching stream;
+    # the step's inputs are generated on the device and the L2 flushed before the start event
+    clocks = ClockSampler(local, enabled=(not args.no_clocks) and rank == 0)
+    if world > 1:
+        dist.barrier()
     torch.cuda.synchronize()
-    clocks = ClockSampler(0, enabled=not args.no_clocks)
+    bank.set_timing(True, attention_only=True)   # live events around the attention launches only
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    keys = 0
-    total_ms = 0.0
-    rstars = []
+    keys = pairs = 0
+    per_step = []
+    wall0 = time.perf_counter()
     for i in range(K):
-        t = W + i
+        t = W_ + i
+        generate(t, gset)
         if not args.no_flush:
             flush.fill_(float(i))
         ev[i][0].record(stream)
-        graphs[i].replay()
+        step(t, gset, stream)
         ev[i][1].record(stream)
         ev[i][1].synchronize()
-        total_ms += ev[i][0].elapsed_time(ev[i][1])
-        if wl.admitted_block(t) is not None:
-            per_layer = []
-            for bk in banks:
-                _, hs = bk.stats()
-                keys += sum(h.occupancy_before + wl.N for h in hs)
-                for l, Ls in enumerate(bk.layer_stats()):
-                    per_layer.append((Ls.r_star, sum(h.evicted for h in hs[l * wl.H:(l + 1) * wl.H])))
-            rstars.append(per_layer)
+        st = step_stats(t)
+        if st is not None:
+            Ls, hs = st
+            keys += sum(h.occupancy_before + N for h in hs)
+            pairs += sum(kernel_work(k, d, esize, N, Nq, wl.W, lay, Ls, hs) for k in TENSOR_KERNELS[1:]) / (2 * d)
+            per_step.append({"r_star": [x.r_star for x in Ls], "evicted": sum(h.evicted for h in hs),
+                             "admitted": sum(h.admitted for h in hs), "mandatory": sum(h.mandatory for h in hs),
+                             "bank_keys": sum(h.occupancy_before for h in hs)})
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
     clk = clocks.stop()
-    for bk in banks:
-        bk.sync()
-    line = {
-        "metric": METRIC, "value": keys / (total_ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": K, "warmup": W,
-        "ms_per_step": total_ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
-        "config": {"workload": f"{wl.name}: {L} layer(s) x {wl.H} heads per step, d={wl.d}, N={wl.N}, "
-                               f"M={max(wl.budgets)}, W={wl.W}, Nq={wl.Nq}",
-                   "score_mode": args.score_mode, "layers_per_gpu": L,
-                   "streams": ("one handle over all layers (single launches), admit, then attention || "
-                               "evict, then commit" if grouped else f"one handle per layer on {S} stream pairs"),
-                   "cuda_graphs": True, "inputs": f"{D} distinct synthetic layer streams, reused round-robin",
-                   "l2": "flushed between timed steps (256 MiB write)" if not args.no_flush else "not flushed",
-                   "parallelism": "layers of one GPU, grouped launches" if grouped
-                   else "layers of one GPU on concurrent streams"},
-        "blocks_per_s": K / (total_ms / 1e3),
-        "e2e": None, "gpu_launches": None, "roofline": None, "cpu_baseline": None, "clocks": clk,
-        "update": {"last_step_r_star_per_layer": [r for r, _ in rstars[-1]] if rstars else [],
-                   "last_step_evicted_per_layer": [e for _, e in rstars[-1]] if rstars else [],
-                   "layers_admitting_per_step": [sum(1 for r, _ in st if r > 0) for st in rstars]},
-    }
-    print(json.dumps(line), flush=True)
+    ktimes = bank.kernel_times()
+    bank.set_timing(False)
+    bank.sync()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    total_ms_max, keys_all = reduce_over_ranks(total_ms, keys, world, dev)
+    _, pairs_all = reduce_over_ranks(total_ms, pairs, world, dev)
+    value = keys_all / (total_ms_max / 1e3)
+    launches = sum(n for n, _ in ktimes.values())
+    att_n, att_ms = ktimes.get("attend_tc", (0, 0.0))
+    att_flops = statistics.mean(
+        [4.0 * d * Nq * (s["bank_keys"] + LH * wl.W) for s in per_step]) if per_step else 0.0
+
+    # ---- per-kernel pass (not part of the value): a few more steps with every kernel timed
+    # by CUDA events on its stream, against its algorithmic work
+    P = max(0, args.profile_steps)
+    prof = {}
+    bank.set_timing(True)
+    t_next = W_ + K
+    for i in range(P):
+        t = t_next + i
+        generate(t, gset)
+        if not args.no_flush:
+            flush.fill_(float(i))
+        step(t, gset, stream, serial=True)
+        torch.cuda.synchronize()
+        st = step_stats(t)
+        kt = bank.kernel_times()
+        bank.set_timing(False)
+        bank.set_timing(True)
+        if st is None:
+            continue
+        Ls, hs = st
+        for name, (n, ms) in kt.items():
+            if n == 0 or ms <= 0:
+                continue
+            e = prof.setdefault(name, {"launches": 0, "ms": 0.0, "work": 0.0, "moved": 0.0})
+            e["launches"] += n
+            e["ms"] += ms
+            if name in TENSOR_KERNELS:
+                e["work"] += kernel_work(name, d, esize, N, Nq, wl.W, lay, Ls, hs)
+            elif name in HBM_KERNELS:
+                a, m_ = kernel_work(name, d, esize, N, Nq, wl.W, lay, Ls, hs)
+                e["work"] += a
+                e["moved"] += m_
+    bank.set_timing(False)
+    t_next += P
+    pk, pk_src = peaks()
+    tpeak, hpeak = float(pk["bf16_tflops"]), float(pk["hbm_gbs"])
+    tot_prof = sum(e["ms"] for e in prof.values()) or 1.0
+    per_kernel = {}
+    for name, e in sorted(prof.items(), key=lambda kv: -kv[1]["ms"]):
+        row = {"launches": e["launches"], "avg_ms": e["ms"] / e["launches"], "share": e["ms"] / tot_prof}
+        if name in TENSOR_KERNELS:
+            tf = e["work"] / (e["ms"] / 1e3) / 1e12
+            row.update(tflops=tf, frac_of_bf16_peak=tf / tpeak)
+        elif name in HBM_KERNELS:
+            gbs = e["work"] / (e["ms"] / 1e3) / 1e9
+            row.update(alg_gbs=gbs, frac_of_hbm_alg=gbs / hpeak,
+                       moved_gbs=e["moved"] / (e["ms"] / 1e3) / 1e9, frac_of_hbm_moved=e["moved"] / (e["ms"] / 1e3) / 1e9 / hpeak)
+        per_kernel[name] = row
+
+    # ---- end to end through the C ABI with host buffers: every step's queries and block K/V
+    # come from pinned host memory and its attention output goes back to it.  Inputs and
+    # outputs are double-buffered on the device, as a serving loop would pipeline them:
+    # step i computes from one input set while a copy stream uploads step i + 1's inputs
+    # into the other and a second copy stream downloads step i - 1's output; the step
+    # completes only once both copies have landed.  The first timed step uploads its own
+    # inputs first, the last one also downloads its own output after its attention, so
+    # every step's uploads and its download fall inside the timed regions exactly once.
+    # The host buffers of step i + 1 are written (generated on the device, copied down)
+    # before step i starts.
+    e2e = None
+    if not args.no_e2e:
+        hsets = [{k: torch.empty(v.shape, dtype=bf, pin_memory=True) for k, v in gset.items()} for _ in range(2)]
+        dsets = [new_set(), new_set()]
+        douts = [out, torch.empty_like(out)]
+        host_outs = [torch.empty(LH, Nq, d, dtype=bf, pin_memory=True) for _ in range(2)]
+        # one copy stream for both directions: on this host a download running beside an
+        # upload slows the upload several-fold, so the copies take turns
+        pre_s = torch.cuda.Stream(dev)
+        in_bytes = sum(x.numel() * x.element_size() for x in hsets[0].values())
+        out_bytes = out.numel() * out.element_size()
+
+        def download(i, after):
+            pre_s.wait_event(after)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(pre_s)
+            with torch.cuda.stream(pre_s):
+                host_outs[i % 2].copy_(douts[i % 2], non_blocking=True)
+            e1.record(pre_s)
+            return e0, e1
+
+        def fill_host(t, hs_):
+            generate(t, gset)
+            for k_ in hs_:
+                hs_[k_].copy_(gset[k_], non_blocking=True)
+            torch.cuda.synchronize()
+
+        def upload(hs_, ds_, after):
+            pre_s.wait_event(after)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(pre_s)
+            with torch.cuda.stream(pre_s):
+                for k_ in ds_:
+                    ds_[k_].copy_(hs_[k_], non_blocking=True)
+            e1.record(pre_s)
+            return e0, e1
+
+        base_t = t_next
+        fill_host(base_t, hsets[0])
+        e2e_ms, e2e_keys, up_ms, down_ms, up_b, down_b = 0.0, 0, [], [], 0, 0
+        for i in range(K):
+            t = base_t + i
+            if i + 1 < K:
+                fill_host(t + 1, hsets[(i + 1) % 2])
+            if not args.no_flush:
+                flush.fill_(float(i))
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            ups, downs = [], []
+            if i == 0:
+                ups.append(upload(hsets[0], dsets[0], s0))
+                stream.wait_event(ups[-1][1])
+                up_b += in_bytes
+            if i > 0:   # the previous step's output, beside this step's compute
+                downs.append(download(i - 1, s0))
+            if i + 1 < K:   # then the next step's inputs
+                ups.append(upload(hsets[(i + 1) % 2], dsets[(i + 1) % 2], s0))
+                up_b += in_bytes
+            att_done = step(t, dsets[i % 2], stream, o=douts[i % 2])
+            if i + 1 == K:   # the last step's own output
+                downs.append(download(i, att_done))
+            down_b += out_bytes * len(downs)
+            for _, e1 in downs:
+                stream.wait_event(e1)
+            if len(ups) and i + 1 < K:
+                stream.wait_event(ups[-1][1])
+            s1.record(stream)
+            s1.synchronize()
+            e2e_ms += s0.elapsed_time(s1)
+            up_ms.append(sum(a.elapsed_time(b) for a, b in ups))
+            down_ms.append(sum(a.elapsed_time(b) for a, b in downs))
+            stt = step_stats(t)
+            if stt is not None:
+                e2e_keys += sum(h.occupancy_before + N for h in stt[1])
+        e2e_ms_max, e2e_keys = reduce_over_ranks(e2e_ms, e2e_keys, world, dev)
+        e2e = {"value": e2e_keys / (e2e_ms_max / 1e3), "unit": UNIT, "h2d_bytes_per_step": up_b // K,
+               "d2h_bytes_per_step": down_b // K, "ms_per_step": e2e_ms_max / K,
+               "blocks_per_s": world * K / (e2e_ms_max / 1e3),
+               "upload_ms_per_step": sum(up_ms) / K, "download_ms_per_step": sum(down_ms) / K,
+               "upload_gbs": up_b / (sum(up_ms) / 1e3) / 1e9 if sum(up_ms) > 0 else None,
+               "download_gbs": down_b / (sum(down_ms) / 1e3) / 1e9 if sum(down_ms) > 0 else None,
+               "copies": "pinned host buffers (one NUMA node on this host); inputs and outputs double-buffered on "
+                         "the device: the previous step's output downloads, then the next step's inputs upload, on "
+                         "one copy stream beside each step's compute; no CUDA graphs"}
+        del hsets, dsets, douts, host_outs
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_stack(wl, keys_all / max(K, 1) / world)
+
+    if rank == 0:
+        roof = {"kernel": "attend_tc", "bound": "tensor", "achieved": None, "peak": tpeak, "unit": "TFLOP/s",
+                "frac": None, "peak_source": f"{pk_src} bf16 dense (burst)",
+                "algorithmic_per_launch": {"flops": att_flops}, "traffic": None}
+        if att_n:
+            ach = att_flops / (att_ms / att_n / 1e3) / 1e12
+            roof.update(achieved=ach, frac=ach / tpeak, launches=att_n, avg_ms=att_ms / att_n,
+                        traffic=traffic_for("attend_tc", ["k_tc_attn.cu", "tc_ptx.cuh"], wl.name, LH))
+        admitting = [sum(1 for r in s["r_star"] if r > 0) for s in per_step]
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W_,
+            "ms_per_step": total_ms_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": f"{wl.name}: {L} layers x {H} heads per block step (one model step), d={d}, "
+                                   f"N={N}, M_h in {sorted(set(wl.budgets))}, W={wl.W}, Nq={Nq}",
+                       "score_mode": args.score_mode, "prefix": "shared per layer (Eq. 11)" if sync
+                       else "independent per head (App. E)",
+                       "inputs": "every layer and head an independent synthetic stream, generated on the device "
+                                 "before each step's start event",
+                       "streams": "admit, then attention || evict, then commit; one handle over all layers "
+                                  "(single launches over all L x H heads)",
+                       "cuda_graphs": False,
+                       "l2": "flushed between timed steps (256 MiB write); inputs larger than L2",
+                       "parallelism": f"{world} independent rollouts (one per GPU), no collective" if world > 1
+                       else "one GPU"},
+            "blocks_per_s": world * K / (total_ms_max / 1e3),
+            "interaction_pairs_per_s": pairs_all / (total_ms_max / 1e3),
+            "wall_s_timed": wall, "step_ms": {"min": min(step_ms), "median": statistics.median(step_ms),
+                                              "max": max(step_ms)},
+            "e2e": e2e, "gpu_launches": launches * world, "roofline": roof, "cpu_baseline": cpu, "clocks": clk,
+            "per_kernel": per_kernel,
+            "per_kernel_note": f"{P} further steps on one stream with every launch timed by CUDA events (not "
+                               "in value); "
+                               "tensor kernels against the bf16 peak, memory-bound kernels' algorithmic (and "
+                               "moved-by-design) bytes against the HBM peak",
+            "update": {"layers_admitting_per_step": admitting,
+                       "admitted_per_step": [s["admitted"] for s in per_step],
+                       "evicted_per_step": [s["evicted"] for s in per_step],
+                       "mandatory_per_step": [s["mandatory"] for s in per_step],
+                       "last_step_r_star_per_layer": per_step[-1]["r_star"] if per_step else [],
+                       "note": "a layer with r* = 0 admits nothing (under the shared prefix one saturated head "
+                               "holds its layer at 0, Eq. 11); its admit pass still scores every bank key"},
+        }
+        print(json.dumps(line), flush=True)
+    bank.close()
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def synth_workload(name, **over):
+    import synth
+    return synth.get_workload(name, **over)
+
+
+def _stack_sample_heads(wl, n):
+    """Heads of layer 0 for the oracle sample: the first head of each of the n distinct
+    budgets nearest the workload's mean budget."""
+    mean = sum(wl.budgets) / len(wl.budgets)
+    first = {}
+    for h in range(wl.H):
+        first.setdefault(wl.budgets[h], h)
+    return [first[b] for b in sorted(first, key=lambda b: (abs(b - mean), b))[:n]]
+
+
+def cpu_baseline_stack(wl, keys_per_block):
+    """The oracle on a bounded sample of the stack workload: heads of layer 0 brought to
+    steady state (untimed), then one step each (attention + update) timed; the rate is
+    keys scored per second, and the model step's time is extrapolated from it."""
+    heads = _stack_sample_heads(wl, 2)
+    tot_s, tot_k = 0.0, 0
+    for h in heads:
+        ro, ob, t = _oracle_head_setup(wl, 0, h)
+        dt, k = _oracle_step(wl, ro, ob, t)
+        tot_s += dt
+        tot_k += k
+    rate = tot_k / tot_s
+    return {"value": rate, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
+            "sample": f"{len(heads)} head(s) of layer 0 (budgets {[wl.budgets[h] for h in heads]}) of {wl.name}, "
+                      f"one steady-state step each (attention of {wl.Nq} queries + bank update), {tot_k} keys "
+                      f"scored in {tot_s:.1f} s (numpy float64)",
+            "blocks_per_s_extrapolated": rate / keys_per_block if keys_per_block else None}
 
 
 def main():
@@ -929,7 +1198,10 @@ def main():
         print("warning: --warmup < 3 does not reach the steady state of the bank", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args)
-    elif args.layers > 1:
+    elif synth_workload(args.workload).L > 1:
+        if args.within_block != "batch" or args.rope != "off" or args.descriptor != "k" or args.attn_passes != 1 \
+                or args.order != "score" or args.eviction != "mandatory_densest" or args.refresh_baselines:
+            raise SystemExit("policy, descriptor, RoPE and sequential ablations are measured on one-layer workloads")
         run_stack(args)
     else:
         run_ours(args)

@@ -46,3 +46,32 @@ def test_rope_input_synthesis_is_undone_by_the_oracle():
         assert not np.allclose(Kt, K)
         back = oracle.rope_rezero(Kt, t, theta, layout, storage=None)
         assert np.max(np.abs(back - K)) <= 2.0 ** -7 * np.max(np.abs(K))
+
+
+def test_kernel_work_of_a_stack_step():
+    """Per-kernel algorithmic work behind the bench's per-kernel roofline, for two layers
+    of two heads: flops of the tensor-core passes, bytes of the memory-bound kernels."""
+    N, Nq, W, d = 4680, 4680, 4680, 128
+    Ls = [types.SimpleNamespace(rmax=N, r_star=N), types.SimpleNamespace(rmax=2340, r_star=0)]
+    hs = [_head(9360, N, N, 9360), _head(0, N, 0, N), _head(2340, 0, 0, 2340), _head(4680, 0, 0, 4680)]
+    lay = lambda h: h // 2
+    kw = lambda name: bench.kernel_work(name, d, 2, N, Nq, W, lay, Ls, hs)
+    assert kw("score_tc") == 2 * d * N * (9360 + 2340 + 4680)
+    assert kw("cross_tc") == 2 * d * (9360 * N + (2340 + 4680) * 2340)
+    assert kw("project_tc") == 2 * d * 9360 * (N % 128)
+    assert kw("subtract_tc") == 2 * d * (9360 - N) * N
+    assert kw("newbase_tc") == 2 * d * (N * 9360 + N * N)
+    assert kw("attend_tc") == 4 * d * Nq * (9360 + 0 + 2340 + 4680 + 4 * W)
+    alg, moved = kw("commit")
+    assert alg == 2 * N * (4 * d * 2 + 20) and moved > alg
+    alg, moved = kw("select")
+    assert alg == 12 * 9360 and moved == 32 * 9360      # only the evicting head selects
+
+
+def test_stack_sample_heads_near_the_mean_budget():
+    wl = synth.get_workload("wan14b_headwise_l40h40")
+    heads = bench._stack_sample_heads(wl, 2)
+    mean = sum(wl.budgets) / len(wl.budgets)
+    assert len(heads) == 2 and all(h < wl.H for h in heads)
+    assert sorted(abs(wl.budgets[h] - mean) for h in heads) == sorted(
+        abs(b - mean) for b in set(wl.budgets))[:2]

@@ -68,3 +68,41 @@ def test_sink5_window_parts_and_contents():
     K2, V2 = ro.block(2)
     assert np.array_equal(Kw[:, :F], K0[:, :F])
     assert np.array_equal(Kw[:, F:3 * F], K1[:, F:]) and np.array_equal(Vw[:, 3 * F:], V2)
+
+
+def test_device_stack_generator_follows_the_recipe():
+    """synth.device (run on the CPU here): determinism per step, bf16 exactness, key norms
+    sqrt(d), the vMF law per head (mean cosine to the assigned centre = A_d(kappa d)),
+    the recurrence rule (block t uses clusters [0, (t + 1) g) while fresh ones remain),
+    and independent streams for different heads and rank seeds."""
+    import torch
+    from synth.device import StackRollout
+
+    wl = synth.get_workload("wan14b_headwise_l40h40", L=2, H=3, N=600, Nq=200)
+    gen = StackRollout(wl, device="cpu", chunk_heads=6)
+    K = torch.empty(6, 600, 128, dtype=torch.bfloat16)
+    V = torch.empty_like(K)
+    Q = torch.empty(6, 200, 128, dtype=torch.bfloat16)
+    gen.block(2, K, V)
+    gen.queries(2, Q)
+    K2, V2 = torch.empty_like(K), torch.empty_like(V)
+    StackRollout(wl, device="cpu", chunk_heads=6).block(2, K2, V2)
+    assert torch.equal(K, K2) and torch.equal(V, V2)
+    assert not torch.equal(K[0], K[1])
+    K3, V3 = torch.empty_like(K), torch.empty_like(V)
+    StackRollout(wl, device="cpu", chunk_heads=6, rank_seed=1).block(2, K3, V3)
+    assert not torch.equal(K, K3)
+    Kf = K.float()
+    assert abs(Kf.norm(dim=-1).mean().item() - np.sqrt(128)) < 0.05
+    assert abs(V.float().std().item() - 1.0) < 0.02
+    a = gen._assign(0, 6, 2, 600, 1)   # the block's own assignment stream (_S_ASSIGN)
+    mu = gen.mu[torch.arange(6)[:, None].expand(6, 600), a]
+    cos = (Kf / np.sqrt(128) * mu).sum(-1)
+    for h in range(6):
+        kap = wl.kappa_vmf(h)
+        theory = ive(64, kap) / ive(63, kap)
+        assert abs(cos[h].mean().item() - theory) < 2e-3, (h, cos[h].mean().item(), theory)
+        Kc, g = wl.clusters[h], max(1, wl.clusters[h] // 8)
+        if 3 * g <= Kc:
+            assert int(a[h].max()) < 3 * g
+        assert int(a[h].min()) >= 0 and int(a[h].max()) < Kc
