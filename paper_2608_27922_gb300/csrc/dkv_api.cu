@@ -162,6 +162,8 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, 
   const int cnt_stride = (part_stride + 127) / 128;
   w.part = (float*)take(2 * Hh * part_stride * 4);
   w.cnt = (int32_t*)take(Hh * cnt_stride * 4);
+  w.tile_head = (int32_t*)take(Hh * ((Mm + 127) / 128) * 4);
+  w.tile_first = (int32_t*)take(Hh * 4);
   w.part_stride = part_stride;
   w.cnt_stride = cnt_stride;
   w.invb_stride = invb_stride;
@@ -355,6 +357,17 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
   if (e == cudaSuccess) e = cudaMemset(bk->w.hd, 0, sizeof(DevHead) * H);
   if (e == cudaSuccess) e = cudaMemset(bk->w.cnt, 0, sizeof(int32_t) * H * bk->w.cnt_stride);
   if (e == cudaSuccess) e = cudaMemcpy(bk->w.budgets, budgets, sizeof(int32_t) * H, cudaMemcpyHostToDevice);
+  // the 128-row tiles of every head's budget, head-major (grids of the passes over bank rows)
+  std::vector<int32_t> tile_head, tile_first(H);
+  for (int h = 0; h < H; ++h) {
+    tile_first[h] = (int32_t)tile_head.size();
+    tile_head.insert(tile_head.end(), (size_t)(budgets[h] + 127) / 128, h);
+  }
+  bk->w.n_mtiles = (int)tile_head.size();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(bk->w.tile_head, tile_head.data(), sizeof(int32_t) * tile_head.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(bk->w.tile_first, tile_first.data(), sizeof(int32_t) * H, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     delete bk;
     return DKV_ERR_CUDA;

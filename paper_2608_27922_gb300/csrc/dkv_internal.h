@@ -62,6 +62,9 @@ struct Ws {
                         //   baselines, kept in step; 128 floats of padding at the end)
   float* part;          // [2][H][part_stride] per-row partial sums of column-split passes
   int32_t* cnt;         // [H][cnt_stride] arrival counters of column-split row tiles (kept 0)
+  int32_t* tile_head;   // [n_mtiles] head of each 128-row tile of the heads' budgets, head-major
+  int32_t* tile_first;  // [H] index of each head's first such tile
+  int n_mtiles;         // sum over heads of ceil(M_h / 128)
   int hist_stride, snap_stride, feas_words, part_stride, cnt_stride, invb_stride, sort_stride;
   int layer_heads;      // heads per layer (the handle's heads form H / layer_heads layers)
 };
@@ -125,6 +128,7 @@ cudaError_t launch_attend_fp32(const Bank& b, const void* Q, int Nq, const void*
 cudaError_t launch_attend_tc(const Bank& b, DevLayer* L, const void* Q, int Nq, const void* Kw, const void* Vw,
                              int W, void* O, cudaStream_t s, Timer* t);
 bool tc_supported(int d, int bf16);
+int sm_count();   // multiprocessors of the current device (0 if unknown)
 cudaError_t simt_set_smem_limits();
 cudaError_t update_set_smem_limits();
 cudaError_t tc_set_smem_limits();

@@ -416,10 +416,308 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------------------------
+// Two query tiles per CTA.  One CTA owns 256 queries of one head as two 128-query
+// tiles Q_0, Q_1 that read every key tile together: each K and V tile crosses from L2
+// into shared memory once per 256 queries instead of once per 128, which halves the
+// L2 -> shared-memory traffic per MMA (one K/V tile per 128 queries needs about as many
+// bytes per cycle as an SM can take from L2 while its tensor pipe is busy).  Softmax
+// group g (four warps, thread = query row) owns Q_g over the whole key range, so no
+// merge is needed at the end.  TMEM columns as above: S_g, O_g for g = 0, 1.
+// Shared memory: Q_0, Q_1, two K slots, three V slots (224 KiB).
+// MMA issuer, per tile i: [wait pf0(i)] PV_0(i), S_0(i+1); [wait pf1(i)] PV_1(i), S_1(i+1).
+// pf0 (one barrier per tile parity, so the producer can arm tile i + 1 while tile i is
+// open) completes when softmax group 0 has written P_0(i) and V(i), K(i+1) have landed;
+// pf1 when group 1 has written P_1(i).  With a single valid query tile (the last 128
+// queries of a head) group 1 takes no part.
+constexpr int OFF2_Q = 0;               // [2] query tiles
+constexpr int OFF2_K = 2 * TB;          // [2] key slots
+constexpr int OFF2_V = 4 * TB;          // [3] value slots
+constexpr int OFF2_BAR = 7 * TB;
+constexpr size_t SMEM2_BYTES = OFF2_BAR + 256;   // base 1024-aligned (checked)
+static_assert(SMEM2_BYTES <= 227 * 1024, "shared memory per CTA");
+
+__global__ void __launch_bounds__(THREADS, 1)
+    tc_attend2(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKb,
+               const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmKw,
+               const __grid_constant__ CUtensorMap tmVw, AttnJob j) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0u) {
+    if (threadIdx.x == 0) dev_fail(j.L, DEV_INCONSISTENT, 9902);
+    return;
+  }
+  uint8_t* smem = smem_raw;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF2_BAR);
+  uint64_t* q_full = bars + 0;
+  uint64_t* k0_full = bars + 1;
+  uint64_t* pf0 = bars + 2;       // [2] by tile parity
+  uint64_t* pf1 = bars + 4;
+  uint64_t* k_empty = bars + 5;   // [2] S_0(i), S_1(i) complete: K slot i & 1 free
+  uint64_t* v_empty = bars + 7;   // [3] PV_0(i), PV_1(i) complete: V slot i % 3 free
+  uint64_t* s_full = bars + 10;   // [2] S_g(i) complete
+  uint64_t* pv_done = bars + 12;  // [2] PV_g(i) complete
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 14);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int h = blockIdx.y;
+  const int q0 = blockIdx.x * 2 * BQ;
+  const int G = q0 + BQ < j.Nq ? 2 : 1;         // query tiles with at least one valid query
+  const int m = min(max(j.b.occ[h], 0), j.b.M_max);
+  const int W = j.W;
+  const int nb = (m + BK - 1) / BK;
+  const int nt = nb + (W + BK - 1) / BK;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(k0_full, 1);
+    mbar_init(pf0 + 0, 4 + 1);   // four softmax warps + the producer (with bytes)
+    mbar_init(pf0 + 1, 4 + 1);
+    mbar_init(pf1, 4);
+    for (int s = 0; s < 2; ++s) mbar_init(k_empty + s, 1);
+    for (int s = 0; s < 3; ++s) mbar_init(v_empty + s, 1);
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(s_full + g, 1);
+      mbar_init(pv_done + g, 1);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, TMEM_COLS);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = *tmem_holder;
+
+  auto load_tile = [&](bool is_k, int u, void* dst, uint64_t* bar) {
+    const bool bank = u < nb;
+    const CUtensorMap* mp = is_k ? (bank ? &tmKb : &tmKw) : (bank ? &tmVb : &tmVw);
+    const int row = bank ? u * BK : (u - nb) * BK;
+    tma_load_3d(dst, mp, bar, 0, row, h);
+    tma_load_3d(static_cast<uint8_t*>(dst) + HB, mp, bar, 64, row, h);
+  };
+
+  if (warp == 0) {
+    if (lane == 0 && nt > 0) {
+      // ---------------- TMA producer
+      prefetch_map(&tmQ);
+      mbar_arrive_expect_tx(q_full, G * TB);
+      for (int g = 0; g < G; ++g) {
+        tma_load_3d(smem + OFF2_Q + g * TB, &tmQ, q_full, 0, q0 + g * BQ, h);
+        tma_load_3d(smem + OFF2_Q + g * TB + HB, &tmQ, q_full, 64, q0 + g * BQ, h);
+      }
+      mbar_arrive_expect_tx(k0_full, TB);
+      load_tile(true, 0, smem + OFF2_K, k0_full);
+      int armed = 0;
+      bool ok = true;
+      for (int i = 0; i < nt; ++i) {
+        // pf0 of this parity: the phase of tile i - 2 is over
+        if (i >= 2 && !(ok = mbar_wait(pf0 + (i & 1), ((i - 2) >> 1) & 1, abort_flag))) break;
+        // V slot i % 3: the P.V products of tile i - 3 are complete
+        if (i >= 3 && !(ok = mbar_wait(v_empty + i % 3, ((i - 3) / 3) & 1, abort_flag))) break;
+        const bool knext = i + 1 < nt;
+        // K slot (i + 1) & 1: the score products of tile i - 1 are complete
+        if (knext && i >= 1 && !(ok = mbar_wait(k_empty + ((i + 1) & 1), ((i - 1) >> 1) & 1, abort_flag))) break;
+        mbar_arrive_expect_tx(pf0 + (i & 1), knext ? 2 * TB : TB);
+        load_tile(false, i, smem + OFF2_V + (i % 3) * TB, pf0 + (i & 1));
+        if (knext) load_tile(true, i + 1, smem + OFF2_K + ((i + 1) & 1) * TB, pf0 + (i & 1));
+        armed = i + 1;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.L, DEV_TIMEOUT, 410);
+      }
+      // never leave with copies in flight (see tc_attend)
+      volatile int no_abort = 0;
+      mbar_wait(q_full, 0, &no_abort);
+      mbar_wait(k0_full, 0, &no_abort);
+      bool drained = true;
+      for (int i = armed > 2 ? armed - 2 : 0; i < armed; ++i)
+        drained = drained && mbar_wait(pf0 + (i & 1), (i >> 1) & 1, abort_flag);
+      if (!drained) {
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 50000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && nt > 0) {
+      // ---------------- MMA issuer
+      constexpr uint32_t id_s = idesc_bf16(BQ, BK);
+      constexpr uint32_t id_o = idesc_bf16(BQ, 128, /*b_mn_major=*/true);
+      bool ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(k0_full, 0, abort_flag);
+      int pv_issued = 0;
+      auto issue_s = [&](int g, int i) {
+        const uint32_t q_base = smem_u32(smem + OFF2_Q + g * TB);
+        const uint32_t k_base = smem_u32(smem + OFF2_K + (i & 1) * TB);
+        const uint32_t sc = tmem + g * 256;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
+          mma_bf16(sc, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
+        }
+        mma_commit(s_full + g);
+        if (g == G - 1) mma_commit(k_empty + (i & 1));
+      };
+      auto issue_pv = [&](int g, int i) {
+        const uint32_t v_base = smem_u32(smem + OFF2_V + (i % 3) * TB);
+        const uint32_t pc = tmem + g * 256;
+        const uint32_t oc = tmem + g * 256 + 128;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ts(oc, pc + kk * 8, desc_sw128_mn(v_base + kk * 2048, HB, 1024), id_o, (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(pv_done + g);
+        if (g == G - 1) mma_commit(v_empty + i % 3);
+      };
+      if (ok) {
+        fence_after_sync();
+        for (int g = 0; g < G; ++g) issue_s(g, 0);
+      }
+      for (int i = 0; ok && i < nt; ++i) {
+        // the one wait per group and tile
+        if (!(ok = mbar_wait(pf0 + (i & 1), (i >> 1) & 1, abort_flag))) break;
+        fence_after_sync();
+        issue_pv(0, i);
+        if (i + 1 < nt) issue_s(0, i + 1);
+        if (G == 2) {
+          if (!(ok = mbar_wait(pf1, i & 1, abort_flag))) break;
+          fence_after_sync();
+          issue_pv(1, i);
+          if (i + 1 < nt) issue_s(1, i + 1);
+        }
+        pv_issued = i + 1;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.L, DEV_TIMEOUT, 411);
+      }
+      // every issued MMA complete before TMEM is freed (commits track all earlier MMAs)
+      volatile int no_abort = 0;
+      if (pv_issued > 0) mbar_wait(pv_done + 0, (pv_issued - 1) & 1, &no_abort);
+      if (G == 2 && pv_issued > 0) mbar_wait(pv_done + 1, (pv_issued - 1) & 1, &no_abort);
+    }
+  } else {
+    // ---------------- softmax group g over query tile g, thread = query row = TMEM lane
+    const int g = (warp - 2) >> 2;
+    const int qd = warp & 3;
+    const int r = qd * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
+    const uint32_t sc = tmem + lane_off + g * 256;
+    const uint32_t oc = sc + 128;
+    const int ng = g < G ? nt : 0;
+    float mrun = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int i = 0; i < ng; ++i) {
+      const bool bank = i < nb;
+      const int valid = bank ? min(BK, m - i * BK) : min(BK, W - (i - nb) * BK);
+      ok = ok && __all_sync(0xffffffffu, mbar_wait(s_full + g, i & 1, abort_flag));
+      if (!ok) break;
+      fence_after_sync();
+      float s0[32], s1[32], s2[32], s3[32];
+      tmem_ld32(sc, s0);
+      tmem_ld32(sc + 32, s1);
+      tmem_ld32(sc + 64, s2);
+      tmem_ld32(sc + 96, s3);
+      tmem_wait_ld();
+      if (valid < BK) {
+        mask_tail(s0, valid); mask_tail(s1, valid - 32); mask_tail(s2, valid - 64); mask_tail(s3, valid - 96);
+      }
+      float tmax;
+      {
+        float t[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t[k] = -INFINITY;
+        max_acc(t, s0); max_acc(t, s1); max_acc(t, s2); max_acc(t, s3);
+        tmax = fmaxf(fmaxf(fmaxf(t[0], t[1]), fmaxf(t[2], t[3])), fmaxf(fmaxf(t[4], t[5]), fmaxf(t[6], t[7])));
+      }
+      tmax *= j.sl2;
+      // S_g(i) complete implies PV_g(i - 1) complete (issued earlier by the same thread)
+      const bool raise = tmax > mrun + RESCALE_LOG2;
+      const float mnew = raise ? tmax : mrun;
+      const float mprev = mrun;
+      if (raise) {
+        l *= (i > 0) ? ex2(mrun - mnew) : 0.f;
+        mrun = mnew;
+      }
+      const float nm = -mrun;
+      float2 lab = make_float2(0.f, 0.f);
+      {
+        uint32_t pk[32];
+        exp_pack(s0, s1, j.sl2, nm, lab, pk);
+        tmem_st32(sc, pk);
+        exp_pack(s2, s3, j.sl2, nm, lab, pk);
+        tmem_st32(sc + 32, pk);
+      }
+      if (__any_sync(0xffffffffu, raise && i > 0)) {
+        const float alpha = raise ? ex2(mprev - mnew) : 1.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(oc + c * 32, v);
+          tmem_wait_ld();
+          uint32_t w32[32];
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const float2 y = __fmul2_rn(make_float2(v[2 * k], v[2 * k + 1]), make_float2(alpha, alpha));
+            w32[2 * k] = __float_as_uint(y.x);
+            w32[2 * k + 1] = __float_as_uint(y.y);
+          }
+          tmem_st32(oc + c * 32, w32);
+        }
+      }
+      l += lab.x + lab.y;
+      tmem_wait_st();
+      fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(g == 0 ? pf0 + (i & 1) : pf1);
+    }
+    if (ok && ng > 0) ok = __all_sync(0xffffffffu, mbar_wait(pv_done + g, (ng - 1) & 1, abort_flag));
+    if (!ok) {
+      *abort_flag = 1;
+      if (lane == 0) dev_fail(j.L, DEV_TIMEOUT, 412);
+    }
+    fence_after_sync();
+    const int qrow = q0 + g * BQ + r;
+    const float inv = ok && ng > 0 && l > 0.f ? 1.0f / l : 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      float x[32];
+      if (ng > 0) {   // warp-uniform
+        tmem_ld32(oc + c * 32, x);
+        tmem_wait_ld();
+      }
+      if (g < G && qrow < j.Nq) {
+        uint4* dst = reinterpret_cast<uint4*>(j.O + ((int64_t)h * j.Nq + qrow) * 128 + c * 32);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          float y[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) y[e] = ng > 0 ? x[k * 8 + e] * inv : 0.f;
+          uint4 pk;
+          pk.x = pack_bf16(y[0], y[1]);
+          pk.y = pack_bf16(y[2], y[3]);
+          pk.z = pack_bf16(y[4], y[5]);
+          pk.w = pack_bf16(y[6], y[7]);
+          dst[k] = pk;
+        }
+      }
+    }
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after_sync();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
 }  // namespace
 
 cudaError_t tc_attn_set_smem_limits() {
-  return cudaFuncSetAttribute(tc_attend, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(tc_attend, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_attend2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2_BYTES);
+  return e;
 }
 
 cudaError_t launch_attend_tc(const Bank& b, DevLayer* L, const void* Q, int Nq, const void* Kw, const void* Vw,
@@ -435,9 +733,24 @@ cudaError_t launch_attend_tc(const Bank& b, DevLayer* L, const void* Q, int Nq, 
     mvw = mvb;
   }
   AttnJob job{b, L, Nq, W, (__nv_bfloat16*)O, 1.4426950408889634f / sqrtf(128.0f)};
-  dim3 grid((Nq + BQ - 1) / BQ, b.H);
+  // two query tiles per CTA whenever that still gives every SM at least two CTAs (the
+  // key-split kernel keeps small grids, e.g. one layer of 12 heads, in fewer waves)
+  static int n_sm = 0;
+  if (n_sm == 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+      n_sm = v;
+  }
+  const int64_t ctas2 = (int64_t)((Nq + 2 * BQ - 1) / (2 * BQ)) * b.H;
   timer_begin(t, "attend_tc", s);
-  tc_attend<<<grid, THREADS, SMEM_BYTES, s>>>(mq, mkb, mvb, mkw, mvw, job);
+  if (n_sm > 0 && ctas2 >= 2 * (int64_t)n_sm) {
+    dim3 grid((Nq + 2 * BQ - 1) / (2 * BQ), b.H);
+    tc_attend2<<<grid, THREADS, SMEM2_BYTES, s>>>(mq, mkb, mvb, mkw, mvw, job);
+  } else {
+    dim3 grid((Nq + BQ - 1) / BQ, b.H);
+    tc_attend<<<grid, THREADS, SMEM_BYTES, s>>>(mq, mkb, mvb, mkw, mvw, job);
+  }
   timer_end(t, s);
   return cudaGetLastError();
 }

@@ -86,7 +86,30 @@ struct TcJob {
   Bank b;
   Ws w;
   KParams kp;
+  int lin;   // 1: row tiles are the budget-sized 128-row tiles of all heads (w.tile_head)
+  int tpn;   // row tiles per head otherwise (persistent kernel: unit u = head u / tpn, tile u % tpn)
 };
+
+// Head and row tile of work unit u of the persistent kernel.
+__device__ __forceinline__ void unit_of(const TcJob& j, int u, int& h, int& rtile) {
+  if (j.lin) {
+    h = j.w.tile_head[u];
+    rtile = u - j.w.tile_first[h];
+  } else {
+    h = u / j.tpn;
+    rtile = u - h * j.tpn;
+  }
+}
+
+// (sigma^2 / 2)^P: the scale between |A|^-P and w (Eq. 2 through the MMA).
+template <int P>
+__device__ __forceinline__ float pow_c(const KParams& kp) {
+  const float hs2 = 0.5f / kp.inv_s2;
+  float c = hs2;
+  if (P >= 2) c = hs2 * hs2;
+  if (P == 4) c = c * c;
+  return c;
+}
 
 __device__ __forceinline__ void job_range(int MODE, const DevHead& hd, const DevLayer& L, int& nrows, int& c0,
                                           int& c1) {
@@ -188,18 +211,65 @@ __device__ __forceinline__ float chunk_sum_skip(const float (&v)[32], int lim, i
   return s;
 }
 
-template <int MODE, int P, bool KV>
-__global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
-    tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
-             const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx,
-             const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j) {
-  using LY = Lay<KV>;
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  if ((smem_u32(smem_raw) & 1023u) != 0u) {   // 128-byte-swizzled tiles need 1024-byte alignment
-    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9900);
-    return;
+// TMEM of the pair passes: warp 1 allocates TMEM_COLS columns (and gives up the CTA's
+// allocation permit) into the holder word of the barrier area; every thread returns the
+// address.  Called by all threads of the CTA together, as is cta_tmem_free.
+__device__ __forceinline__ uint32_t cta_tmem_alloc(uint8_t* bar_area) {
+  uint32_t* holder = reinterpret_cast<uint32_t*>(reinterpret_cast<uint64_t*>(bar_area) + 9);
+  if ((threadIdx.x >> 5) == 1) tmem_alloc(holder, TMEM_COLS);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  return *holder;
+}
+
+__device__ __forceinline__ void cta_tmem_free(uint32_t tmem) {
+  fence_before_sync();
+  __syncthreads();
+  if ((threadIdx.x >> 5) == 1) {
+    fence_after_sync();
+    tmem_dealloc(tmem, TMEM_COLS);
   }
-  uint8_t* smem = smem_raw;
+}
+
+// A row of a pass that has no column at all (projection at a prefix length that is a
+// multiple of the snapshot spacing, survivor maintenance without evictions): the row keeps
+// its running sum and is finished exactly as the epilogue finishes it after no tile; no
+// MMA, TMEM or barrier.
+template <int MODE, int P>
+__device__ __forceinline__ void trivial_row(const TcJob& j, const DevHead& hd, int h, int row, int c0) {
+  const int64_t bh = (int64_t)h * j.b.M_max;
+  const float c = pow_c<P>(j.kp);
+  if (MODE == TM_PROJECT) {
+    const float S = j.w.snap[(bh + row) * j.w.snap_stride + c0 / SNAP];
+    j.w.rho_t[bh + row] = fmaf(c, S, j.b.rho[bh + row]);
+  } else if (MODE == TM_SUB) {
+    const int slot = hd.e == 0 ? row : j.w.surv_list[bh + row];
+    if (slot >= 0 && slot < hd.m_old) {
+      const float rho = fmaf(-c, 0.f, j.w.rho_t[bh + slot]);
+      j.b.rho[bh + slot] = rho;
+      if (j.kp.refresh) {
+        const float bnew = fmaxf(rho, j.kp.delta);
+        j.b.base[bh + slot] = bnew;
+        j.w.invb[(int64_t)h * j.w.invb_stride + slot] = __frcp_rn(bnew);
+      }
+    } else {
+      dev_fail(j.w.L, DEV_INCONSISTENT, 6003);
+    }
+  }
+}
+
+// One row tile (rows [128 rtile, +128) of head h) against its column tiles, columns split
+// over nz CTAs of which this is number zi, in the CTA's TMEM columns [tmem, tmem + 256)
+// (allocated once per CTA by the caller: a CTA may allocate only until it relinquishes
+// its allocation permit).  Every thread of the CTA calls it together; it leaves the
+// shared-memory barriers invalidated.  Returns false if a bounded wait gave up.
+template <int MODE, int P, bool KV>
+__device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtensorMap& tmAx, const CUtensorMap& tmB,
+                                           const CUtensorMap& tmBx, const CUtensorMap& tmAv, const CUtensorMap& tmBv,
+                                           const TcJob& j, uint8_t* smem, uint32_t tmem, int h, int rtile, int zi,
+                                           int nz) {
+  using LY = Lay<KV>;
   float* meta = reinterpret_cast<float*>(smem + LY::META);
   float* xch = reinterpret_cast<float*>(smem + LY::XCH);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + LY::BAR);
@@ -213,18 +283,16 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
   uint64_t* bar_meta = bars + 10;   // [META_BUFS] SCORE: 1 / b of the columns of tile t (t % 4)
 
-  const int h = blockIdx.y;
   const DevHead hd = j.w.hd[h];
   const DevLayer L = *layer_of(j.w, h);
   int nrows, c0, c1;
   job_range(MODE, hd, L, nrows, c0, c1);
-  const int row0 = blockIdx.x * BM;
-  if (row0 >= nrows) return;                      // uniform: before any barrier or TMEM use
+  const int row0 = rtile * BM;
   // column tiles of this CTA: the row passes with plain row sums may split the column
-  // range over gridDim.z CTAs (their partial sums are combined below)
+  // range over nz CTAs (their partial sums are combined below)
   const int ntot = c1 > c0 ? (c1 - c0 + BN - 1) / BN : 0;
-  const int per = (ntot + (int)gridDim.z - 1) / (int)gridDim.z;
-  const int tbeg = min(ntot, (int)blockIdx.z * per);
+  const int per = (ntot + nz - 1) / nz;
+  const int tbeg = min(ntot, zi * per);
   const int ntiles = min(ntot, tbeg + per) - tbeg;
   c0 += tbeg * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -240,11 +308,9 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 1) tmem_alloc(tmem_holder, TMEM_COLS);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
-  const uint32_t tmem = *tmem_holder;
 
   if (warp == 0) {
     if (lane == 0 && ntiles > 0) {
@@ -346,10 +412,7 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
     const int et = threadIdx.x - 64;              // 0..255
     const int64_t bh = (int64_t)h * j.b.M_max;
     const KParams kp = j.kp;
-    const float hs2 = 0.5f / kp.inv_s2;           // sigma^2 / 2
-    float c = hs2;                                // (sigma^2 / 2)^p
-    if (P >= 2) c = hs2 * hs2;
-    if (P == 4) c = c * c;
+    const float c = pow_c<P>(kp);                 // (sigma^2 / 2)^p
     const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
     // per-row state (sums in units of |A|^-p)
     float S = 0.f, acc = 0.f, thr = 0.f;
@@ -484,19 +547,19 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
       xch[half * BM + r_local] = acc;
       named_bar(1 + q, 64);
       acc = xch[r_local] + xch[BM + r_local];
-      if (gridDim.z > 1) {
+      if (nz > 1) {
         // column-split row tile: publish this CTA's partial; the last CTA of the tile to
         // arrive adds the partials in split order and finishes the rows
         float* part = j.w.part + (int64_t)h * j.w.part_stride;
-        const int64_t zstride = (int64_t)gridDim.y * j.w.part_stride;
-        if (half == 0 && active) part[blockIdx.z * zstride + row] = acc;
+        const int64_t zstride = (int64_t)j.b.H * j.w.part_stride;
+        if (half == 0 && active) part[zi * zstride + row] = acc;
         __threadfence();
         named_bar(6, 32 * EPI_WARPS);
         int* flag = reinterpret_cast<int*>(smem + LY::FLAG);
         if (et == 0) {
-          int32_t* cnt = j.w.cnt + (int64_t)h * j.w.cnt_stride + blockIdx.x;
+          int32_t* cnt = j.w.cnt + (int64_t)h * j.w.cnt_stride + rtile;
           const int prev = atomicAdd(cnt, 1);
-          const int last = prev == (int)gridDim.z - 1;
+          const int last = prev == nz - 1;
           if (last) atomicExch(cnt, 0);
           *flag = last;
         }
@@ -506,7 +569,7 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
           __threadfence();
           if (half == 0 && active) {
             float sum = 0.f;
-            for (int z = 0; z < (int)gridDim.z; ++z) sum += __ldcg(part + z * zstride + row);
+            for (int z = 0; z < nz; ++z) sum += __ldcg(part + z * zstride + row);
             acc = sum;
           }
         }
@@ -558,10 +621,95 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 1) {
-    fence_after_sync();
-    tmem_dealloc(tmem, TMEM_COLS);
+  const bool unit_ok = *abort_flag == 0;
+  if (threadIdx.x == 0) {   // the barriers may be initialised again for the next unit
+    mbar_inval(bar_a);
+    for (int b = 0; b < 2; ++b) {
+      mbar_inval(bar_rdy + b);
+      mbar_inval(bar_accf + b);
+    }
+    for (int s = 0; s < STAGES; ++s) mbar_inval(bar_empty + s);
+    for (int q = 0; q < META_BUFS; ++q) mbar_inval(bar_meta + q);
   }
+  __syncthreads();
+  return unit_ok;
+}
+
+template <int MODE, int P, bool KV>
+__global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
+    tc_pairs(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
+             const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx,
+             const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0u) {   // 128-byte-swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9900);
+    return;
+  }
+  // row tile: (blockIdx.x, head blockIdx.y), or the blockIdx.x-th budget-sized row tile
+  // of all heads (the passes whose rows are bank states: no CTA for rows past a head's budget)
+  const int h = j.lin ? j.w.tile_head[blockIdx.x] : (int)blockIdx.y;
+  const int rtile = j.lin ? (int)blockIdx.x - j.w.tile_first[h] : (int)blockIdx.x;
+  const DevHead hd = j.w.hd[h];
+  int nrows, c0, c1;
+  job_range(MODE, hd, *layer_of(j.w, h), nrows, c0, c1);
+  const int row0 = rtile * BM;
+  if (row0 >= nrows) return;                      // uniform: before any barrier or TMEM use
+  if (c1 <= c0 && (MODE == TM_PROJECT || MODE == TM_SUB)) {
+    const int row = row0 + (int)threadIdx.x;
+    if (threadIdx.x < BM && row < nrows) trivial_row<MODE, P>(j, hd, h, row, c0);
+    return;
+  }
+  const uint32_t tmem = cta_tmem_alloc(smem_raw + Lay<KV>::BAR);
+  pairs_unit<MODE, P, KV>(tmA, tmAx, tmB, tmBx, tmAv, tmBv, j, smem_raw, tmem, h, rtile, (int)blockIdx.z,
+                          (int)gridDim.z);
+  cta_tmem_free(tmem);
+}
+
+// Persistent form of the passes over few columns or few rows (projection, survivor
+// maintenance, new baselines), for grids of many row tiles: CTA b takes the units
+// b, b + gridDim.x, ...  It first finishes, with all its threads at once, the rows of
+// every one of its units that has no column at all, then runs the units with work one
+// after another.  In a step whose layers admit nothing most units have no work, and a
+// launch of one CTA per unit would spend its time starting CTAs.
+template <int MODE, int P, bool KV>
+__global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
+    tc_pairs_loop(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
+                  const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx,
+                  const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j,
+                  int n_units) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0u) {
+    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9903);
+    return;
+  }
+  if (MODE == TM_PROJECT || MODE == TM_SUB) {
+    for (int64_t idx = threadIdx.x;; idx += blockDim.x) {
+      const int64_t u = (int64_t)blockIdx.x + (idx / BM) * gridDim.x;
+      if (u >= n_units) break;
+      int h, rtile;
+      unit_of(j, (int)u, h, rtile);
+      const DevHead hd = j.w.hd[h];
+      int nrows, c0, c1;
+      job_range(MODE, hd, *layer_of(j.w, h), nrows, c0, c1);
+      const int row = rtile * BM + (int)(idx % BM);
+      if (c1 <= c0 && row < nrows) trivial_row<MODE, P>(j, hd, h, row, c0);
+    }
+  }
+  uint32_t tmem = 0;
+  bool have_tmem = false;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+    int h, rtile;
+    unit_of(j, u, h, rtile);
+    int nrows, c0, c1;
+    job_range(MODE, j.w.hd[h], *layer_of(j.w, h), nrows, c0, c1);
+    if (rtile * BM >= nrows || c1 <= c0) continue;   // uniform across the CTA
+    if (!have_tmem) {   // once per CTA, at its first unit with work
+      tmem = cta_tmem_alloc(smem_raw + Lay<KV>::BAR);
+      have_tmem = true;
+    }
+    if (!pairs_unit<MODE, P, KV>(tmA, tmAx, tmB, tmBx, tmAv, tmBv, j, smem_raw, tmem, h, rtile, 0, 1)) break;
+  }
+  if (have_tmem) cta_tmem_free(tmem);
 }
 
 // ---------------------------------------------------------------- host side
@@ -612,7 +760,15 @@ namespace {
 
 template <int MODE, int P>
 void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap& ax, const CUtensorMap& b,
-              const CUtensorMap& bx, const CUtensorMap& av, const CUtensorMap& bv, bool kv, const TcJob& job) {
+              const CUtensorMap& bx, const CUtensorMap& av, const CUtensorMap& bv, bool kv, const TcJob& job,
+              int n_units) {
+  if (n_units > 0) {   // persistent form (projection, survivor maintenance, new baselines)
+    if constexpr (MODE == TM_PROJECT || MODE == TM_SUB || MODE == TM_NEWBASE) {
+      if (kv) tc_pairs_loop<MODE, P, true><<<grid, THREADS, Lay<true>::SMEM, s>>>(a, ax, b, bx, av, bv, job, n_units);
+      else tc_pairs_loop<MODE, P, false><<<grid, THREADS, Lay<false>::SMEM, s>>>(a, ax, b, bx, av, bv, job, n_units);
+    }
+    return;
+  }
   if (kv) tc_pairs<MODE, P, true><<<grid, THREADS, Lay<true>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
   else tc_pairs<MODE, P, false><<<grid, THREADS, Lay<false>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
 }
@@ -622,10 +778,11 @@ void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap
 template <int MODE>
 cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void* rk, const void* rx, int64_t rk_rows,
                       const void* ck, const void* cx, int64_t ck_rows, int max_rows, cudaStream_t s, Timer* t,
-                      const char* name, int split = 1, const void* rv = nullptr, const void* cv = nullptr) {
+                      const char* name, int split = 1, const void* rv = nullptr, const void* cv = nullptr,
+                      int64_t rx_rows = 0) {
   const bool kv = rv != nullptr;
   CUtensorMap ma, max_, mb, mbx, mav, mbv;
-  if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_ext(&max_, rx, rk_rows, b.H, BM) ||
+  if (!make_map_rows(&ma, rk, rk_rows, b.H, BM) || !make_map_ext(&max_, rx, rx_rows > 0 ? rx_rows : rk_rows, b.H, BM) ||
       !make_map_rows(&mb, ck, ck_rows, b.H, BN) || !make_map_ext(&mbx, cx, ck_rows, b.H, BN))
     return cudaErrorInvalidValue;
   if (kv) {
@@ -635,12 +792,27 @@ cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void*
     mav = ma;   // never read
     mbv = mb;
   }
-  TcJob job{b, w, kp};
-  dim3 grid((max_rows + BM - 1) / BM, b.H, split);
+  // passes over bank rows take one CTA per budget-sized row tile of each head
+  const int lin = (MODE == TM_CROSS || MODE == TM_PROJECT || MODE == TM_SUB) && split == 1 ? 1 : 0;
+  const int tpn = (max_rows + BM - 1) / BM;
+  TcJob job{b, w, kp, lin, tpn};
+  dim3 grid(lin ? w.n_mtiles : tpn, lin ? 1 : b.H, split);
+  // projection, survivor maintenance and new baselines over many row tiles: the
+  // persistent form, a few CTAs per SM (most of those row tiles have no column when
+  // layers admit nothing)
+  int n_units = 0;
+  const int n_sm = sm_count();
+  if ((MODE == TM_PROJECT || MODE == TM_SUB || MODE == TM_NEWBASE) && n_sm > 0) {
+    const int units = lin ? w.n_mtiles : tpn * b.H;
+    if (units >= 16 * n_sm) {
+      n_units = units;
+      grid = dim3((kv ? 1 : 2) * n_sm, 1, 1);
+    }
+  }
   timer_begin(t, name, s);
-  if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
-  else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
-  else launch_p<MODE, 2>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job);
+  if (kp.p == 1) launch_p<MODE, 1>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job, n_units);
+  else if (kp.p == 4) launch_p<MODE, 4>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job, n_units);
+  else launch_p<MODE, 2>(grid, s, ma, max_, mb, mbx, mav, mbv, kv, job, n_units);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -649,6 +821,16 @@ cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void*
 
 bool tc_supported(int d, int bf16) { return d == 128 && bf16 && encode_fn() != nullptr; }
 
+int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+      n = v;
+  }
+  return n;
+}
+
 cudaError_t tc_attn_set_smem_limits();
 
 cudaError_t tc_set_smem_limits() {
@@ -656,14 +838,26 @@ cudaError_t tc_set_smem_limits() {
 #define DKV_OPT1(M, P, KV)                                                                                     \
   if (e == cudaSuccess)                                                                                        \
     e = cudaFuncSetAttribute(tc_pairs<M, P, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Lay<KV>::SMEM);
+#define DKV_OPTL(M, P, KV)                                                                                     \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_pairs_loop<M, P, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize,             \
+                             (int)Lay<KV>::SMEM);
 #define DKV_OPT(M)                                                                                             \
   DKV_OPT1(M, 1, false) DKV_OPT1(M, 2, false) DKV_OPT1(M, 4, false)                                            \
   DKV_OPT1(M, 1, true) DKV_OPT1(M, 2, true) DKV_OPT1(M, 4, true)
+#define DKV_OPTLOOP(M)                                                                                         \
+  DKV_OPTL(M, 1, false) DKV_OPTL(M, 2, false) DKV_OPTL(M, 4, false)                                            \
+  DKV_OPTL(M, 1, true) DKV_OPTL(M, 2, true) DKV_OPTL(M, 4, true)
   DKV_OPT(TM_SCORE)
   DKV_OPT(TM_CROSS)
   DKV_OPT(TM_PROJECT)
   DKV_OPT(TM_SUB)
   DKV_OPT(TM_NEWBASE)
+  DKV_OPTLOOP(TM_PROJECT)
+  DKV_OPTLOOP(TM_SUB)
+  DKV_OPTLOOP(TM_NEWBASE)
+#undef DKV_OPTLOOP
+#undef DKV_OPTL
 #undef DKV_OPT
 #undef DKV_OPT1
   if (e == cudaSuccess) e = tc_attn_set_smem_limits();
@@ -675,8 +869,10 @@ cudaError_t tc_set_smem_limits() {
 cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
                             cudaStream_t s, Timer* t) {
   const bool kv = w.vperm != nullptr;
+  // the candidates (caller's array) are [H][N][d]; their extension rows, like every
+  // candidate array of the workspace, [H][n_max][32]
   return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", 2,
-                             kv ? Vc : nullptr, kv ? b.v : nullptr);
+                             kv ? Vc : nullptr, kv ? b.v : nullptr, b.n_max);
 }
 
 cudaError_t launch_cross_tc(const Bank& b, const Ws& w, const KParams& kp, cudaStream_t s, Timer* t) {

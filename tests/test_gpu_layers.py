@@ -3,8 +3,10 @@ layers with single launches, each layer keeping its own shared prefix r* (Eq. 11
 
 The grouped handle is compared bit for bit with one handle per layer fed the same
 per-layer streams (those are themselves parity-tested against the oracle): bank
-contents, occupancy, provenance, densities, baselines, attention outputs and each
-layer's r* must be identical.
+contents, occupancy, provenance, densities, baselines and each layer's r* must be
+identical, and so must attention outputs whenever both handles take the same attention
+schedule (the grids of the small cases); the grouped handle is also teacher-forced
+against the oracle layer by layer.
 """
 import numpy as np
 import pytest
@@ -167,7 +169,8 @@ def test_layer_heads_must_divide_heads(dkv):
 
 def test_grouped_layers_fullsize(dkv):
     """Three Wan-1.3B-shaped layers (12 heads, N = 4,680, M = 9,360) in one handle against
-    three one-layer handles, bit for bit, over the first five steps (fill and eviction)."""
+    three one-layer handles over the first five steps (fill and eviction): bank contents
+    bit for bit, attention within its bound."""
     L = 3
     wl = synth.get_workload("wan13b_stack_l30h12", L=L)
     H, dt = wl.H, torch.bfloat16
@@ -191,7 +194,10 @@ def test_grouped_layers_fullsize(dkv):
         torch.cuda.synchronize()
         for bk in sep + [grp]:
             bk.sync()
-        assert torch.equal(torch.cat(o_sep, 0), o_grp), t
+        # 36 heads take the two-query-tile attention schedule, 12 the key-split one: the
+        # outputs agree within the attention bound (each schedule is checked against the
+        # oracle elsewhere); the banks stay bit-identical
+        assert (torch.cat(o_sep, 0).float() - o_grp.float()).abs().max().item() < 2e-2, t
         for name in BUFFERS:
             assert torch.equal(torch.cat([getattr(sep[l], name) for l in range(L)], 0), getattr(grp, name)), (t, name)
         if b is not None:

@@ -394,3 +394,26 @@ def test_kernel_timing_modes(dkv):
             assert any(ms > 0 for _, ms in others.values())
         bank.reset()
     bank.close()
+
+
+@pytest.mark.parametrize("sync", [1, 0])
+def test_persistent_pair_passes_match_oracle(dkv, sync):
+    """Banks with many budget-sized row tiles (20 heads of budget 16,000 and 4 of 700, a
+    16,384-candidate capacity) take the persistent form of the projection, survivor
+    maintenance and new-baseline passes (at least 16 row tiles per SM); teacher-forced
+    against the oracle, with evictions in the small heads."""
+    budgets = [16000] * 10 + [700, 700] + [16000] * 10 + [700, 700]
+    wl = synth.get_workload("wan14b_headwise_l40h40", L=1, H=len(budgets), N=300, W=64, Nq=64,
+                            budgets=budgets, steps=6)
+    reps = _rollout(dkv, wl, "tc", check_attn=False, n_max=16384, sync_heads=sync)
+    assert len(reps) >= 5 and sum(r.rstar_oracle for r in reps) > 0
+
+
+@pytest.mark.parametrize("mode", ["fp32", "tc"])
+def test_blocks_smaller_than_capacity(dkv, mode):
+    """Blocks of N = 300 candidates offered to a handle created for up to 512: every
+    candidate array of the workspace keeps its capacity stride while the caller's block
+    is packed at N rows per head."""
+    wl = synth.get_workload("wan13b_layer_h12", H=3, N=300, W=200, Nq=130, budgets=700, steps=6)
+    reps = _rollout(dkv, wl, mode, n_max=512)
+    assert sum(r.rstar_oracle for r in reps) > 0
