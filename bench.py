@@ -1,27 +1,32 @@
 #!/usr/bin/env python3
 """Benchmark of the DensityKV hot path on GB300: bank update + bank-reading attention.
 
-One step = one rollout step of one layer (all H heads): attention of the current
-block's queries over [bank | window], then admit + compress of the block leaving
-the window (Sec. 3.4, Alg. 1), all through the C ABI (libdkv.so).
+Default workload: the Wan-14B-shaped stack (40 layers x 40 heads, d = 128, bf16,
+4,680-token blocks, per-head budgets drawn from {2,340, 4,680, 9,360, 18,720}, window =
+previous block, 4,680 queries).  One step = one generated block through the whole
+model: in every layer, attention of the block's queries over [bank | window], then
+admit, evict and commit of the block leaving the window (Sec. 3.4, Alg. 1 per layer,
+each layer with its own prefix r*, Eq. 11), all through one handle of the C ABI
+(libdkv.so) whose calls are single launches over all 1,600 heads.  Every layer and head
+draws its own synthetic stream (synth.device, generated on the GPU before each step's
+start event).  W warm-up steps start from empty banks; K steps are timed one by one with
+CUDA events on the launching stream, a 256 MiB buffer written between them.
 
-Default workload: the Wan-1.3B-shaped single layer (12 heads, d = 128, bf16,
-4,680-token blocks, 9,360-token bank, window = previous block, 4,680 queries),
-synthetic clustered keys from ``synth``.  W warm-up steps start from an empty bank
-(the first two fill it, eviction starts at the third), then K steps are timed one
-by one with CUDA events on the launching stream; a 256 MiB buffer is written
-between timed steps to flush the 129 MB L2.
+Metric: bank keys scored per second = sum over heads of (m_h + N) per update (every
+bank key's projected growth and every candidate are scored) / step time; blocks/s =
+model steps per second.
 
-Metric: bank keys scored per second = sum over heads of (m_h + N) per update
-(every bank key's projected growth and every candidate are scored) / step time.
+A one-layer workload (--workload wan13b_layer_h12 and the like) runs the single-layer
+step with its ablation flags (policies, descriptor, RoPE re-zeroing, sequential
+admission, repeated attention passes), CUDA graphs and the numpy input generator.
 
-``--impl reference`` times the CPU oracle (oracle/, numpy float64) on the host
-cores, each step a bounded sample of the same workload (one head).
+``--impl reference`` times the CPU oracle (oracle/, numpy float64) on the host cores,
+each step a bounded sample of the same workload (one head at steady state).
 
-Multi-GPU (torchrun): every rank runs an independent layer of the same shape (the
-bank update and attention are per layer and head, with no exchange), so no
-collective is on the data path; ranks meet only at the barriers around the timed
-region and in a max-reduction of the elapsed time.
+Multi-GPU (torchrun): every rank runs its own independent rollout (an independent video
+on a stack workload, an independent layer on a one-layer workload), so no collective
+is on the data path; ranks meet only at the barriers around the timed region and in a
+reduction of the elapsed time and the keys.
 """
 from __future__ import annotations
 
@@ -74,9 +79,15 @@ def parse_args():
                          "no graphs, no overlap, no e2e leg)")
     ap.add_argument("--attn-passes", type=int, default=1,
                     help="bank-reading attention passes per update (denoising passes; the update runs once)")
+    ap.add_argument("--stack", action="store_true",
+                    help="run a one-layer workload through the stack path (per-kernel roofline pass, "
+                         "device-generated inputs)")
     ap.add_argument("--layers", type=int, default=0,
                     help="stack run: number of layers (default: the workload's; fewer for small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-schedule", choices=["overlap", "serial"], default="overlap",
+                    help="stack run, end-to-end leg: copies beside the compute of the neighbouring steps, or "
+                         "each step's copies before its compute")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between steps")
@@ -219,6 +230,22 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------- helpers
+def numa_info(gpu_index: int):
+    """NUMA nodes of this host and the GPU's own node (where the pinned buffers can live)."""
+    info = {"host_nodes": None, "gpu_node": None}
+    try:
+        info["host_nodes"] = len([n for n in os.listdir("/sys/devices/system/node") if n.startswith("node")])
+        bus = subprocess.run(["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader", "-i", str(gpu_index)],
+                             capture_output=True, text=True, timeout=30).stdout.strip().lower()
+        if bus.startswith("00000000:"):
+            bus = "0000:" + bus[9:]
+        with open(f"/sys/bus/pci/devices/{bus}/numa_node") as f:
+            info["gpu_node"] = int(f.read().strip())
+    except Exception:
+        pass
+    return info
+
+
 def peaks():
     if os.path.exists(PEAKS_FILE):
         p = json.load(open(PEAKS_FILE))
@@ -1030,13 +1057,17 @@ def run_stack(args):
         in_bytes = sum(x.numel() * x.element_size() for x in hsets[0].values())
         out_bytes = out.numel() * out.element_size()
 
+        # serial schedule: the download beside the upload (both directions at once, with the
+        # GPU otherwise idle, move more bytes per second than one direction)
+        dn_s = torch.cuda.Stream(dev) if args.e2e_schedule == "serial" else pre_s
+
         def download(i, after):
-            pre_s.wait_event(after)
+            dn_s.wait_event(after)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(pre_s)
-            with torch.cuda.stream(pre_s):
+            e0.record(dn_s)
+            with torch.cuda.stream(dn_s):
                 host_outs[i % 2].copy_(douts[i % 2], non_blocking=True)
-            e1.record(pre_s)
+            e1.record(dn_s)
             return e0, e1
 
         def fill_host(t, hs_):
@@ -1067,22 +1098,28 @@ def run_stack(args):
             s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             s0.record(stream)
             ups, downs = [], []
-            if i == 0:
-                ups.append(upload(hsets[0], dsets[0], s0))
-                stream.wait_event(ups[-1][1])
+            serial = args.e2e_schedule == "serial"
+            if i == 0 or serial:   # this step's own inputs first
+                ups.append(upload(hsets[i % 2], dsets[i % 2], s0))
                 up_b += in_bytes
-            if i > 0:   # the previous step's output, beside this step's compute
+            if i > 0:   # the previous step's output
                 downs.append(download(i - 1, s0))
-            if i + 1 < K:   # then the next step's inputs
-                ups.append(upload(hsets[(i + 1) % 2], dsets[(i + 1) % 2], s0))
-                up_b += in_bytes
+            if serial:   # copies first, then the compute with the GPU to itself
+                for _, e1 in ups + downs:
+                    stream.wait_event(e1)
+            else:
+                if i == 0:
+                    stream.wait_event(ups[-1][1])
+                if i + 1 < K:   # the next step's inputs, beside this step's compute
+                    ups.append(upload(hsets[(i + 1) % 2], dsets[(i + 1) % 2], s0))
+                    up_b += in_bytes
             att_done = step(t, dsets[i % 2], stream, o=douts[i % 2])
             if i + 1 == K:   # the last step's own output
                 downs.append(download(i, att_done))
             down_b += out_bytes * len(downs)
             for _, e1 in downs:
                 stream.wait_event(e1)
-            if len(ups) and i + 1 < K:
+            if ups:
                 stream.wait_event(ups[-1][1])
             s1.record(stream)
             s1.synchronize()
@@ -1099,9 +1136,12 @@ def run_stack(args):
                "upload_ms_per_step": sum(up_ms) / K, "download_ms_per_step": sum(down_ms) / K,
                "upload_gbs": up_b / (sum(up_ms) / 1e3) / 1e9 if sum(up_ms) > 0 else None,
                "download_gbs": down_b / (sum(down_ms) / 1e3) / 1e9 if sum(down_ms) > 0 else None,
-               "copies": "pinned host buffers (one NUMA node on this host); inputs and outputs double-buffered on "
-                         "the device: the previous step's output downloads, then the next step's inputs upload, on "
-                         "one copy stream beside each step's compute; no CUDA graphs"}
+               "schedule": args.e2e_schedule, "numa": numa_info(local),
+               "copies": ("pinned host buffers (one NUMA node on this host); each step uploads its own inputs "
+                          "while the previous step's output downloads, then computes" if args.e2e_schedule == "serial"
+                          else "pinned host buffers (one NUMA node on this host); inputs and outputs double-buffered "
+                          "on the device: the previous step's output downloads, then the next step's inputs upload, "
+                          "on one copy stream beside each step's compute") + "; no CUDA graphs"}
         del hsets, dsets, douts, host_outs
 
     cpu = None
@@ -1198,7 +1238,7 @@ def main():
         print("warning: --warmup < 3 does not reach the steady state of the bank", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args)
-    elif synth_workload(args.workload).L > 1:
+    elif synth_workload(args.workload).L > 1 or args.stack:
         if args.within_block != "batch" or args.rope != "off" or args.descriptor != "k" or args.attn_passes != 1 \
                 or args.order != "score" or args.eviction != "mandatory_densest" or args.refresh_baselines:
             raise SystemExit("policy, descriptor, RoPE and sequential ablations are measured on one-layer workloads")

@@ -9,6 +9,7 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <algorithm>
 #include <vector>
 
 namespace dkv {
@@ -164,6 +165,9 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, 
   w.cnt = (int32_t*)take(Hh * cnt_stride * 4);
   w.tile_head = (int32_t*)take(Hh * ((Mm + 127) / 128) * 4);
   w.tile_first = (int32_t*)take(Hh * 4);
+  w.loop_stride = (int64_t)(Hh * std::max((Mm + 127) / 128, (Nm + 127) / 128));
+  w.loop_list = (int32_t*)take(3 * (size_t)w.loop_stride * 4);
+  w.loop_ctr = (int32_t*)take(3 * 2 * 4);
   w.part_stride = part_stride;
   w.cnt_stride = cnt_stride;
   w.invb_stride = invb_stride;

@@ -65,6 +65,11 @@ struct Ws {
   int32_t* tile_head;   // [n_mtiles] head of each 128-row tile of the heads' budgets, head-major
   int32_t* tile_first;  // [H] index of each head's first such tile
   int n_mtiles;         // sum over heads of ceil(M_h / 128)
+  int32_t* loop_list;   // [3][loop_stride] row tiles with work of the persistent projection,
+                        //   survivor and new-baseline passes (each its own: the last two run
+                        //   side by side), appended by the pass's classification kernel
+  int32_t* loop_ctr;    // [3][2] their count, and the next one to take
+  int64_t loop_stride;  // H * max(ceil(M_max / 128), ceil(n_max / 128))
   int hist_stride, snap_stride, feas_words, part_stride, cnt_stride, invb_stride, sort_stride;
   int layer_heads;      // heads per layer (the handle's heads form H / layer_heads layers)
 };

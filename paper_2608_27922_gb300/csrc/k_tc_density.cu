@@ -37,6 +37,7 @@
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
+#include <algorithm>
 #include <climits>
 #include <mutex>
 
@@ -189,6 +190,47 @@ __device__ __forceinline__ float chunk_sum_w(const float (&v)[32], const float* 
   }
   const float2 a = __fadd2_rn(a0, a1);
   return P == 1 ? -(a.x + a.y) : a.x + a.y;
+}
+
+// Score pass, one warp's 64-column half of a tile in the 16x256b layout (va: lanes
+// 0..15 of the warp's quarter, vb: lanes 16..31): this thread holds rows i/4, i/4 + 8,
+// i/4 + 16, i/4 + 24 at columns 8k + 2 (i % 4) + {0, 1}, k = 0..7, so it needs 16
+// weights for 4 rows.  acc[j] += sum of wb_c |v|^-P over row j's columns, in the
+// accumulation convention of acc2wx2 (negated for P = 1); columns from lim on are left
+// out (term by term in a partial tile).
+template <int P>
+__device__ __forceinline__ void score_rows4(const float (&va)[32], const float (&vb)[32], const float* wb, int lim,
+                                            int c2, float2 (&acc)[4]) {
+  if (lim >= 64) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 w0 = *reinterpret_cast<const float2*>(wb + 8 * k + c2);
+      const float2 w1 = *reinterpret_cast<const float2*>(wb + 8 * (k + 4) + c2);
+      acc[0] = acc2wx2<P>(make_float2(va[4 * k], va[4 * k + 1]), make_float2(va[4 * k + 16], va[4 * k + 17]), w0, w1,
+                          acc[0]);
+      acc[1] = acc2wx2<P>(make_float2(va[4 * k + 2], va[4 * k + 3]), make_float2(va[4 * k + 18], va[4 * k + 19]), w0,
+                          w1, acc[1]);
+      acc[2] = acc2wx2<P>(make_float2(vb[4 * k], vb[4 * k + 1]), make_float2(vb[4 * k + 16], vb[4 * k + 17]), w0, w1,
+                          acc[2]);
+      acc[3] = acc2wx2<P>(make_float2(vb[4 * k + 2], vb[4 * k + 3]), make_float2(vb[4 * k + 18], vb[4 * k + 19]), w0,
+                          w1, acc[3]);
+    }
+    return;
+  }
+  const float sg = P == 1 ? -1.f : 1.f;
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int c = 8 * k + c2 + e;
+      if (c < lim) {
+        const float w = sg * wb[c];
+        acc[0].x = fmaf(term1<P>(va[4 * k + e]), w, acc[0].x);
+        acc[1].x = fmaf(term1<P>(va[4 * k + 2 + e]), w, acc[1].x);
+        acc[2].x = fmaf(term1<P>(vb[4 * k + e]), w, acc[2].x);
+        acc[3].x = fmaf(term1<P>(vb[4 * k + 2 + e]), w, acc[3].x);
+      }
+    }
 }
 
 // Same over the first `lim` columns (lim < 32), term by term.
@@ -437,6 +479,9 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
       mbar_arrive(bar_rdy + 1);
     }
 
+    float2 sacc[4];   // score pass: rows lane/4 + 8 j of the quarter (16x256b layout)
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) sacc[jj] = make_float2(0.f, 0.f);
     bool ok = true;
     for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
@@ -448,7 +493,20 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
                         mbar_wait(bar_meta + t % META_BUFS, (t / META_BUFS) & 1, abort_flag));
       float tot[2] = {0.f, 0.f};
       constexpr bool kEarlyRelease = MODE == TM_SCORE || MODE == TM_SUB || MODE == TM_NEWBASE;
-      if (ok) {
+      if (ok && MODE == TM_SCORE) {
+        fence_after_sync();
+        const int cs = half * 64;
+        if (cs < nc) {   // warp-uniform
+          float va[32], vb[32];
+          tmem_ld16x256b_x8(lane_base + b * BN + cs, va);
+          tmem_ld16x256b_x8(lane_base + (16u << 16) + b * BN + cs, vb);
+          tmem_wait_ld();
+          fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile t + 2
+          score_rows4<P>(va, vb, meta + (t % META_BUFS) * BN + cs, nc - cs, 2 * (lane & 3), sacc);
+        }
+      } else if (ok) {
         fence_after_sync();
 #pragma unroll
         for (int ch = 0; ch < 2; ++ch) {
@@ -544,7 +602,18 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
     bool finalize = true;
     if (MODE == TM_SCORE || MODE == TM_SUB || MODE == TM_NEWBASE) {
       // combine the two column halves of each row (no per-tile exchange in these passes)
-      xch[half * BM + r_local] = acc;
+      if (MODE == TM_SCORE) {
+        // the four threads of a row quad hold a quarter of the half's columns each
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          float x = sacc[jj].x + sacc[jj].y;
+          x += __shfl_xor_sync(0xffffffffu, x, 1);
+          x += __shfl_xor_sync(0xffffffffu, x, 2);
+          if ((lane & 3) == 0) xch[half * BM + q * 32 + (lane >> 2) + 8 * jj] = P == 1 ? -x : x;
+        }
+      } else {
+        xch[half * BM + r_local] = acc;
+      }
       named_bar(1 + q, 64);
       acc = xch[r_local] + xch[BM + r_local];
       if (nz > 1) {
@@ -666,44 +735,71 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
 }
 
 // Persistent form of the passes over few columns or few rows (projection, survivor
-// maintenance, new baselines), for grids of many row tiles: CTA b takes the units
-// b, b + gridDim.x, ...  It first finishes, with all its threads at once, the rows of
-// every one of its units that has no column at all, then runs the units with work one
-// after another.  In a step whose layers admit nothing most units have no work, and a
-// launch of one CTA per unit would spend its time starting CTAs.
+// maintenance, new baselines), for grids of many row tiles, in two kernels.
+// pairs_classify: one thread per row of every unit (a 128-row tile of one head); the
+// rows of units without any column (projection at r* = 0 mod 128, survivor maintenance
+// without evictions) are finished there without TMEM, and every unit with work is
+// appended to w.loop_list.  tc_pairs_loop: 2 CTAs per SM take those units one at a time
+// from a counter and run the tensor pipeline on each, TMEM allocated once per CTA; the
+// units are taken as the CTAs free up, so heads of different budgets (rows of 2,340 to
+// 18,720 columns) spread evenly.  In a step whose layers admit nothing almost no unit has
+// work, and a launch of one CTA per unit would spend its time starting CTAs.
+// Work list and counters of a persistent pass (projection 0, survivors 1, new baselines 2).
+template <int MODE>
+__host__ __device__ __forceinline__ int loop_slot() {
+  return MODE == TM_PROJECT ? 0 : (MODE == TM_SUB ? 1 : 2);
+}
+
+template <int MODE, int P>
+__global__ void __launch_bounds__(256) pairs_classify(TcJob j, int n_units) {
+  int32_t* list = j.w.loop_list + loop_slot<MODE>() * j.w.loop_stride;
+  int32_t* ctr = j.w.loop_ctr + 2 * loop_slot<MODE>();
+  const int64_t total = (int64_t)n_units * BM;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int u = (int)(idx / BM), rr = (int)(idx % BM);
+    int h, rtile;
+    unit_of(j, u, h, rtile);
+    const DevHead hd = j.w.hd[h];
+    int nrows, c0, c1;
+    job_range(MODE, hd, *layer_of(j.w, h), nrows, c0, c1);
+    const int row = rtile * BM + rr;
+    if (row >= nrows) continue;
+    if (c1 > c0) {
+      if (rr == 0) list[atomicAdd(&ctr[0], 1)] = u;
+    } else if (MODE == TM_PROJECT || MODE == TM_SUB) {
+      trivial_row<MODE, P>(j, hd, h, row, c0);
+    }
+  }
+}
+
 template <int MODE, int P, bool KV>
 __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
     tc_pairs_loop(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
                   const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx,
-                  const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j,
-                  int n_units) {
+                  const __grid_constant__ CUtensorMap tmAv, const __grid_constant__ CUtensorMap tmBv, TcJob j) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if ((smem_u32(smem_raw) & 1023u) != 0u) {
     if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9903);
     return;
   }
-  if (MODE == TM_PROJECT || MODE == TM_SUB) {
-    for (int64_t idx = threadIdx.x;; idx += blockDim.x) {
-      const int64_t u = (int64_t)blockIdx.x + (idx / BM) * gridDim.x;
-      if (u >= n_units) break;
-      int h, rtile;
-      unit_of(j, (int)u, h, rtile);
-      const DevHead hd = j.w.hd[h];
-      int nrows, c0, c1;
-      job_range(MODE, hd, *layer_of(j.w, h), nrows, c0, c1);
-      const int row = rtile * BM + (int)(idx % BM);
-      if (c1 <= c0 && row < nrows) trivial_row<MODE, P>(j, hd, h, row, c0);
-    }
-  }
+  // the unit index taken by thread 0, passed through the split-tile flag word (unused
+  // by these passes)
+  volatile int* s_unit = reinterpret_cast<volatile int*>(smem_raw + Lay<KV>::FLAG);
+  const int32_t* list = j.w.loop_list + loop_slot<MODE>() * j.w.loop_stride;
+  int32_t* ctr = j.w.loop_ctr + 2 * loop_slot<MODE>();
+  const int count = __ldcg(&ctr[0]);
   uint32_t tmem = 0;
   bool have_tmem = false;
-  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+  for (;;) {
+    if (threadIdx.x == 0) *s_unit = atomicAdd(&ctr[1], 1);
+    __syncthreads();
+    const int k = *s_unit;
+    __syncthreads();   // every thread has read it before thread 0 takes the next one
+    if (k >= count) break;
     int h, rtile;
-    unit_of(j, u, h, rtile);
-    int nrows, c0, c1;
-    job_range(MODE, j.w.hd[h], *layer_of(j.w, h), nrows, c0, c1);
-    if (rtile * BM >= nrows || c1 <= c0) continue;   // uniform across the CTA
-    if (!have_tmem) {   // once per CTA, at its first unit with work
+    unit_of(j, __ldcg(&list[k]), h, rtile);
+    if (!have_tmem) {   // once per CTA, at its first unit
       tmem = cta_tmem_alloc(smem_raw + Lay<KV>::BAR);
       have_tmem = true;
     }
@@ -764,8 +860,12 @@ void launch_p(dim3 grid, cudaStream_t s, const CUtensorMap& a, const CUtensorMap
               int n_units) {
   if (n_units > 0) {   // persistent form (projection, survivor maintenance, new baselines)
     if constexpr (MODE == TM_PROJECT || MODE == TM_SUB || MODE == TM_NEWBASE) {
-      if (kv) tc_pairs_loop<MODE, P, true><<<grid, THREADS, Lay<true>::SMEM, s>>>(a, ax, b, bx, av, bv, job, n_units);
-      else tc_pairs_loop<MODE, P, false><<<grid, THREADS, Lay<false>::SMEM, s>>>(a, ax, b, bx, av, bv, job, n_units);
+      if (cudaMemsetAsync(job.w.loop_ctr + 2 * loop_slot<MODE>(), 0, 2 * sizeof(int32_t), s) != cudaSuccess) return;
+      const int64_t threads = (int64_t)n_units * BM;
+      const int cblocks = (int)std::min<int64_t>((threads + 255) / 256, (int64_t)grid.x * 8);
+      pairs_classify<MODE, P><<<cblocks, 256, 0, s>>>(job, n_units);
+      if (kv) tc_pairs_loop<MODE, P, true><<<grid, THREADS, Lay<true>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
+      else tc_pairs_loop<MODE, P, false><<<grid, THREADS, Lay<false>::SMEM, s>>>(a, ax, b, bx, av, bv, job);
     }
     return;
   }
