@@ -226,13 +226,15 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = mbar_wait(q_full, 0, abort_flag);
       int pv_issued[2] = {0, 0};
       // S_g(i): its K tile has landed (K(0): k0_full; K(i + 1): with p_full_g phase i)
+      const uint64_t qd = desc_sw128(q_base), kd0 = desc_sw128(smem_u32(smem + OFF_K));
+      const uint64_t vd0 = desc_sw128_mn(smem_u32(smem + OFF_V), HB, 1024);
       auto issue_s = [&](int g, int i) {
-        const uint32_t k_base = smem_u32(smem + OFF_K + (2 * g + (i & 1)) * TB);
+        const uint64_t kd = desc_add(kd0, (2 * g + (i & 1)) * TB);
         const uint32_t sc = tmem + g * 256;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
-          mma_bf16(sc, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
+          mma_bf16(sc, desc_add(qd, off), desc_add(kd, off), id_s, kk > 0);
         }
         mma_commit(k_empty + 2 * g + (i & 1));
         mma_commit(s_full + g);
@@ -240,12 +242,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       auto issue_pv = [&](int g, int i) -> bool {
         if (!mbar_wait(p_full + g, i & 1, abort_flag)) return false;   // the one wait
         fence_after_sync();
-        const uint32_t v_base = smem_u32(smem + OFF_V + g * TB);
+        const uint64_t vd = desc_add(vd0, g * TB);
         const uint32_t pc = tmem + g * 256;          // P: packed bf16 pairs over S columns [0, 64)
         const uint32_t oc = tmem + g * 256 + 128;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ts(oc, pc + kk * 8, desc_sw128_mn(v_base + kk * 2048, HB, 1024), id_o, (i > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(oc, pc + kk * 8, desc_add(vd, kk * 2048), id_o, (i > 0 || kk > 0) ? 1u : 0u);
         mma_commit(v_empty + g);
         mma_commit(pv_done + g);
         pv_issued[g] = i + 1;
@@ -547,25 +549,30 @@ __global__ void __launch_bounds__(THREADS, 1)
       constexpr uint32_t id_o = idesc_bf16(BQ, 128, /*b_mn_major=*/true);
       bool ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(k0_full, 0, abort_flag);
       int pv_issued = 0;
+      // every operand's descriptor once; the k-steps' by one add each (desc_add): the
+      // issuing thread's time per MMA is what paces the tensor pipe here
+      const uint64_t qd0 = desc_sw128(smem_u32(smem + OFF2_Q)), qd1 = desc_sw128(smem_u32(smem + OFF2_Q + TB));
+      const uint64_t kd0 = desc_sw128(smem_u32(smem + OFF2_K));
+      const uint64_t vd0 = desc_sw128_mn(smem_u32(smem + OFF2_V), HB, 1024);
       auto issue_s = [&](int g, int i) {
-        const uint32_t q_base = smem_u32(smem + OFF2_Q + g * TB);
-        const uint32_t k_base = smem_u32(smem + OFF2_K + (i & 1) * TB);
+        const uint64_t qd = g ? qd1 : qd0;
+        const uint64_t kd = desc_add(kd0, (i & 1) * TB);
         const uint32_t sc = tmem + g * 256;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * HB + (kk & 3) * 32;
-          mma_bf16(sc, desc_sw128(q_base + off), desc_sw128(k_base + off), id_s, kk > 0);
+          mma_bf16(sc, desc_add(qd, off), desc_add(kd, off), id_s, kk > 0);
         }
         mma_commit(s_full + g);
         if (g == G - 1) mma_commit(k_empty + (i & 1));
       };
       auto issue_pv = [&](int g, int i) {
-        const uint32_t v_base = smem_u32(smem + OFF2_V + (i % 3) * TB);
+        const uint64_t vd = desc_add(vd0, (i % 3) * TB);
         const uint32_t pc = tmem + g * 256;
         const uint32_t oc = tmem + g * 256 + 128;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ts(oc, pc + kk * 8, desc_sw128_mn(v_base + kk * 2048, HB, 1024), id_o, (i > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(oc, pc + kk * 8, desc_add(vd, kk * 2048), id_o, (i > 0 || kk > 0) ? 1u : 0u);
         mma_commit(pv_done + g);
         if (g == G - 1) mma_commit(v_empty + i % 3);
       };

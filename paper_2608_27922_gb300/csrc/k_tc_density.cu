@@ -412,8 +412,11 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
       // ---------------- MMA issuer: 8 k-steps per key (16 per [key; value]) + 1 of the extension
       constexpr uint32_t idesc = idesc_bf16(BM, BN);
       bool ok = mbar_wait(bar_a, 0, abort_flag);
-      const uint32_t a_base = smem_u32(smem + LY::A);
-      const uint32_t ax_base = smem_u32(smem + LY::AX);
+      // every operand's descriptor once; the k-steps' by one add each (desc_add)
+      const uint64_t ad0 = desc_sw128(smem_u32(smem + LY::A));
+      const uint64_t axd = desc_sw32(smem_u32(smem + LY::AX));
+      const uint64_t bd0 = desc_sw128(smem_u32(smem + LY::B));
+      const uint64_t bxd0 = desc_sw32(smem_u32(smem + LY::BX));
       int done = 0;
       for (int t = 0; ok && t < ntiles; ++t) {
         const int s = t % STAGES;
@@ -421,14 +424,13 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
         // one wait per tile: every other wait in this thread stalls the tensor pipe
         if (!(ok = mbar_wait(bar_rdy + b, (t >> 1) & 1, abort_flag))) break;
         fence_after_sync();
-        const uint32_t b_base = smem_u32(smem + LY::B + s * LY::TILE);
-        const uint32_t bx_base = smem_u32(smem + LY::BX + s * EXT_BYTES);
+        const uint64_t bd = desc_add(bd0, s * LY::TILE);
 #pragma unroll
         for (int kk = 0; kk < 4 * LY::NP; ++kk) {
           const uint32_t koff = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
-          mma_bf16(tmem + b * BN, desc_sw128(a_base + koff), desc_sw128(b_base + koff), idesc, kk > 0);
+          mma_bf16(tmem + b * BN, desc_add(ad0, koff), desc_add(bd, koff), idesc, kk > 0);
         }
-        mma_bf16(tmem + b * BN, desc_sw32(ax_base), desc_sw32(bx_base), idesc, 1u);
+        mma_bf16(tmem + b * BN, axd, desc_add(bxd0, s * EXT_BYTES), idesc, 1u);
         mma_commit(bar_empty + s);
         mma_commit(bar_accf + b);
         done = t + 1;

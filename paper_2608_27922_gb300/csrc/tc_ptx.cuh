@@ -167,6 +167,15 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t addr) {
          | ((uint64_t)2u << 61);               // layout: 128-byte swizzle
 }
 
+// The descriptor of the same operand `bytes` further on: the start-address field is the
+// low 14 bits (address >> 4), and an address inside one CTA's shared memory plus an offset
+// inside the same tile never carries out of it, so one add on the low word suffices (the
+// issuing thread builds each operand's descriptor once and derives the k-steps' from it).
+__device__ __forceinline__ uint64_t desc_add(uint64_t desc, uint32_t bytes) {
+  const uint32_t lo = static_cast<uint32_t>(desc) + (bytes >> 4);
+  return (desc & 0xFFFFFFFF00000000ull) | lo;
+}
+
 // Shared-memory matrix descriptor, 32-byte swizzle, K-major: rows of 32 bytes (16 bf16,
 // one MMA k-step), 8-row groups 256 bytes apart, base 256-byte aligned.
 __device__ __forceinline__ uint64_t desc_sw32(uint32_t addr) {
