@@ -308,6 +308,23 @@ dkv_status_t dkv_bank_update_sequential(dkv_bank_t bank, const void* Kc, const v
  * between admit and compress (DKV_ERR_STATE).                                 */
 dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* stream);
 
+/* Checkpoint read, the inverse of dkv_bank_import (the bank of (K, V, rho, b,
+ * provenance, occupancy) that Alg. 1 carries from one update to the next,
+ * Sec. 3.4): waits for the work enqueued by this handle, then copies every
+ * head's state into the caller's arrays in dst, laid out as in dkv_buffers_t
+ * for this handle's H and M_max:
+ *   k, v              [H][M_max][d] keys / values, dtype of the handle
+ *   rho, base         [H][M_max] fp32 cached density rho_i, baseline b_i
+ *   prov_step         [H][M_max] int64, prov_src [H][M_max] int32
+ *   occupancy         [H] int32
+ * Each of these may point to host memory (pageable or pinned) or device memory;
+ * a NULL field is skipped.  knorm, workspace and workspace_bytes are ignored:
+ * the key norms are derived, and dkv_bank_import recomputes them.  Only rows
+ * [0, occupancy[h]) of head h are meaningful.  Synchronous: returns after the
+ * copies have completed.  DKV_ERR_STATE between admit and compress; a failed
+ * copy gives DKV_ERR_CUDA and leaves dst partly written.                      */
+dkv_status_t dkv_bank_export(dkv_bank_t bank, const dkv_buffers_t* dst);
+
 /* Waits for all work enqueued by this handle, then reports the sticky device
  * error word (DKV_ERR_TIMEOUT / DKV_ERR_DEVICE) or a CUDA error.  Clears the
  * word after reporting it.                                                    */

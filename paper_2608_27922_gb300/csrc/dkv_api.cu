@@ -596,6 +596,31 @@ dkv_status_t dkv_bank_import(dkv_bank_t bank, const int32_t* occupancy, void* st
   return cuda_status(e);
 }
 
+dkv_status_t dkv_bank_export(dkv_bank_t bank, const dkv_buffers_t* dst) {
+  NvtxRange nvtx_range("dkv_bank_export");
+  if (!bank || !dst) return DKV_ERR_ARG;
+  if (bank->state != 0) return DKV_ERR_STATE;
+  cudaStream_t s = bank->last;
+  const Bank& b = bank->b;
+  const size_t rows = (size_t)b.H * b.M_max;
+  const size_t esz = b.bf16 ? 2 : 4;
+  struct Item {
+    void* to;
+    const void* from;
+    size_t bytes;
+  } items[] = {
+      {dst->k, b.k, rows * b.d * esz},          {dst->v, b.v, rows * b.d * esz},
+      {dst->rho, b.rho, rows * 4},              {dst->base, b.base, rows * 4},
+      {dst->prov_step, b.prov_step, rows * 8},  {dst->prov_src, b.prov_src, rows * 4},
+      {dst->occupancy, b.occ, (size_t)b.H * 4},
+  };
+  cudaError_t e = cudaSuccess;
+  for (const Item& it : items)   // one copy per array; the direction follows from the pointers
+    if (e == cudaSuccess && it.to) e = cudaMemcpyAsync(it.to, it.from, it.bytes, cudaMemcpyDefault, s);
+  const cudaError_t es = cudaStreamSynchronize(s);
+  return cuda_status(e != cudaSuccess ? e : es);
+}
+
 dkv_status_t dkv_bank_sync(dkv_bank_t bank) {
   if (!bank) return DKV_ERR_ARG;
   cudaError_t e = cudaStreamSynchronize(bank->last);

@@ -82,6 +82,7 @@ SIGNATURES = [
     ("dkv_bank_commit", _I, [_P, _P]),
     ("dkv_bank_attend", _I, [_P, _P, _I, _P, _P, _I, _P, _P]),
     ("dkv_bank_import", _I, [_P, ctypes.POINTER(ctypes.c_int32), _P]),
+    ("dkv_bank_export", _I, [_P, ctypes.POINTER(dkv_buffers_t)]),
     ("dkv_bank_sync", _I, [_P]),
     ("dkv_bank_stats", _I, [_P, ctypes.POINTER(dkv_layer_stats_t), ctypes.POINTER(dkv_head_stats_t)]),
     ("dkv_bank_occupancy", _I, [_P, ctypes.POINTER(ctypes.c_int32)]),
@@ -223,6 +224,10 @@ def dkv_bank_attend(bank: int, Q, Nq: int, Kw, Vw, W: int, O, stream=None) -> No
 
 def dkv_bank_import(bank: int, occupancy: Sequence[int], stream=None) -> None:
     _check(lib().dkv_bank_import(bank, _i32(occupancy), _stream(stream)), "dkv_bank_import")
+
+
+def dkv_bank_export(bank: int, dst: dkv_buffers_t) -> None:
+    _check(lib().dkv_bank_export(bank, ctypes.byref(dst)), "dkv_bank_export")
 
 
 def dkv_bank_sync(bank: int) -> None:
@@ -425,6 +430,25 @@ class BankLayer:
 
     def import_state(self, occupancy: Sequence[int], stream=None):
         dkv_bank_import(self.handle, occupancy, stream)
+
+    def export_state(self, device="cpu") -> Dict[str, torch.Tensor]:
+        """Checkpoint of every head (k, v, rho, base, prov_step, prov_src, occupancy), copied
+        by dkv_bank_export into new tensors on `device` (host tensors are pinned)."""
+        dev = torch.device(device)
+        pin = dev.type == "cpu"
+        H, M, d = self.H, self.M_max, self.d
+
+        def new(shape, dtype):
+            return torch.empty(shape, dtype=dtype, device=dev, pin_memory=pin)
+        out = {"k": new((H, M, d), self.dtype), "v": new((H, M, d), self.dtype),
+               "rho": new((H, M), torch.float32), "base": new((H, M), torch.float32),
+               "prov_step": new((H, M), torch.int64), "prov_src": new((H, M), torch.int32),
+               "occupancy": new((H,), torch.int32)}
+        dst = dkv_buffers_t()
+        for name in ("k", "v", "rho", "base", "prov_step", "prov_src", "occupancy"):
+            setattr(dst, name, out[name].data_ptr())
+        dkv_bank_export(self.handle, dst)
+        return out
 
     def sync(self):
         dkv_bank_sync(self.handle)
