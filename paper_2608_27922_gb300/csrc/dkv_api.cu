@@ -165,6 +165,8 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, 
   w.cnt = (int32_t*)take(Hh * cnt_stride * 4);
   w.tile_head = (int32_t*)take(Hh * ((Mm + 127) / 128) * 4);
   w.tile_first = (int32_t*)take(Hh * 4);
+  w.pair_head = (int32_t*)take(Hh * (((Mm + 127) / 128 + 1) / 2) * 4);
+  w.pair_first = (int32_t*)take(Hh * 4);
   w.loop_stride = (int64_t)(Hh * std::max((Mm + 127) / 128, (Nm + 127) / 128));
   w.loop_list = (int32_t*)take(3 * (size_t)w.loop_stride * 4);
   w.loop_ctr = (int32_t*)take(3 * 2 * 4);
@@ -372,6 +374,17 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
     e = cudaMemcpy(bk->w.tile_head, tile_head.data(), sizeof(int32_t) * tile_head.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(bk->w.tile_first, tile_first.data(), sizeof(int32_t) * H, cudaMemcpyHostToDevice);
+  // pairs of those tiles (the units of the two-row-tile crossing pass)
+  std::vector<int32_t> pair_head, pair_first(H);
+  for (int h = 0; h < H; ++h) {
+    pair_first[h] = (int32_t)pair_head.size();
+    pair_head.insert(pair_head.end(), (size_t)((budgets[h] + 127) / 128 + 1) / 2, h);
+  }
+  bk->w.n_mpairs = (int)pair_head.size();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(bk->w.pair_head, pair_head.data(), sizeof(int32_t) * pair_head.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(bk->w.pair_first, pair_first.data(), sizeof(int32_t) * H, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     delete bk;
     return DKV_ERR_CUDA;

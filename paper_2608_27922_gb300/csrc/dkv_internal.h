@@ -65,6 +65,10 @@ struct Ws {
   int32_t* tile_head;   // [n_mtiles] head of each 128-row tile of the heads' budgets, head-major
   int32_t* tile_first;  // [H] index of each head's first such tile
   int n_mtiles;         // sum over heads of ceil(M_h / 128)
+  int32_t* pair_head;   // [n_mpairs] head of each pair of those tiles (tiles 2k, 2k + 1 of a
+                        //   head): the units of the two-row-tile crossing pass
+  int32_t* pair_first;  // [H] index of each head's first pair
+  int n_mpairs;         // sum over heads of ceil(ceil(M_h / 128) / 2)
   int32_t* loop_list;   // [3][loop_stride] row tiles with work of the persistent projection,
                         //   survivor and new-baseline passes (each its own: the last two run
                         //   side by side), appended by the pass's classification kernel

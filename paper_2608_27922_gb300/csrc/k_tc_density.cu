@@ -825,6 +825,336 @@ __global__ void __launch_bounds__(THREADS, KV ? 1 : 2)
   if (have_tmem) cta_tmem_free(tmem);
 }
 
+// ---------------------------------------------------------------- crossings, two row tiles
+// Persistent form of the crossing pass (keys only).  One CTA per SM takes units of two
+// row tiles (256 bank rows of one head) at a fixed stride; each column tile of candidates
+// is loaded into shared memory once and feeds the MMAs of both row tiles.  The next
+// unit's row tiles load into the second row-tile buffer while the current unit's last
+// column tiles run, and the barrier phases run on across units (global tile count T), so
+// units follow each other without draining the pipeline or starting a CTA.  TMEM: row
+// tile r, accumulator b = T & 1 at columns 128 (2 r + b).  Warps: 0 TMA producer, 1 MMA
+// issuer, 2-9 the epilogue of row tile 0 and 10-17 that of row tile 1, each as in the
+// one-row-tile form (warps w and w + 4 share TMEM lanes 32 (w % 4) .. +31 and take the
+// halves of each column tile, exchanging their half totals every tile).
+#ifndef DKV_CROSS_DUAL
+#define DKV_CROSS_DUAL 1
+#endif
+constexpr int DU_EPI = 16;
+constexpr int DU_THREADS = 64 + 32 * DU_EPI;
+constexpr uint32_t DU_TMEM_COLS = 512;
+// Column-tile stages == accumulators: then one barrier per stage can stand for both "the
+// tile landed" and "its accumulator is free" (the producer re-arms stage T & 1 only after
+// the MMAs of tile T - 2, which waited for that barrier's previous phase).  With more
+// stages than accumulators the producer could arm a phase that is still open.
+constexpr int DU_STAGES = 2;
+
+struct LayC {
+  static constexpr int TILE = 2 * HALF_BYTES;                 // one 128 x 128 bf16 tile
+  static constexpr int A = 0;                                 // [2 buffers][2 row tiles]
+  static constexpr int B = 4 * TILE;                          // [DU_STAGES] column tiles
+  static constexpr int AX = B + DU_STAGES * TILE;             // [2][2] row-form extensions
+  static constexpr int BX = AX + 4 * EXT_BYTES;               // [DU_STAGES] column-form
+  static constexpr int XCH = BX + DU_STAGES * EXT_BYTES;      // float [2 r][2 b][2 half][BM]
+  static constexpr int BAR = XCH + 2 * 2 * 2 * BM * 4;
+  // a_full[2] a_free[2] empty[DU_STAGES] rdy[DU_STAGES] accf[2 r][2 b], then the TMEM
+  // holder and the abort flag
+  static constexpr int NBAR = 2 + 2 + 2 * DU_STAGES + 4;
+  static constexpr size_t SMEM = BAR + NBAR * 8 + 16;
+  static_assert(B % 1024 == 0 && AX % 1024 == 0, "128-byte-swizzled tiles need 1024-byte alignment");
+  static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+};
+
+// Unit u: head h, first row tile rt0 (even) of the pairs of 128-row tiles of each head's
+// budget, the pass's rows and columns.  False if the unit has no row.
+__device__ __forceinline__ bool cross_unit(const TcJob& j, int u, int& h, int& rt0, int& nrows, int& c0, int& c1) {
+  h = j.w.pair_head[u];
+  rt0 = 2 * (u - j.w.pair_first[h]);
+  job_range(TM_CROSS, j.w.hd[h], *layer_of(j.w, h), nrows, c0, c1);
+  return rt0 * BM < nrows;
+}
+
+template <int P>
+__global__ void __launch_bounds__(DU_THREADS, 1)
+    tc_cross_dual(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
+                  const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx, TcJob j,
+                  int n_units) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0u) {
+    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9904);
+    return;
+  }
+  using LY = LayC;
+  float* xch = reinterpret_cast<float*>(smem + LY::XCH);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + LY::BAR);
+  uint64_t* a_full = bars + 0;                   // [2] row tiles of a unit landed
+  uint64_t* a_free = bars + 2;                   // [2] MMAs of the buffer's last unit complete
+  uint64_t* bar_empty = bars + 4;                // [DU_STAGES] MMAs of the stage's tile complete
+  uint64_t* bar_rdy = bar_empty + DU_STAGES;     // [DU_STAGES] column tile T landed (stage T & 1)
+                                                 //   and accumulator T & 1 released by all 16
+                                                 //   epilogue warps: the issuer's one wait per tile
+  uint64_t* bar_accf = bar_rdy + DU_STAGES;      // [2 r][2 b] MMAs of row tile r into b complete
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + LY::NBAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(a_full + i, 1);
+      mbar_init(a_free + i, 1);
+    }
+    for (int s = 0; s < DU_STAGES; ++s) {
+      mbar_init(bar_empty + s, 1);
+      mbar_init(bar_rdy + s, DU_EPI + 1);   // the epilogue warps + the producer (with bytes)
+    }
+    for (int i = 0; i < 4; ++i) mbar_init(bar_accf + i, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, DU_TMEM_COLS);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer
+      prefetch_map(&tmA); prefetch_map(&tmAx); prefetch_map(&tmB); prefetch_map(&tmBx);
+      int k = 0;          // units with columns so far (row-tile buffer k & 1)
+      uint32_t T = 0;     // column tiles so far
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+        int h, rt0, nrows, c0, c1;
+        if (!cross_unit(j, u, h, rt0, nrows, c0, c1) || c1 <= c0) continue;
+        const int nt = (c1 - c0 + BN - 1) / BN;
+        const int a = k & 1;
+        const bool two = (rt0 + 1) * BM < nrows;
+        if (!(ok = mbar_wait(a_free + a, ((k >> 1) & 1) ^ 1, abort_flag))) break;
+        mbar_arrive_expect_tx(a_full + a, (two ? 2u : 1u) * (uint32_t)(LY::TILE + EXT_BYTES));
+        for (int r = 0; r < (two ? 2 : 1); ++r) {
+          for (int pn = 0; pn < 2; ++pn)
+            tma_load_3d(smem + LY::A + (2 * a + r) * LY::TILE + pn * HALF_BYTES, &tmA, a_full + a, pn * 64,
+                        (rt0 + r) * BM, h);
+          tma_load_3d(smem + LY::AX + (2 * a + r) * EXT_BYTES, &tmAx, a_full + a, 0, (rt0 + r) * BM, h);
+        }
+        for (int t = 0; t < nt; ++t, ++T) {
+          const int s = (int)(T & 1);
+          if (!(ok = mbar_wait(bar_empty + s, ((T >> 1) & 1) ^ 1, abort_flag))) break;
+          mbar_arrive_expect_tx(bar_rdy + s, LY::TILE + EXT_BYTES);
+          const int col = c0 + t * BN;
+          for (int pn = 0; pn < 2; ++pn)
+            tma_load_3d(smem + LY::B + s * LY::TILE + pn * HALF_BYTES, &tmB, bar_rdy + s, pn * 64, col, h);
+          tma_load_3d(smem + LY::BX + s * EXT_BYTES, &tmBx, bar_rdy + s, 16, col, h);
+        }
+        ++k;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.w.L, DEV_TIMEOUT, 130);
+        // copies may still be in flight and nothing will consume them: wait a fixed 50 us,
+        // far longer than any copy takes to land
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 50000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer: per column tile 9 MMAs for each row tile (8 k-steps
+      // of the keys + 1 of the extension), one wait
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      const uint64_t bd0 = desc_sw128(smem_u32(smem + LY::B));
+      const uint64_t bxd0 = desc_sw32(smem_u32(smem + LY::BX));
+      int k = 0;
+      uint32_t T = 0;
+      bool ok = true, any = false;
+      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+        int h, rt0, nrows, c0, c1;
+        if (!cross_unit(j, u, h, rt0, nrows, c0, c1) || c1 <= c0) continue;
+        const int nt = (c1 - c0 + BN - 1) / BN;
+        const int a = k & 1;
+        const bool two = (rt0 + 1) * BM < nrows;
+        if (!(ok = mbar_wait(a_full + a, (k >> 1) & 1, abort_flag))) break;
+        const uint64_t ad0 = desc_sw128(smem_u32(smem + LY::A + 2 * a * LY::TILE));
+        const uint64_t axd0 = desc_sw32(smem_u32(smem + LY::AX + 2 * a * EXT_BYTES));
+        for (int t = 0; t < nt; ++t, ++T) {
+          const int b = (int)(T & 1);   // stage and accumulator
+          if (!(ok = mbar_wait(bar_rdy + b, (T >> 1) & 1, abort_flag))) break;
+          fence_after_sync();
+          const uint64_t bd = desc_add(bd0, b * LY::TILE);
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            if (r == 0 || two) {
+              const uint64_t ad = desc_add(ad0, r * LY::TILE);
+              const uint32_t acc = tmem + (uint32_t)((2 * r + b) * BN);
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
+                mma_bf16(acc, desc_add(ad, koff), desc_add(bd, koff), idesc, kk > 0);
+              }
+              mma_bf16(acc, desc_add(axd0, r * EXT_BYTES), desc_add(bxd0, b * EXT_BYTES), idesc, 1u);
+            }
+            mma_commit(bar_accf + 2 * r + b);   // (no new MMA for an absent row tile: arrives at once)
+          }
+          mma_commit(bar_empty + b);
+          any = true;
+        }
+        if (!ok) break;
+        mma_commit(a_free + a);
+        ++k;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.w.L, DEV_TIMEOUT, 230);
+      }
+      // every issued MMA complete before TMEM is freed: a last commit covers all of them
+      if (any) {
+        mma_commit(a_free + (k & 1));
+        volatile int no_abort = 0;
+        mbar_wait(a_free + (k & 1), (k >> 1) & 1, &no_abort);
+      }
+    }
+  } else {
+    // ---------------- epilogue: thread = row (TMEM lane) of row tile r
+    const int ew = warp - 2;                      // 0..15
+    const int r = ew >> 3;                        // row tile of the unit
+    const int half = (ew >> 2) & 1;               // columns [64 half, 64 half + 64) of each tile
+    const int q = warp & 3;                       // TMEM lane quarter
+    const int r_local = q * 32 + lane;
+    const int bar_id = 1 + q + 4 * r;             // the two warps of this (row tile, quarter)
+    const KParams kp = j.kp;
+    const float c = pow_c<P>(kp);                 // (sigma^2 / 2)^p
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(2 * r * BN);
+    float* xr = xch + r * (2 * 2 * BM);           // this row tile's exchange slots [b][half][BM]
+    // both accumulators start free: this warp's release for tiles 0 and 1
+    if (lane == 0) {
+      mbar_arrive(bar_rdy + 0);
+      mbar_arrive(bar_rdy + 1);
+    }
+    uint32_t T = 0;
+    bool ok = true;
+    // after a failed wait the warp keeps walking every unit and tile without work: the
+    // two warps of a row quarter must meet at the same named barriers
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+      int h, rt0, nrows, c0, c1;
+      if (!cross_unit(j, u, h, rt0, nrows, c0, c1)) continue;
+      const int nt = c1 > c0 ? (c1 - c0 + BN - 1) / BN : 0;
+      const int row = (rt0 + r) * BM + r_local;
+      const bool active = row < nrows;
+      const bool tile_live = (rt0 + r) * BM < nrows;   // warp-uniform: the row tile has MMAs
+      const int64_t bh = (int64_t)h * j.b.M_max;
+      // per-row state (sums in units of |A|^-p)
+      float S = 0.f, thr = 0.f;
+      int cross = INT_MAX;
+      float* snap_row = nullptr;
+      if (active) {
+        const float rho = j.b.rho[bh + row];
+        thr = (__fmul_rn(kp.tau, j.b.base[bh + row]) - rho) / c;
+        if (thr <= 0.f) cross = 0;
+        snap_row = j.w.snap + (bh + row) * j.w.snap_stride;
+        if (half == 0) snap_row[0] = 0.f;
+      }
+      for (int t = 0; t < nt; ++t, ++T) {
+        const int b = (int)(T & 1);
+        const int col0 = c0 + t * BN;
+        const int nc = min(BN, c1 - col0);
+        // every warp waits for the MMAs of its row tile (also an absent one: its release
+        // of accumulator b must not run ahead of tile T)
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_accf + 2 * r + b, (T >> 1) & 1, abort_flag));
+        if (!ok) *abort_flag = 1;
+        fence_after_sync();
+        // chunk totals of this warp's half, then the running sum of the row
+        float tot[2] = {0.f, 0.f};
+        if (ok && tile_live) {
+#pragma unroll
+          for (int ch = 0; ch < 2; ++ch) {
+            const int cs = half * 64 + ch * 32;
+            if (cs >= nc) continue;   // warp-uniform
+            float v[32];
+            tmem_ld32(lane_base + b * BN + cs, v);
+            tmem_wait_ld();
+            const int lim = min(32, nc - cs);
+            tot[ch] = lim == 32 ? chunk_sum<P>(v) : chunk_sum_partial<P>(v, lim);
+          }
+        }
+        // exchange the half totals of this row, so both warps carry the same running sum
+        const float mine = tot[0] + tot[1];
+        xr[(b * 2 + half) * BM + r_local] = mine;
+        named_bar(bar_id, 64);
+        const float other = xr[(b * 2 + (half ^ 1)) * BM + r_local];
+        const float T0 = half == 0 ? mine : other;
+        const float T1 = half == 0 ? other : mine;
+        const float base0 = half == 0 ? S : S + T0;
+        int hit = -1;
+        float run = base0;
+        if (ok && active && cross == INT_MAX) {
+          if (base0 + tot[0] >= thr) hit = 0;
+          else if ((base0 + tot[0]) + tot[1] >= thr) { hit = 1; run = base0 + tot[0]; }
+        }
+        // exact position inside the chunk, term by term (at most once per row); the TMEM
+        // load is warp-collective, so the whole warp takes part for each chunk hit
+#pragma unroll
+        for (int hc = 0; hc < 2; ++hc) {
+          const int cs = half * 64 + hc * 32;
+          if (cs < nc && __any_sync(0xffffffffu, hit == hc)) {
+            float v[32];
+            tmem_ld32(lane_base + b * BN + cs, v);
+            tmem_wait_ld();
+            if (hit == hc) {
+              const int lim = min(32, nc - cs);
+              // the 32 terms are independent: all of them first (in place), then the
+              // running sum
+#pragma unroll
+              for (int jj = 0; jj < 32; ++jj) v[jj] = term1<P>(v[jj]);
+              int pos = lim;
+#pragma unroll
+              for (int jj = 0; jj < 32; ++jj) {
+                if (jj < lim && pos == lim) {
+                  run += v[jj];
+                  if (run >= thr) pos = jj + 1;
+                }
+              }
+              cross = col0 + cs + pos;
+            }
+          }
+        }
+        S = (S + T0) + T1;
+        if (ok && active && half == 0 && nc == BN) snap_row[(col0 + BN) / SNAP] = S;
+        if (ok) {
+          fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile T + 2
+        }
+      }
+      // unit end: each half saw only its own columns, the row's first crossing is the
+      // earlier one.  The exchange slots of accumulator T & 1 were last read before the
+      // barrier of tile T - 1; a second barrier keeps the next unit's first tile from
+      // writing them before the partner warp has read.
+      int* xi = reinterpret_cast<int*>(xr + (T & 1) * 2 * BM);
+      xi[half * BM + r_local] = cross;
+      named_bar(bar_id, 64);
+      cross = min(xi[r_local], xi[BM + r_local]);
+      named_bar(bar_id, 64);
+      if (ok && active && half == 0) {
+        const DevLayer L = *layer_of(j.w, h);
+        j.w.cross[bh + row] = cross;
+        const int bin = cross == INT_MAX ? L.rmax + 1 : cross;
+        atomicAdd(&j.w.hist[(int64_t)h * j.w.hist_stride + bin], 1);
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      if (lane == 0) dev_fail(j.w.L, DEV_TIMEOUT, 330);
+    }
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after_sync();
+    tmem_dealloc(tmem, DU_TMEM_COLS);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -909,6 +1239,18 @@ cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void*
     mav = ma;   // never read
     mbv = mb;
   }
+  const int n_sm = sm_count();
+  if constexpr (MODE == TM_CROSS) {
+    if (DKV_CROSS_DUAL && !kv && n_sm > 0) {   // the persistent two-row-tile form
+      TcJob job{b, w, kp, 0, 0};
+      timer_begin(t, name, s);
+      if (kp.p == 1) tc_cross_dual<1><<<n_sm, DU_THREADS, LayC::SMEM, s>>>(ma, max_, mb, mbx, job, w.n_mpairs);
+      else if (kp.p == 4) tc_cross_dual<4><<<n_sm, DU_THREADS, LayC::SMEM, s>>>(ma, max_, mb, mbx, job, w.n_mpairs);
+      else tc_cross_dual<2><<<n_sm, DU_THREADS, LayC::SMEM, s>>>(ma, max_, mb, mbx, job, w.n_mpairs);
+      timer_end(t, s);
+      return cudaGetLastError();
+    }
+  }
   // passes over bank rows take one CTA per budget-sized row tile of each head
   const int lin = (MODE == TM_CROSS || MODE == TM_PROJECT || MODE == TM_SUB) && split == 1 ? 1 : 0;
   const int tpn = (max_rows + BM - 1) / BM;
@@ -918,7 +1260,6 @@ cudaError_t launch_tc(const Bank& b, const Ws& w, const KParams& kp, const void*
   // persistent form, a few CTAs per SM (most of those row tiles have no column when
   // layers admit nothing)
   int n_units = 0;
-  const int n_sm = sm_count();
   if ((MODE == TM_PROJECT || MODE == TM_SUB || MODE == TM_NEWBASE) && n_sm > 0) {
     const int units = lin ? w.n_mtiles : tpn * b.H;
     if (units >= 16 * n_sm) {
@@ -973,6 +1314,11 @@ cudaError_t tc_set_smem_limits() {
   DKV_OPTLOOP(TM_PROJECT)
   DKV_OPTLOOP(TM_SUB)
   DKV_OPTLOOP(TM_NEWBASE)
+#define DKV_OPTD(P)                                                                                           \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_cross_dual<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LayC::SMEM);
+  DKV_OPTD(1) DKV_OPTD(2) DKV_OPTD(4)
+#undef DKV_OPTD
 #undef DKV_OPTLOOP
 #undef DKV_OPTL
 #undef DKV_OPT
