@@ -496,10 +496,6 @@ __global__ void __launch_bounds__(256) k_sort_runs(Ws w, int n_max, int identity
 }
 
 // Number of keys of the sorted run r[0..RUN) below x (branchless, 9 probes).
-#ifndef DKV_SORT_RUNS_PER_CTA
-#define DKV_SORT_RUNS_PER_CTA 4
-#endif
-
 __device__ __forceinline__ int run_rank(const unsigned long long* r, unsigned long long x) {
   int pos = 0;
 #pragma unroll
@@ -1110,12 +1106,18 @@ cudaError_t launch_sort(const Bank& b, const Ws& w, const void* Kc, const void* 
   k_sort_runs<<<dim3((max_runs + 7) / 8, b.H), 256, 0, s>>>(w, b.n_max, identity);
   timer_end(t, s);
   timer_begin(t, "sort_rank", s);
-  // four runs per CTA (1,024 threads): each CTA loads every run of its head into shared
-  // memory once for four runs (config 4: 1.35 ms with one run per CTA, 1.16 with two, 1.13
-  // with four)
-  constexpr int RB = DKV_SORT_RUNS_PER_CTA;
-  k_sort_rank<RB><<<dim3((max_runs + RB - 1) / RB, b.H), RUN * RB, (size_t)max_runs * RUN * 8, s>>>(
-      b, w, (const char*)Kc, (const char*)Vc, b.bf16 ? 2 : 4, identity);
+  // four runs per CTA (1,024 threads) when that still gives every SM two CTAs: each CTA
+  // loads every run of its head into shared memory once for four runs (config 4: 1.35 ms
+  // with one run per CTA, 1.16 with two, 1.13 with four); one run per CTA otherwise (config
+  // 1, 228 runs: 22 us against 33 with four)
+  const int n_sm = sm_count();
+  const size_t sm_bytes = (size_t)max_runs * RUN * 8;
+  if ((int64_t)b.H * ((max_runs + 3) / 4) >= 2 * (int64_t)n_sm)
+    k_sort_rank<4><<<dim3((max_runs + 3) / 4, b.H), RUN * 4, sm_bytes, s>>>(b, w, (const char*)Kc, (const char*)Vc,
+                                                                          b.bf16 ? 2 : 4, identity);
+  else
+    k_sort_rank<1><<<dim3(max_runs, b.H), RUN, sm_bytes, s>>>(b, w, (const char*)Kc, (const char*)Vc,
+                                                             b.bf16 ? 2 : 4, identity);
   timer_end(t, s);
   return cudaGetLastError();
 }
@@ -1162,8 +1164,9 @@ cudaError_t launch_seq_gather(const Bank& b, const Ws& w, const void* Kc, const 
 
 cudaError_t update_set_smem_limits() {
   // phase 2 of the sort holds every run of a head: up to 64 runs of 2 KiB
-  cudaError_t e = cudaFuncSetAttribute(k_sort_rank<DKV_SORT_RUNS_PER_CTA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       64 * RUN * 8);
+  cudaError_t e = cudaFuncSetAttribute(k_sort_rank<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * RUN * 8);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_sort_rank<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * RUN * 8);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sel_smem_bytes(SEL_STAGE));
   return e;

@@ -417,3 +417,12 @@ def test_blocks_smaller_than_capacity(dkv, mode):
     wl = synth.get_workload("wan13b_layer_h12", H=3, N=300, W=200, Nq=130, budgets=700, steps=6)
     reps = _rollout(dkv, wl, mode, n_max=512)
     assert sum(r.rstar_oracle for r in reps) > 0
+
+
+def test_many_heads_sort_schedule(dkv):
+    """Enough heads that the sort's rank phase places four runs per CTA (152 heads of five
+    runs: blocks of 1,280 candidates into banks of 640), teacher-forced against the oracle
+    on the empty-bank block and one evicting block (about 40 s of host time)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=152, N=1280, W=64, Nq=64, budgets=640, steps=3)
+    reps = _rollout(dkv, wl, "tc", check_attn=False)
+    assert len(reps) == 2 and reps[1].rstar_oracle > 0
