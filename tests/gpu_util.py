@@ -133,6 +133,7 @@ class Report:
     cross_gap_max: float = 0.0
     set_gap_max: float = 0.0
     kv_bit_exact: bool = True
+    heads_set_differs: int = 0          # heads whose final banks differ by explained decisions
     notes: List[str] = dataclasses.field(default_factory=list)
 
     def ok(self) -> bool:
@@ -293,9 +294,22 @@ def _compare_layer(rep: Report, prm: oracle.Params, before: oracle.LayerBank, ob
                 cut = min(hr.rho_tilde[fill]) if fill else None
                 for key in only_g | only_o:
                     i = pre.get(key)
-                    if i is None:      # a candidate admitted on one side only
-                        ok = False
-                        break
+                    if i is None:
+                        # a candidate admitted on one side only: explained when its score is
+                        # within `tol` of the admission cut-off (the scores of the last
+                        # admitted and the first refused candidate in the oracle's order)
+                        r = hr.r_used
+                        src = key[1]
+                        if prm.order != "score" or r <= 0 or r >= N or not 0 <= src < N:
+                            ok = False
+                            break
+                        cuts = [hr.s[hr.pi[r - 1]], hr.s[hr.pi[r]]]
+                        gap = min(abs(hr.s[src] - c) / max(abs(c), 1e-300) for c in cuts)
+                        rep.set_gap_max = max(rep.set_gap_max, gap)
+                        if gap > tol:
+                            ok = False
+                            break
+                        continue
                     gap = abs(hr.g_star[i] - prm.tau) / prm.tau
                     if cut is not None:
                         gap = min(gap, abs(hr.rho_tilde[i] - cut) / abs(cut))
@@ -305,11 +319,18 @@ def _compare_layer(rep: Report, prm: oracle.Params, before: oracle.LayerBank, ob
                         break
             if not ok:
                 rep.set_unexplained += len(only_g) + len(only_o)
+            else:
+                rep.heads_set_differs += 1
+        # an equally valid but different final bank (explained decisions): the densities of
+        # Eq. 5 / C.4 are sums over it, so they are compared only in heads whose banks agree
+        same_bank = not (only_g or only_o)
         for key in set(g) & set(o):
             kg, vg, rg, bg, kn, _ = g[key]
             ko, vo, ro, bo = o[key]
             if not (np.array_equal(kg, ko[:kg.shape[0]].astype(np.float32)) and np.array_equal(vg, vo.astype(np.float32))):
                 rep.kv_bit_exact = False
+            if not same_bank:
+                continue
             rep.rho_max_rel = max(rep.rho_max_rel, abs(rg - ro) / max(abs(ro), 1e-30))
             rep.base_max_rel = max(rep.base_max_rel, abs(bg - bo) / max(abs(bo), 1e-30))
             i = pre.get(key)

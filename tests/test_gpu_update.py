@@ -426,3 +426,6 @@ def test_many_heads_sort_schedule(dkv):
     wl = synth.get_workload("wan13b_layer_h12", H=152, N=1280, W=64, Nq=64, budgets=640, steps=3)
     reps = _rollout(dkv, wl, "tc", check_attn=False)
     assert len(reps) == 2 and reps[1].rstar_oracle > 0
+    # N > M: r* = M < N, so near-tied scores at the admission cut-off may swap a candidate
+    # (explained by check_report); only a few heads may differ
+    assert all(r.heads_set_differs <= wl.H // 20 for r in reps), [r.heads_set_differs for r in reps]
