@@ -1329,12 +1329,23 @@ cudaError_t tc_set_smem_limits() {
 
 // With the [K; V] descriptor every pass also reads the values beside its keys (same
 // sources as the fp32 passes: the candidates' values, vperm, the bank's, vsurv, vevict).
+#ifndef DKV_SCORE_SPLIT
+#define DKV_SCORE_SPLIT 0   // 0: by grid size, else the split itself
+#endif
+
 cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, const void* Vc, int N, const KParams& kp,
                             cudaStream_t s, Timer* t) {
   const bool kv = w.vperm != nullptr;
   // the candidates (caller's array) are [H][N][d]; their extension rows, like every
-  // candidate array of the workspace, [H][n_max][32]
-  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", 2,
+  // candidate array of the workspace, [H][n_max][32].  The bank columns are split over two
+  // CTAs per row tile while the row tiles alone would not fill the GPU several times over
+  int split = DKV_SCORE_SPLIT;
+  if (split == 0) {
+    const int n_sm = sm_count();
+    const int64_t ctas = (int64_t)((N + BM - 1) / BM) * b.H;
+    split = n_sm > 0 && ctas >= 16 * (int64_t)n_sm ? 1 : 2;
+  }
+  return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", split,
                              kv ? Vc : nullptr, kv ? b.v : nullptr, b.n_max);
 }
 

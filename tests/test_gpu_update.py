@@ -420,10 +420,11 @@ def test_blocks_smaller_than_capacity(dkv, mode):
 
 
 def test_many_heads_sort_schedule(dkv):
-    """Enough heads that the sort's rank phase places four runs per CTA (152 heads of five
-    runs: blocks of 1,280 candidates into banks of 640), teacher-forced against the oracle
-    on the empty-bank block and one evicting block (about 40 s of host time)."""
-    wl = synth.get_workload("wan13b_layer_h12", H=152, N=1280, W=64, Nq=64, budgets=640, steps=3)
+    """Enough heads that the sort's rank phase places four runs per CTA and the score pass
+    leaves the bank columns unsplit (256 heads of 1,280 candidates: 2,560 score row tiles,
+    five runs each, into banks of 640), teacher-forced against the oracle on the
+    empty-bank block and one evicting block (about a minute of host time)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=256, N=1280, W=64, Nq=64, budgets=640, steps=3)
     reps = _rollout(dkv, wl, "tc", check_attn=False)
     assert len(reps) == 2 and reps[1].rstar_oracle > 0
     # N > M: r* = M < N, so near-tied scores at the admission cut-off may swap a candidate
