@@ -1180,7 +1180,7 @@ def run_stack(args):
             "e2e": e2e, "gpu_launches": launches * world, "roofline": roof, "cpu_baseline": cpu, "clocks": clk,
             "per_kernel": per_kernel,
             "per_kernel_note": f"{P} further steps on one stream with every launch timed by CUDA events (not "
-                               "in value); "
+                               "in value; the survivor and new-baseline passes then run one after the other); "
                                "tensor kernels against the bf16 peak, memory-bound kernels' algorithmic (and "
                                "moved-by-design) bytes against the HBM peak",
             "update": {"layers_admitting_per_step": admitting,

@@ -360,8 +360,11 @@ dkv_status_t dkv_bank_intermediates(dkv_bank_t bank, dkv_intermediates_t* out);
  * other values: DKV_ERR_ARG).  dkv_bank_kernel_times() returns, per kernel
  * name, the number of launches and the summed device milliseconds of the
  * launches whose events have completed (it synchronises); with enable = 2 the
- * other kernels are counted with 0 ms.  Timing adds two event records per
- * timed launch; keep it off when not measuring.                             */
+ * other kernels are counted with 0 ms.  With enable = 1 the commit runs the
+ * survivor and new-baseline passes one after the other on the caller's stream
+ * (otherwise side by side on two streams), so that each launch's time is its
+ * own.  Timing adds two event records per timed launch; keep it off when not
+ * measuring.                                                                 */
 dkv_status_t dkv_bank_set_timing(dkv_bank_t bank, int32_t enable);
 dkv_status_t dkv_bank_kernel_times(dkv_bank_t bank, int32_t max_kernels, char* names /* [max][48] */,
                                    int32_t* launches, double* total_ms, int32_t* n_kernels);

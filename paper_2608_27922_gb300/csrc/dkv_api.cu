@@ -475,6 +475,13 @@ dkv_status_t dkv_bank_commit(dkv_bank_t bank, void* stream) {
   bank->last = s;
   bank->state = 0;
   cudaError_t e = launch_commit(b, w, bank->Vc, bank->N, bank->src_map, s, t);
+  if (t->on && !t->attend_only) {
+    // every launch timed: the two passes one after the other on `stream`, so that each
+    // launch's time is its own
+    if (e == cudaSuccess) e = bank->tc ? launch_subtract_tc(b, w, kp, s, t) : launch_subtract_fp32(b, w, kp, s, t);
+    if (e == cudaSuccess) e = bank->tc ? launch_newbase_tc(b, w, kp, s, t) : launch_newbase_fp32(b, w, kp, s, t);
+    return cuda_status(e);
+  }
   // Eq. C.4 (survivors) on `stream` beside Eq. 5 (admitted states) on the handle's own
   // stream: disjoint slots, read-only inputs; `stream` waits for both
   if (e == cudaSuccess) e = cudaEventRecord(bank->ev_fork, s);
