@@ -175,23 +175,6 @@ __device__ __forceinline__ float chunk_sum(const float (&v)[32]) {
   return P == 1 ? -(a.x + a.y) : a.x + a.y;
 }
 
-// Sum of wb_j |v_j|^-P over a full 32-column chunk (wb in shared memory, 16-byte aligned).
-template <int P>
-__device__ __forceinline__ float chunk_sum_w(const float (&v)[32], const float* wb) {
-  const float4* w4 = reinterpret_cast<const float4*>(wb);
-  float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
-#pragma unroll
-  for (int k = 0; k < 8; k += 2) {
-    const float4 wx = w4[k / 2], wy = w4[4 + k / 2];
-    a0 = acc2wx2<P>(make_float2(v[2 * k], v[2 * k + 1]), make_float2(v[2 * k + 16], v[2 * k + 17]),
-                    make_float2(wx.x, wx.y), make_float2(wy.x, wy.y), a0);
-    a1 = acc2wx2<P>(make_float2(v[2 * k + 2], v[2 * k + 3]), make_float2(v[2 * k + 18], v[2 * k + 19]),
-                    make_float2(wx.z, wx.w), make_float2(wy.z, wy.w), a1);
-  }
-  const float2 a = __fadd2_rn(a0, a1);
-  return P == 1 ? -(a.x + a.y) : a.x + a.y;
-}
-
 // Score pass, one warp's 64-column half of a tile in the 16x256b layout (va: lanes
 // 0..15 of the warp's quarter, vb: lanes 16..31): this thread holds rows i/4, i/4 + 8,
 // i/4 + 16, i/4 + 24 at columns 8k + 2 (i % 4) + {0, 1}, k = 0..7, so it needs 16
@@ -527,18 +510,7 @@ __device__ __forceinline__ bool pairs_unit(const CUtensorMap& tmA, const CUtenso
             if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile t + 2
           }
           const int lim = min(32, nc - cs);
-          if (MODE == TM_SCORE) {
-            const float* ib = meta + (t % META_BUFS) * BN + cs;
-            if (lim == 32) {
-              tot[ch] = chunk_sum_w<P>(v, ib);
-            } else {
-              float s = 0.f;
-#pragma unroll
-              for (int jj = 0; jj < 32; ++jj)
-                if (jj < lim) s = fmaf(term1<P>(v[jj]), ib[jj], s);
-              tot[ch] = s;
-            }
-          } else if (MODE == TM_NEWBASE) {
+          if (MODE == TM_NEWBASE) {   // (the score pass takes the 16x256b branch above)
             const int sk = self - (col0 + cs);
             if (lim == 32 && (sk < 0 || sk >= 32)) tot[ch] = chunk_sum<P>(v);
             else tot[ch] = chunk_sum_skip<P>(v, lim, sk);
