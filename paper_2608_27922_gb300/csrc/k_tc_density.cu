@@ -33,7 +33,9 @@
 // CTA (320 threads, 2 per SM): warp 0 TMA producer, warp 1 MMA issuer, warps 2-9
 // epilogue.  Epilogue warps w and w+4 share TMEM lanes 32 (w % 4) .. +31 (one row
 // per lane) and split each 128-column tile into halves of 64 columns; the crossing
-// and projection passes exchange half totals through shared memory every tile.
+// and projection passes exchange half totals through shared memory every tile.  The
+// crossing pass over keys runs in a persistent form with two row tiles per CTA
+// (tc_cross_dual, below); the [K; V] descriptor keeps the one-row-tile form.
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
