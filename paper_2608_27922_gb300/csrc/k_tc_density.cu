@@ -268,7 +268,9 @@ __device__ __forceinline__ void trivial_row(const TcJob& j, const DevHead& hd, i
   const int64_t bh = (int64_t)h * j.b.M_max;
   const float c = pow_c<P>(j.kp);
   if (MODE == TM_PROJECT) {
-    const float S = j.w.snap[(bh + row) * j.w.snap_stride + c0 / SNAP];
+    // the snapshot at column 0 is the empty sum, 0 (written by the crossing pass): rows of
+    // a prefix shorter than a snapshot spacing skip its strided load
+    const float S = c0 == 0 ? 0.f : j.w.snap[(bh + row) * j.w.snap_stride + c0 / SNAP];
     j.w.rho_t[bh + row] = fmaf(c, S, j.b.rho[bh + row]);
   } else if (MODE == TM_SUB) {
     const int slot = hd.e == 0 ? row : j.w.surv_list[bh + row];
