@@ -743,12 +743,26 @@ def _oracle_step(wl, ro, ob, t):
     return time.perf_counter() - t0, m + wl.N
 
 
+def _oracle_steps(wl, ro, ob, t, n):
+    """n consecutive steady-state steps of one head in the oracle: (seconds, keys scored)."""
+    tot_s, tot_k = 0.0, 0
+    for i in range(n):
+        dt, k = _oracle_step(wl, ro, ob, t + i)
+        tot_s += dt
+        tot_k += k
+    return tot_s, tot_k
+
+
+CPU_SAMPLE_STEPS = 4         # single-layer workloads: steady-state steps of one head
+CPU_SAMPLE_STACK = (3, 2)    # stacks: heads of layer 0, steady-state steps each
+
+
 def cpu_baseline_sample(wl, layer):
     ro, ob, t = _oracle_head_setup(wl, layer, 0)
-    dt, keys = _oracle_step(wl, ro, ob, t)
+    dt, keys = _oracle_steps(wl, ro, ob, t, CPU_SAMPLE_STEPS)
     return {"value": keys / dt, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
-            "sample": f"1 head (of {wl.H}), 1 steady-state step of {wl.name}: attention of {wl.Nq} queries "
-                      f"+ bank update, {keys} keys scored in {dt:.2f} s (numpy float64)"}
+            "sample": f"1 head (of {wl.H}), {CPU_SAMPLE_STEPS} steady-state steps of {wl.name}: attention of "
+                      f"{wl.Nq} queries + bank update each, {keys} keys scored in {dt:.2f} s (numpy float64)"}
 
 
 def run_reference(args):
@@ -1217,18 +1231,19 @@ def cpu_baseline_stack(wl, keys_per_block):
     """The oracle on a bounded sample of the stack workload: heads of layer 0 brought to
     steady state (untimed), then one step each (attention + update) timed; the rate is
     keys scored per second, and the model step's time is extrapolated from it."""
-    heads = _stack_sample_heads(wl, 2)
+    n_heads, n_steps = CPU_SAMPLE_STACK
+    heads = _stack_sample_heads(wl, n_heads)
     tot_s, tot_k = 0.0, 0
     for h in heads:
         ro, ob, t = _oracle_head_setup(wl, 0, h)
-        dt, k = _oracle_step(wl, ro, ob, t)
+        dt, k = _oracle_steps(wl, ro, ob, t, n_steps)
         tot_s += dt
         tot_k += k
     rate = tot_k / tot_s
     return {"value": rate, "unit": UNIT, "cores": oracle_threads(), "kind": "oracle",
             "sample": f"{len(heads)} head(s) of layer 0 (budgets {[wl.budgets[h] for h in heads]}) of {wl.name}, "
-                      f"one steady-state step each (attention of {wl.Nq} queries + bank update), {tot_k} keys "
-                      f"scored in {tot_s:.1f} s (numpy float64)",
+                      f"{n_steps} steady-state steps each (attention of {wl.Nq} queries + bank update), {tot_k} "
+                      f"keys scored in {tot_s:.1f} s (numpy float64)",
             "blocks_per_s_extrapolated": rate / keys_per_block if keys_per_block else None}
 
 
