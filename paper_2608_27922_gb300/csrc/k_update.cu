@@ -561,10 +561,15 @@ __global__ void __launch_bounds__(RUN * RB) k_sort_rank(Bank bk, Ws w, const cha
   const int kg = rb / 64;                         // key groups, one extension group, then
   const int vg = w.vperm ? kg : 0;                // value groups ([K; V] descriptor)
   const int per_row = kg + 1 + vg;
+  // every reader of the copy takes positions below the layer's rmax (the crossing,
+  // projection and new-baseline passes, the commit), or, in an empty bank, below
+  // min(N, M_h) (the candidates it admits in source order): later positions are not copied
+  const DevHead hd = w.hd[h];
+  const int need = hd.empty ? min(N, hd.M) : layer_of(w, h)->rmax;
   for (int c = t; c < RUN * RB * per_row; c += RUN * RB) {
     const int row = c / per_row, grp = c - row * per_row;
     const int pos = s_pos[row], src = s_src[row];
-    if (pos < 0 || src < 0 || src >= N) continue;   // no row (past N), or reported above
+    if (pos < 0 || pos >= need || src < 0 || src >= N) continue;   // not needed, no row, or reported above
     if (grp < kg) {
       copy64(reinterpret_cast<const uint4*>(Kc + ((int64_t)h * N + src) * rb) + 4 * grp,
              reinterpret_cast<uint4*>((char*)w.kperm + (hn + pos) * rb) + 4 * grp);
