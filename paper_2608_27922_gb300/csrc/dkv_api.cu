@@ -158,7 +158,7 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, 
   const int sort_stride = (n_max + 255) / 256 * 256;
   w.sortbuf = (unsigned long long*)take(Hh * (size_t)sort_stride * 8);
   const int invb_stride = (M_max + 3) & ~3;   // 16-byte rows for the bulk copies
-  w.invb = (float*)take((Hh * (size_t)invb_stride + 128) * 4);
+  w.invb = (float*)take((Hh * (size_t)invb_stride + 256) * 4);   // a whole 256-column tile past the end
   const int part_stride = (M_max > n_max ? M_max : n_max);
   const int cnt_stride = (part_stride + 127) / 128;
   w.part = (float*)take(2 * Hh * part_stride * 4);
@@ -167,6 +167,7 @@ size_t ws_layout(int H, int d, int M_max, int n_max, int bf16, int kv, Ws* out, 
   w.tile_first = (int32_t*)take(Hh * 4);
   w.pair_head = (int32_t*)take(Hh * (((Mm + 127) / 128 + 1) / 2) * 4);
   w.pair_first = (int32_t*)take(Hh * 4);
+  w.head_order = (int32_t*)take(Hh * 4);
   w.loop_stride = (int64_t)(Hh * std::max((Mm + 127) / 128, (Nm + 127) / 128));
   w.loop_list = (int32_t*)take(3 * (size_t)w.loop_stride * 4);
   w.loop_ctr = (int32_t*)take(3 * 2 * 4);
@@ -374,13 +375,20 @@ dkv_status_t dkv_bank_create(dkv_bank_t* out, int32_t H, int32_t d, const int32_
     e = cudaMemcpy(bk->w.tile_head, tile_head.data(), sizeof(int32_t) * tile_head.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(bk->w.tile_first, tile_first.data(), sizeof(int32_t) * H, cudaMemcpyHostToDevice);
-  // pairs of those tiles (the units of the two-row-tile crossing pass)
-  std::vector<int32_t> pair_head, pair_first(H);
+  // pairs of those tiles (the units of the two-row-tile crossing pass); the heads by
+  // decreasing budget (the persistent score pass takes the largest units first, so that
+  // its fixed stride ends on small ones)
+  std::vector<int32_t> pair_head, pair_first(H), head_order(H);
   for (int h = 0; h < H; ++h) {
     pair_first[h] = (int32_t)pair_head.size();
     pair_head.insert(pair_head.end(), (size_t)((budgets[h] + 127) / 128 + 1) / 2, h);
+    head_order[h] = h;
   }
+  std::stable_sort(head_order.begin(), head_order.end(),
+                   [&](int32_t a, int32_t b) { return budgets[a] > budgets[b]; });
   bk->w.n_mpairs = (int)pair_head.size();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(bk->w.head_order, head_order.data(), sizeof(int32_t) * H, cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(bk->w.pair_head, pair_head.data(), sizeof(int32_t) * pair_head.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess)

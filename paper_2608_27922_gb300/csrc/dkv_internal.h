@@ -59,7 +59,7 @@ struct Ws {
   void* vevict;         // [H][n_max][d]  values of evicted states
   unsigned long long* sortbuf;   // [H][sort_stride] sorted runs of 256 sort keys
   float* invb;          // [H][invb_stride] 1 / b of the bank states (derived from the
-                        //   baselines, kept in step; 128 floats of padding at the end)
+                        //   baselines, kept in step; 256 floats of padding at the end)
   float* part;          // [2][H][part_stride] per-row partial sums of column-split passes
   int32_t* cnt;         // [H][cnt_stride] arrival counters of column-split row tiles (kept 0)
   int32_t* tile_head;   // [n_mtiles] head of each 128-row tile of the heads' budgets, head-major
@@ -69,6 +69,8 @@ struct Ws {
                         //   head): the units of the two-row-tile crossing pass
   int32_t* pair_first;  // [H] index of each head's first pair
   int n_mpairs;         // sum over heads of ceil(ceil(M_h / 128) / 2)
+  int32_t* head_order;  // [H] heads by decreasing budget, ties by index (the order of the
+                        //   persistent score pass's units: largest first)
   int32_t* loop_list;   // [3][loop_stride] row tiles with work of the persistent projection,
                         //   survivor and new-baseline passes (each its own: the last two run
                         //   side by side), appended by the pass's classification kernel

@@ -1122,6 +1122,261 @@ __global__ void __launch_bounds__(DU_THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- scores, 256-column tiles
+// Persistent form of the score pass (keys only) for grids of many candidate row tiles.
+// One CTA per SM takes candidate row tiles (units) at a fixed stride; each bank tile of
+// 256 columns is one MMA instruction per k-step (N = 256), so the row tile is read from
+// shared memory once per 256 columns instead of once per 128 and the issuing thread has
+// half the instructions per FLOP.  TMEM: two accumulators of 256 columns (all 512).  The
+// next unit's row tile loads into the second row-tile buffer during the current unit and
+// barrier phases run on across units (global tile count T).  Warps: 0 TMA producer, 1
+// MMA issuer, 2-17 the epilogue: warp w takes TMEM lane quarter w % 4 and the 64-column
+// quarter (w - 2) / 4 of each tile, in the 16x256b layout of the one-row-tile form.
+#ifndef DKV_SCORE_WIDE
+#define DKV_SCORE_WIDE 1
+#endif
+constexpr int SW_BN = 256;                         // columns per tile
+constexpr int SW_EPI = 16;
+constexpr int SW_THREADS = 64 + 32 * SW_EPI;
+constexpr int SW_STAGES = 2;                       // == accumulators (one barrier per stage)
+constexpr int SW_META = SW_STAGES + 3;             // weights ring (the argument of META_BUFS)
+constexpr int SW_APANEL = BM * 128;                // 64-column panel of the 128-row tile (16 KiB)
+constexpr int SW_BPANEL = SW_BN * 128;             // 64-column panel of the 256-row tile (32 KiB)
+constexpr int SW_BEXT = SW_BN * 32;                // 256 extension rows (8 KiB)
+
+struct LayW {
+  static constexpr int A = 0;                                    // [2 buffers][2 panels]
+  static constexpr int B = 2 * 2 * SW_APANEL;                    // [SW_STAGES][2 panels]
+  static constexpr int AX = B + SW_STAGES * 2 * SW_BPANEL;       // [2] row-form extensions
+  static constexpr int BX = AX + 2 * EXT_BYTES;                  // [SW_STAGES] column-form
+  static constexpr int META = BX + SW_STAGES * SW_BEXT;          // float [SW_META][SW_BN]
+  static constexpr int XF = META + SW_META * SW_BN * 4;          // float [4 column quarters][BM]
+  static constexpr int BAR = XF + 4 * BM * 4;
+  // a_full[2] a_free[2] empty[S] rdy[S] accf[2] meta[SW_META], then the TMEM holder and
+  // the abort flag
+  static constexpr int NBAR = 2 + 2 + 2 * SW_STAGES + 2 + SW_META;
+  static constexpr size_t SMEM = BAR + NBAR * 8 + 16;
+  static_assert(B % 1024 == 0 && AX % 1024 == 0 && BX % 256 == 0, "swizzled tiles need aligned bases");
+  static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+};
+
+// Unit u: candidate row tile u % tpn of the (u / tpn)-th head in order of decreasing
+// budget (the largest units first: the fixed stride then ends on small ones); the pass's
+// rows and bank columns.  False if the unit has no row.
+__device__ __forceinline__ bool wide_unit(const TcJob& j, int u, int& h, int& rt, int& nrows, int& c0, int& c1) {
+  h = j.w.head_order[u / j.tpn];
+  rt = u % j.tpn;
+  job_range(TM_SCORE, j.w.hd[h], *layer_of(j.w, h), nrows, c0, c1);
+  return rt * BM < nrows && c1 > c0;
+}
+
+template <int P>
+__global__ void __launch_bounds__(SW_THREADS, 1)
+    tc_score_wide(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAx,
+                  const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBx, TcJob j,
+                  int n_units) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0u) {
+    if (threadIdx.x == 0) dev_fail(j.w.L, DEV_INCONSISTENT, 9906);
+    return;
+  }
+  using LY = LayW;
+  float* meta = reinterpret_cast<float*>(smem + LY::META);
+  float* xf = reinterpret_cast<float*>(smem + LY::XF);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + LY::BAR);
+  uint64_t* a_full = bars + 0;                   // [2] row tile of a unit landed
+  uint64_t* a_free = bars + 2;                   // [2] MMAs of the buffer's last unit complete
+  uint64_t* bar_empty = bars + 4;                // [S] MMAs of the stage's tile complete
+  uint64_t* bar_rdy = bar_empty + SW_STAGES;     // [S] bank tile T landed (stage T & 1) and
+                                                 //   accumulator T & 1 released by all 16 warps
+  uint64_t* bar_accf = bar_rdy + SW_STAGES;      // [2] MMAs into the accumulator complete
+  uint64_t* bar_meta = bar_accf + 2;             // [SW_META] weights of tile T
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + LY::NBAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(a_full + i, 1);
+      mbar_init(a_free + i, 1);
+      mbar_init(bar_accf + i, 1);
+    }
+    for (int s = 0; s < SW_STAGES; ++s) {
+      mbar_init(bar_empty + s, 1);
+      mbar_init(bar_rdy + s, SW_EPI + 1);   // the epilogue warps + the producer (with bytes)
+    }
+    for (int q = 0; q < SW_META; ++q) mbar_init(bar_meta + q, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, DU_TMEM_COLS);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer
+      prefetch_map(&tmA); prefetch_map(&tmAx); prefetch_map(&tmB); prefetch_map(&tmBx);
+      int k = 0;
+      uint32_t T = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+        int h, rt, nrows, c0, c1;
+        if (!wide_unit(j, u, h, rt, nrows, c0, c1)) continue;
+        const int nt = (c1 - c0 + SW_BN - 1) / SW_BN;
+        const int a = k & 1;
+        if (!(ok = mbar_wait(a_free + a, ((k >> 1) & 1) ^ 1, abort_flag))) break;
+        mbar_arrive_expect_tx(a_full + a, 2 * SW_APANEL + EXT_BYTES);
+        for (int pn = 0; pn < 2; ++pn)
+          tma_load_3d(smem + LY::A + (2 * a + pn) * SW_APANEL, &tmA, a_full + a, pn * 64, rt * BM, h);
+        tma_load_3d(smem + LY::AX + a * EXT_BYTES, &tmAx, a_full + a, 0, rt * BM, h);
+        for (int t = 0; t < nt; ++t, ++T) {
+          const int s = (int)(T & 1);
+          if (!(ok = mbar_wait(bar_empty + s, ((T >> 1) & 1) ^ 1, abort_flag))) break;
+          mbar_arrive_expect_tx(bar_rdy + s, 2 * SW_BPANEL + SW_BEXT);
+          const int col = c0 + t * SW_BN;
+          for (int pn = 0; pn < 2; ++pn)
+            tma_load_3d(smem + LY::B + (2 * s + pn) * SW_BPANEL, &tmB, bar_rdy + s, pn * 64, col, h);
+          tma_load_3d(smem + LY::BX + s * SW_BEXT, &tmBx, bar_rdy + s, 16, col, h);
+          const int q = (int)(T % SW_META);
+          mbar_arrive_expect_tx(bar_meta + q, SW_BN * 4);
+          bulk_load(meta + q * SW_BN, j.w.invb + (int64_t)h * j.w.invb_stride + col, SW_BN * 4, bar_meta + q);
+        }
+        ++k;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.w.L, DEV_TIMEOUT, 150);
+        const uint64_t t0 = globaltimer_ns();   // copies may still land: a fixed 50 us
+        while (globaltimer_ns() - t0 < 50000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer: per bank tile 8 k-steps of N = 256 + 1 of the extension
+      constexpr uint32_t idesc = idesc_bf16(BM, SW_BN);
+      const uint64_t bd0 = desc_sw128(smem_u32(smem + LY::B));
+      const uint64_t bxd0 = desc_sw32(smem_u32(smem + LY::BX));
+      int k = 0;
+      uint32_t T = 0;
+      bool ok = true, any = false;
+      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+        int h, rt, nrows, c0, c1;
+        if (!wide_unit(j, u, h, rt, nrows, c0, c1)) continue;
+        const int nt = (c1 - c0 + SW_BN - 1) / SW_BN;
+        const int a = k & 1;
+        if (!(ok = mbar_wait(a_full + a, (k >> 1) & 1, abort_flag))) break;
+        const uint64_t ad = desc_sw128(smem_u32(smem + LY::A + 2 * a * SW_APANEL));
+        const uint64_t axd = desc_sw32(smem_u32(smem + LY::AX + a * EXT_BYTES));
+        for (int t = 0; t < nt; ++t, ++T) {
+          const int b = (int)(T & 1);   // stage and accumulator
+          if (!(ok = mbar_wait(bar_rdy + b, (T >> 1) & 1, abort_flag))) break;
+          fence_after_sync();
+          const uint64_t bd = desc_add(bd0, 2 * b * SW_BPANEL);
+          const uint32_t acc = tmem + (uint32_t)(b * SW_BN);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16(acc, desc_add(ad, (kk >> 2) * SW_APANEL + (kk & 3) * 32),
+                     desc_add(bd, (kk >> 2) * SW_BPANEL + (kk & 3) * 32), idesc, kk > 0);
+          mma_bf16(acc, axd, desc_add(bxd0, b * SW_BEXT), idesc, 1u);
+          mma_commit(bar_accf + b);
+          mma_commit(bar_empty + b);
+          any = true;
+        }
+        if (!ok) break;
+        mma_commit(a_free + a);
+        ++k;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        dev_fail(j.w.L, DEV_TIMEOUT, 250);
+      }
+      if (any) {   // every issued MMA complete before TMEM is freed
+        mma_commit(a_free + (k & 1));
+        volatile int no_abort = 0;
+        mbar_wait(a_free + (k & 1), (k >> 1) & 1, &no_abort);
+      }
+    }
+  } else {
+    // ---------------- epilogue: lane quarter q, columns [64 cq, 64 cq + 64) of each tile
+    const int ew = warp - 2;                      // 0..15
+    const int cq = ew >> 2;                       // column quarter
+    const int q = warp & 3;                       // TMEM lane quarter
+    const int r_local = q * 32 + lane;
+    const int bar_id = 1 + q;                     // the four warps of this lane quarter
+    const float c = pow_c<P>(j.kp);
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    if (lane == 0) {   // both accumulators start free: this warp's release for tiles 0 and 1
+      mbar_arrive(bar_rdy + 0);
+      mbar_arrive(bar_rdy + 1);
+    }
+    uint32_t T = 0;
+    bool ok = true;
+    // after a failed wait the warp keeps walking every unit and tile without work: the
+    // four warps of a lane quarter must meet at the same named barriers
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+      int h, rt, nrows, c0, c1;
+      if (!wide_unit(j, u, h, rt, nrows, c0, c1)) continue;
+      const int nt = (c1 - c0 + SW_BN - 1) / SW_BN;
+      float2 sacc[4];   // rows lane/4 + 8 jj of the quarter (16x256b layout)
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) sacc[jj] = make_float2(0.f, 0.f);
+      for (int t = 0; t < nt; ++t, ++T) {
+        const int b = (int)(T & 1);
+        const int col0 = c0 + t * SW_BN;
+        const int nc = min(SW_BN, c1 - col0);
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_accf + b, (T >> 1) & 1, abort_flag));
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar_meta + T % SW_META, (T / SW_META) & 1, abort_flag));
+        if (!ok) {
+          *abort_flag = 1;
+          continue;
+        }
+        fence_after_sync();
+        const int cs = 64 * cq;
+        if (cs < nc) {   // warp-uniform
+          float va[32], vb[32];
+          tmem_ld16x256b_x8(lane_base + b * SW_BN + cs, va);
+          tmem_ld16x256b_x8(lane_base + (16u << 16) + b * SW_BN + cs, vb);
+          tmem_wait_ld();
+          fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_rdy + b);   // accumulator b free for tile T + 2
+          score_rows4<P>(va, vb, meta + (T % SW_META) * SW_BN + cs, nc - cs, 2 * (lane & 3), sacc);
+        } else {
+          fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_rdy + b);
+        }
+      }
+      // unit end: the four column quarters of each row, added in quarter order; a second
+      // barrier keeps the next unit's sums from being written before every warp has read
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        float x = sacc[jj].x + sacc[jj].y;
+        x += __shfl_xor_sync(0xffffffffu, x, 1);
+        x += __shfl_xor_sync(0xffffffffu, x, 2);
+        if ((lane & 3) == 0) xf[cq * BM + q * 32 + (lane >> 2) + 8 * jj] = P == 1 ? -x : x;
+      }
+      named_bar(bar_id, 128);
+      const float acc = ((xf[r_local] + xf[BM + r_local]) + xf[2 * BM + r_local]) + xf[3 * BM + r_local];
+      named_bar(bar_id, 128);
+      const int row = rt * BM + r_local;
+      if (ok && cq == 0 && row < nrows)
+        j.w.score[(int64_t)h * j.b.n_max + row] = (acc * c) / (float)j.w.hd[h].m_old;
+    }
+    if (!ok && lane == 0) dev_fail(j.w.L, DEV_TIMEOUT, 350);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after_sync();
+    tmem_dealloc(tmem, DU_TMEM_COLS);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -1286,6 +1541,11 @@ cudaError_t tc_set_smem_limits() {
     e = cudaFuncSetAttribute(tc_cross_dual<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LayC::SMEM);
   DKV_OPTD(1) DKV_OPTD(2) DKV_OPTD(4)
 #undef DKV_OPTD
+#define DKV_OPTW(P)                                                                                           \
+  if (e == cudaSuccess)                                                                                        \
+    e = cudaFuncSetAttribute(tc_score_wide<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LayW::SMEM);
+  DKV_OPTW(1) DKV_OPTW(2) DKV_OPTW(4)
+#undef DKV_OPTW
 #undef DKV_OPTLOOP
 #undef DKV_OPTL
 #undef DKV_OPT
@@ -1307,10 +1567,24 @@ cudaError_t launch_score_tc(const Bank& b, const Ws& w, const void* Kc, const vo
   // candidate array of the workspace, [H][n_max][32].  The bank columns are split over two
   // CTAs per row tile while the row tiles alone would not fill the GPU several times over
   int split = DKV_SCORE_SPLIT;
-  if (split == 0) {
-    const int n_sm = sm_count();
-    const int64_t ctas = (int64_t)((N + BM - 1) / BM) * b.H;
-    split = n_sm > 0 && ctas >= 16 * (int64_t)n_sm ? 1 : 2;
+  const int n_sm = sm_count();
+  const int64_t ctas = (int64_t)((N + BM - 1) / BM) * b.H;
+  if (split == 0) split = n_sm > 0 && ctas >= 16 * (int64_t)n_sm ? 1 : 2;
+  if (DKV_SCORE_WIDE && split == 1 && !kv && n_sm > 0) {
+    // the persistent 256-column form over the many row tiles
+    CUtensorMap ma, max_, mb, mbx;
+    if (!make_map_rows(&ma, Kc, N, b.H, BM) || !make_map_ext(&max_, w.cext, b.n_max, b.H, BM) ||
+        !make_map_rows(&mb, b.k, b.M_max, b.H, SW_BN) || !make_map_ext(&mbx, w.bext, b.M_max, b.H, SW_BN))
+      return cudaErrorInvalidValue;
+    const int tpn = (N + BM - 1) / BM;
+    TcJob job{b, w, kp, 0, tpn};
+    const int n_units = (int)ctas;
+    timer_begin(t, "score_tc", s);
+    if (kp.p == 1) tc_score_wide<1><<<n_sm, SW_THREADS, LayW::SMEM, s>>>(ma, max_, mb, mbx, job, n_units);
+    else if (kp.p == 4) tc_score_wide<4><<<n_sm, SW_THREADS, LayW::SMEM, s>>>(ma, max_, mb, mbx, job, n_units);
+    else tc_score_wide<2><<<n_sm, SW_THREADS, LayW::SMEM, s>>>(ma, max_, mb, mbx, job, n_units);
+    timer_end(t, s);
+    return cudaGetLastError();
   }
   return launch_tc<TM_SCORE>(b, w, kp, Kc, w.cext, N, b.k, w.bext, b.M_max, N, s, t, "score_tc", split,
                              kv ? Vc : nullptr, kv ? b.v : nullptr, b.n_max);
