@@ -52,6 +52,9 @@ UNIT = "keys/s"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# GB300's nominal dense bf16 tensor rate and HBM3e bandwidth: fractions are also given
+# against these, beside the measured peaks above
+NOMINAL_BF16_TFLOPS, NOMINAL_HBM_GBS = 2250.0, 8000.0
 
 
 def parse_args():
@@ -652,6 +655,7 @@ def run_ours(args):
         peak = float(pk["bf16_tflops"])
         roof = {"kernel": dom_name, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "peak_source": f"{pk_src} bf16 dense (burst)",
+                "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
                 "algorithmic_per_launch": {"flops": flops, "keys_per_query": m_bank + wl.W},
                 "traffic": traffic_for(dom_name, ["k_tc_attn.cu", "tc_ptx.cuh"], wl.name, wl.H)}
     else:
@@ -1042,10 +1046,10 @@ def run_stack(args):
         row = {"launches": e["launches"], "avg_ms": e["ms"] / e["launches"], "share": e["ms"] / tot_prof}
         if name in TENSOR_KERNELS:
             tf = e["work"] / (e["ms"] / 1e3) / 1e12
-            row.update(tflops=tf, frac_of_bf16_peak=tf / tpeak)
+            row.update(tflops=tf, frac_of_bf16_peak=tf / tpeak, frac_of_bf16_nominal=tf / NOMINAL_BF16_TFLOPS)
         elif name in HBM_KERNELS:
             gbs = e["work"] / (e["ms"] / 1e3) / 1e9
-            row.update(alg_gbs=gbs, frac_of_hbm_alg=gbs / hpeak,
+            row.update(alg_gbs=gbs, frac_of_hbm_alg=gbs / hpeak, frac_of_hbm_alg_nominal=gbs / NOMINAL_HBM_GBS,
                        moved_gbs=e["moved"] / (e["ms"] / 1e3) / 1e9, frac_of_hbm_moved=e["moved"] / (e["ms"] / 1e3) / 1e9 / hpeak)
         per_kernel[name] = row
 
@@ -1168,7 +1172,8 @@ def run_stack(args):
                 "algorithmic_per_launch": {"flops": att_flops}, "traffic": None}
         if att_n:
             ach = att_flops / (att_ms / att_n / 1e3) / 1e12
-            roof.update(achieved=ach, frac=ach / tpeak, launches=att_n, avg_ms=att_ms / att_n,
+            roof.update(achieved=ach, frac=ach / tpeak, frac_of_nominal=ach / NOMINAL_BF16_TFLOPS,
+                        launches=att_n, avg_ms=att_ms / att_n,
                         traffic=traffic_for("attend_tc", ["k_tc_attn.cu", "tc_ptx.cuh"], wl.name, LH))
         admitting = [sum(1 for r in s["r_star"] if r > 0) for s in per_step]
         line = {

@@ -430,3 +430,15 @@ def test_many_heads_sort_schedule(dkv):
     # N > M: r* = M < N, so near-tied scores at the admission cut-off may swap a candidate
     # (explained by check_report); only a few heads may differ
     assert all(r.heads_set_differs <= wl.H // 20 for r in reps), [r.heads_set_differs for r in reps]
+
+
+@pytest.mark.parametrize("p,sigma,tau", [(1.0, 8.0, 2.0), (4.0, 16.0, 1.5)])
+def test_many_heads_other_exponents(dkv, p, sigma, tau):
+    """The many-row-tile score pass (2,560 candidate row tiles, bank columns unsplit) at
+    the other exponents of Table 2a: the empty-bank block, then one block scored against
+    full banks of 640 (two and a half 256-column bank tiles) and evicting (a block is
+    admitted one step after its own, when it leaves the window)."""
+    wl = synth.get_workload("wan13b_layer_h12", H=256, N=1280, W=64, Nq=64, budgets=640, steps=3)
+    reps = _rollout(dkv, wl, "tc", check_attn=False, p=p, sigma=sigma, tau=tau)
+    assert len(reps) == 2
+    assert all(r.heads_set_differs <= wl.H // 20 for r in reps), [r.heads_set_differs for r in reps]
