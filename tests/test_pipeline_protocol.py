@@ -1,0 +1,387 @@
+"""Host model of the mbarrier protocol of the persistent tensor-core passes.
+
+The persistent score pass (one 128-row candidate tile per unit, 256-column bank tiles)
+and the persistent crossing pass (two 128-row bank tiles per unit, 128-column candidate
+tiles) each run one TMA-producer thread, one MMA-issuing thread and 16 epilogue warps
+that meet only at mbarriers, whose phases run on across units.  A mistake there shows up
+on the GPU as a hang or an exception, not as a wrong number, so the protocol is replayed
+here on the host:
+
+- every barrier keeps its completed-phase count, pending arrivals and transaction bytes
+  (a phase completes when both reach zero), and every arrival and every landed copy
+  names the phase it is meant for: one that lands in an earlier, still open phase would
+  complete that phase early;
+- a waiter waits for the completion of one phase (the kernels' parity waits) and must
+  not find the barrier two phases on;
+- the producer, the issuer and the epilogue warps are generator actors interleaved at
+  random; copies land at random later points, in any order; MMAs and tcgen05 commits
+  complete at random later points, in issue order;
+- no shared-memory stage, row-tile buffer, weight slot or TMEM accumulator is written
+  while a reader still needs it, and every reader finds the tile it expects;
+- every run ends (no deadlock), and every epilogue warp sees every tile in order.
+
+Two planted variants must be caught: four column stages with the combined "tile landed
+and accumulator free" barrier still indexed by accumulator (the form that raised a GPU
+exception: the producer arms the barrier for tile T + 2 while tile T's phase is open),
+and an epilogue that releases its accumulator before its TMEM loads are done.
+"""
+import random
+
+import pytest
+
+
+class ProtocolError(AssertionError):
+    pass
+
+
+class Bar:
+    """One mbarrier: `count` arrivals and the expected transaction bytes per phase."""
+
+    def __init__(self, name, count):
+        self.name, self.count = name, count
+        self.pending, self.tx, self.phase = count, 0, 0
+
+    def _own(self, idx, what):
+        if idx != self.phase:
+            raise ProtocolError(f"{what} on {self.name} meant for phase {idx} while phase {self.phase} is open")
+
+    def _settle(self):
+        if self.pending == 0 and self.tx == 0:
+            self.phase += 1
+            self.pending = self.count
+
+    def arrive(self, idx, tx=0):
+        self._own(idx, "arrival")
+        self.tx += tx
+        self.pending -= 1
+        self._settle()
+
+    def land(self, idx, nbytes):
+        self._own(idx, "copy")
+        self.tx -= nbytes
+        if self.tx < 0:
+            raise ProtocolError(f"{self.name}: more bytes landed than expected")
+        self._settle()
+
+    def passed(self, idx):
+        """A parity wait for the completion of phase idx (-1: the phase before the first)."""
+        if self.phase > idx + 1:
+            raise ProtocolError(f"{self.name} completed phase {self.phase - 1} before its waiter for phase {idx}")
+        return self.phase == idx + 1
+
+
+class Sim:
+    """Random interleaving of actors (generators yielding None, or (bar, phase) to wait)
+    with the asynchronous copies and the in-order tensor-core queue."""
+
+    def __init__(self, rng):
+        self.rng = rng
+        self.copies = []   # (bar, phase, bytes, on_land)
+        self.tc = []       # ("mma", fn) / ("commit", bar, phase), in issue order
+
+    def copy(self, bar, idx, nbytes, on_land):
+        self.copies.append((bar, idx, nbytes, on_land))
+
+    def run(self, actors, max_events=2_000_000):
+        cond = {i: None for i in range(len(actors))}
+        live = set(range(len(actors)))
+        for _ in range(max_events):
+            if not live and not self.copies and not self.tc:
+                return
+            ready = [i for i in sorted(live) if cond[i] is None or cond[i][0].passed(cond[i][1])]
+            n = len(ready) + len(self.copies) + (1 if self.tc else 0)
+            if n == 0:
+                waits = {i: (cond[i][0].name, cond[i][1]) for i in live}
+                raise ProtocolError(f"deadlock: {waits}")
+            pick = self.rng.randrange(n)
+            if pick < len(ready):
+                i = ready[pick]
+                try:
+                    cond[i] = next(actors[i])
+                except StopIteration:
+                    live.discard(i)
+            elif pick < len(ready) + len(self.copies):
+                bar, idx, nbytes, on_land = self.copies.pop(pick - len(ready))
+                on_land()
+                bar.land(idx, nbytes)
+            else:
+                op = self.tc.pop(0)
+                if op[0] == "mma":
+                    op[1]()
+                else:
+                    op[1].arrive(op[2])
+        raise ProtocolError("no end after the event limit")
+
+
+EPI = 16   # epilogue warps of both persistent kernels
+
+
+def score_wide_model(sim, units, stages=2, meta_slots=5, release_early=False):
+    """The score pass with 256-column bank tiles: units = bank tiles per candidate row
+    tile (0 for an empty bank; the row tile is still loaded and its buffer released)."""
+    A, B, M = 36864, 73728, 1024          # row tile + extension, bank tile + extension, 1/b weights
+    a_full = [Bar(f"a_full{i}", 1) for i in range(2)]
+    a_free = [Bar(f"a_free{i}", 1) for i in range(2)]
+    empty = [Bar(f"empty{s}", 1) for s in range(stages)]
+    rdy = [Bar(f"rdy{b}", EPI + 1) for b in range(2)]     # indexed by accumulator T & 1
+    accf = [Bar(f"accf{b}", 1) for b in range(2)]
+    meta = [Bar(f"meta{q}", 1) for q in range(meta_slots)]
+    st = dict(a_loaded=[-1, -1], a_reads=[0, 0], b_loaded=[-1] * stages, b_reads=[0] * stages,
+              acc_tile=[-1, -1], acc_reading=[0, 0], meta_loaded=[-1] * meta_slots,
+              meta_reading=[0] * meta_slots, released=[-1] * EPI, seen=[[] for _ in range(EPI)])
+
+    def setter(key, i, v):
+        return lambda: st[key].__setitem__(i, v)
+
+    def producer():
+        k = T = 0
+        for nt in units:
+            a = k & 1
+            yield (a_free[a], (k >> 1) - 1)
+            if st["a_reads"][a]:
+                raise ProtocolError("row-tile buffer reloaded while MMAs read it")
+            a_full[a].arrive(k >> 1, tx=A)
+            sim.copy(a_full[a], k >> 1, A, setter("a_loaded", a, k))
+            for _ in range(nt):
+                s = T % stages
+                yield (empty[s], T // stages - 1)
+                if st["b_reads"][s]:
+                    raise ProtocolError("bank-tile stage reloaded while MMAs read it")
+                rdy[T & 1].arrive(T >> 1, tx=B)
+                sim.copy(rdy[T & 1], T >> 1, B, setter("b_loaded", s, T))
+                q = T % meta_slots
+                if st["meta_reading"][q]:
+                    raise ProtocolError("weight slot reloaded while an epilogue warp reads it")
+                meta[q].arrive(T // meta_slots, tx=M)
+                sim.copy(meta[q], T // meta_slots, M, setter("meta_loaded", q, T))
+                T += 1
+                yield None
+            k += 1
+
+    def mma(a, s, b, T):
+        def run():
+            if st["acc_reading"][b]:
+                raise ProtocolError("accumulator overwritten while an epilogue warp reads it")
+            st["acc_tile"][b] = T
+            st["a_reads"][a] -= 1
+            st["b_reads"][s] -= 1
+        return run
+
+    def issuer():
+        k = T = 0
+        issued = False
+        for nt in units:
+            a = k & 1
+            yield (a_full[a], k >> 1)
+            if st["a_loaded"][a] != k:
+                raise ProtocolError("MMAs issued on a row tile that has not landed")
+            for _ in range(nt):
+                b, s = T & 1, T % stages
+                yield (rdy[b], T >> 1)
+                if st["b_loaded"][s] != T:
+                    raise ProtocolError(f"MMAs of tile {T} issued before its bank tile landed")
+                if T >= 2 and min(st["released"]) < T - 2:
+                    raise ProtocolError("accumulator reused before every epilogue warp released it")
+                st["a_reads"][a] += 1
+                st["b_reads"][s] += 1
+                sim.tc.append(("mma", mma(a, s, b, T)))
+                sim.tc.append(("commit", accf[b], T >> 1))
+                sim.tc.append(("commit", empty[s], T // stages))
+                issued = True
+                T += 1
+                yield None
+            sim.tc.append(("commit", a_free[a], k >> 1))
+            k += 1
+        if issued:   # every MMA complete before TMEM is freed
+            sim.tc.append(("commit", a_free[k & 1], k >> 1))
+            yield (a_free[k & 1], k >> 1)
+
+    def epilogue(w):
+        rdy[0].arrive(0)
+        rdy[1].arrive(0)
+        T = 0
+        for nt in units:
+            for _ in range(nt):
+                b, q = T & 1, T % meta_slots
+                yield (accf[b], T >> 1)
+                yield (meta[q], T // meta_slots)
+                if st["acc_tile"][b] != T:
+                    raise ProtocolError(f"warp {w} finds tile {st['acc_tile'][b]} in the accumulator of tile {T}")
+                if release_early:
+                    st["released"][w] = T
+                    rdy[b].arrive((T >> 1) + 1)
+                st["acc_reading"][b] += 1
+                yield None                               # TMEM loads in flight
+                st["acc_reading"][b] -= 1
+                if not release_early:
+                    st["released"][w] = T
+                    rdy[b].arrive((T >> 1) + 1)          # accumulator b free for tile T + 2
+                if st["meta_loaded"][q] != T:
+                    raise ProtocolError(f"warp {w} reads the weights of tile {st['meta_loaded'][q]} for tile {T}")
+                st["meta_reading"][q] += 1
+                yield None
+                st["meta_reading"][q] -= 1
+                st["seen"][w].append(T)
+                T += 1
+
+    actors = [producer(), issuer()] + [epilogue(w) for w in range(EPI)]
+    sim.run(actors)
+    total = sum(units)
+    assert all(s == list(range(total)) for s in st["seen"])
+
+
+def cross_dual_model(sim, units, stages=2):
+    """The crossing pass, two row tiles per unit: units = (candidate tiles, second row
+    tile present) (0 tiles: no column, the producer and issuer skip the unit)."""
+    TILE, EXT = 32768, 4096
+    a_full = [Bar(f"a_full{i}", 1) for i in range(2)]
+    a_free = [Bar(f"a_free{i}", 1) for i in range(2)]
+    empty = [Bar(f"empty{s}", 1) for s in range(stages)]
+    rdy = [Bar(f"rdy{b}", EPI + 1) for b in range(2)]      # indexed by accumulator T & 1
+    accf = [[Bar(f"accf{r}{b}", 1) for b in range(2)] for r in range(2)]
+    st = dict(a_loaded=[-1, -1], a_reads=[0, 0], b_loaded=[-1] * stages, b_reads=[0] * stages,
+              acc_tile=[[-1, -1], [-1, -1]], acc_reading=[[0, 0], [0, 0]], released=[-1] * EPI,
+              seen=[[] for _ in range(EPI)])
+
+    def setter(key, i, v):
+        return lambda: st[key].__setitem__(i, v)
+
+    def producer():
+        k = T = 0
+        for nt, two in units:
+            if nt == 0:
+                continue
+            a = k & 1
+            yield (a_free[a], (k >> 1) - 1)
+            if st["a_reads"][a]:
+                raise ProtocolError("row-tile buffer reloaded while MMAs read it")
+            nb = (2 if two else 1) * (TILE + EXT)
+            a_full[a].arrive(k >> 1, tx=nb)
+            sim.copy(a_full[a], k >> 1, nb, setter("a_loaded", a, k))
+            for _ in range(nt):
+                s = T % stages
+                yield (empty[s], T // stages - 1)
+                if st["b_reads"][s]:
+                    raise ProtocolError("column-tile stage reloaded while MMAs read it")
+                rdy[T & 1].arrive(T >> 1, tx=TILE + EXT)
+                sim.copy(rdy[T & 1], T >> 1, TILE + EXT, setter("b_loaded", s, T))
+                T += 1
+                yield None
+            k += 1
+
+    def mma(a, s, r, b, T):
+        def run():
+            if st["acc_reading"][r][b]:
+                raise ProtocolError("accumulator overwritten while an epilogue warp reads it")
+            st["acc_tile"][r][b] = T
+            st["a_reads"][a] -= 1
+            st["b_reads"][s] -= 1
+        return run
+
+    def issuer():
+        k = T = 0
+        issued = False
+        for nt, two in units:
+            if nt == 0:
+                continue
+            a = k & 1
+            yield (a_full[a], k >> 1)
+            if st["a_loaded"][a] != k:
+                raise ProtocolError("MMAs issued on row tiles that have not landed")
+            for _ in range(nt):
+                b, s = T & 1, T % stages
+                yield (rdy[b], T >> 1)
+                if st["b_loaded"][s] != T:
+                    raise ProtocolError(f"MMAs of tile {T} issued before its column tile landed")
+                if T >= 2 and min(st["released"]) < T - 2:
+                    raise ProtocolError("accumulator reused before every epilogue warp released it")
+                for r in range(2):
+                    if r == 0 or two:
+                        st["a_reads"][a] += 1
+                        st["b_reads"][s] += 1
+                        sim.tc.append(("mma", mma(a, s, r, b, T)))
+                    sim.tc.append(("commit", accf[r][b], T >> 1))   # an absent row tile: at once
+                sim.tc.append(("commit", empty[s], T // stages))
+                issued = True
+                T += 1
+                yield None
+            sim.tc.append(("commit", a_free[a], k >> 1))
+            k += 1
+        if issued:
+            sim.tc.append(("commit", a_free[k & 1], k >> 1))
+            yield (a_free[k & 1], k >> 1)
+
+    def epilogue(w):
+        r = w // 8   # row tile of the unit
+        rdy[0].arrive(0)
+        rdy[1].arrive(0)
+        T = 0
+        for nt, two in units:
+            live = r == 0 or two
+            for _ in range(nt):
+                b = T & 1
+                yield (accf[r][b], T >> 1)
+                if live:
+                    if st["acc_tile"][r][b] != T:
+                        raise ProtocolError(f"warp {w} finds tile {st['acc_tile'][r][b]} for tile {T}")
+                    st["acc_reading"][r][b] += 1
+                    yield None                           # TMEM loads, chunk sums, exchange
+                    st["acc_reading"][r][b] -= 1
+                st["released"][w] = T
+                rdy[b].arrive((T >> 1) + 1)
+                st["seen"][w].append(T)
+                T += 1
+
+    actors = [producer(), issuer()] + [epilogue(w) for w in range(EPI)]
+    sim.run(actors)
+    total = sum(nt for nt, _ in units)
+    assert all(s == list(range(total)) for s in st["seen"])
+
+
+def _score_units(rng):
+    return [rng.choice([0, 1, 1, 2, 3, 5]) for _ in range(rng.randrange(1, 8))]
+
+
+def _cross_units(rng):
+    return [(rng.choice([0, 1, 2, 3, 4, 7]), rng.random() < 0.7) for _ in range(rng.randrange(1, 7))]
+
+
+@pytest.mark.parametrize("seed", range(60))
+def test_score_pass_protocol(seed):
+    rng = random.Random(seed)
+    score_wide_model(Sim(rng), _score_units(rng))
+
+
+@pytest.mark.parametrize("seed", range(60))
+def test_crossing_pass_protocol(seed):
+    rng = random.Random(1000 + seed)
+    cross_dual_model(Sim(rng), _cross_units(rng))
+
+
+def test_long_units_both_passes():
+    rng = random.Random(7)
+    score_wide_model(Sim(rng), [0, 9, 1, 0, 12, 2])
+    cross_dual_model(Sim(rng), [(9, True), (0, True), (1, False), (12, True), (2, False)])
+
+
+def _caught(fn, seeds):
+    for seed in seeds:
+        try:
+            fn(seed)
+        except ProtocolError:
+            return True
+    return False
+
+
+def test_planted_four_stages_with_accumulator_barrier_is_caught():
+    """Four column stages, the combined barrier still one per accumulator: the producer,
+    up to four tiles ahead, arms the barrier of tile T + 2 while tile T's phase is open."""
+    assert _caught(lambda s: cross_dual_model(Sim(random.Random(s)), [(8, True), (6, False)], stages=4),
+                   range(40))
+    assert _caught(lambda s: score_wide_model(Sim(random.Random(s)), [8, 6], stages=4), range(40))
+
+
+def test_planted_early_release_is_caught():
+    """An epilogue warp that frees its accumulator before its TMEM loads are done lets
+    the MMAs of tile T + 2 overwrite what it still reads."""
+    assert _caught(lambda s: score_wide_model(Sim(random.Random(s)), [6, 5], release_early=True), range(60))
