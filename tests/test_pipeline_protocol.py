@@ -3,7 +3,9 @@
 The persistent score pass (one 128-row candidate tile per unit, 256-column bank tiles)
 and the persistent crossing pass (two 128-row bank tiles per unit, 128-column candidate
 tiles) each run one TMA-producer thread, one MMA-issuing thread and 16 epilogue warps
-that meet only at mbarriers, whose phases run on across units.  A mistake there shows up
+that meet only at mbarriers, whose phases run on across units.  The persistent
+projection, survivor and new-baseline passes initialise their barriers again for every
+unit, so each unit must end with nothing in flight.  A mistake there shows up
 on the GPU as a hang or an exception, not as a wrong number, so the protocol is replayed
 here on the host:
 
@@ -20,10 +22,12 @@ here on the host:
   while a reader still needs it, and every reader finds the tile it expects;
 - every run ends (no deadlock), and every epilogue warp sees every tile in order.
 
-Two planted variants must be caught: four column stages with the combined "tile landed
-and accumulator free" barrier still indexed by accumulator (the form that raised a GPU
-exception: the producer arms the barrier for tile T + 2 while tile T's phase is open),
-and an epilogue that releases its accumulator before its TMEM loads are done.
+Three planted variants must be caught: four column stages with the combined "tile
+landed and accumulator free" barrier still indexed by accumulator (the form that raised
+a GPU exception: the producer arms the barrier for tile T + 2 while tile T's phase is
+open), an epilogue that releases its accumulator before its TMEM loads are done, and,
+in the re-initialising passes, a tile's two MMA commits issued in the other order (the
+stage barrier's commit then outlives the unit).
 """
 import random
 
@@ -82,11 +86,13 @@ class Sim:
     def copy(self, bar, idx, nbytes, on_land):
         self.copies.append((bar, idx, nbytes, on_land))
 
-    def run(self, actors, max_events=2_000_000):
+    def run(self, actors, max_events=2_000_000, drain=True):
+        """drain=False: return once every actor has finished (a CTA-wide barrier), with
+        whatever copies and commits are still in flight."""
         cond = {i: None for i in range(len(actors))}
         live = set(range(len(actors)))
         for _ in range(max_events):
-            if not live and not self.copies and not self.tc:
+            if not live and (not drain or (not self.copies and not self.tc)):
                 return
             ready = [i for i in sorted(live) if cond[i] is None or cond[i][0].passed(cond[i][1])]
             n = len(ready) + len(self.copies) + (1 if self.tc else 0)
@@ -338,6 +344,93 @@ def cross_dual_model(sim, units, stages=2):
     assert all(s == list(range(total)) for s in st["seen"])
 
 
+def pairs_loop_model(sim, units, stages=2, accf_first=False):
+    """The persistent projection / survivor / new-baseline passes: a CTA takes units (one
+    128-row tile, `nt` column tiles) one after the other and initialises its barriers
+    again for every unit, after a CTA-wide barrier; so when every thread has left a unit,
+    no copy and no MMA commit may still be in flight (it would land in a barrier of the
+    next unit).  Eight epilogue warps; the row-sum passes free an accumulator after their
+    last TMEM load of the tile."""
+    LOAD = 36864
+    warps = 8
+    for u, nt in enumerate(units):
+        bar_a = Bar(f"u{u}.a", 1)
+        empty = [Bar(f"u{u}.empty{s}", 1) for s in range(stages)]
+        rdy = [Bar(f"u{u}.rdy{b}", warps + 1) for b in range(2)]
+        accf = [Bar(f"u{u}.accf{b}", 1) for b in range(2)]
+        st = dict(b_loaded=[-1] * stages, b_reads=[0] * stages, acc_tile=[-1, -1], acc_reading=[0, 0],
+                  released=[-1] * warps, seen=[[] for _ in range(warps)], a_loaded=False)
+
+        def setter(i, v, st=st):
+            return lambda: st["b_loaded"].__setitem__(i, v)
+
+        def producer(nt=nt, st=st, bar_a=bar_a, empty=empty, rdy=rdy):
+            bar_a.arrive(0, tx=LOAD)
+            sim.copy(bar_a, 0, LOAD, lambda: st.__setitem__("a_loaded", True))
+            for t in range(nt):
+                s = t % stages
+                yield (empty[s], t // stages - 1)
+                if st["b_reads"][s]:
+                    raise ProtocolError("column-tile stage reloaded while MMAs read it")
+                rdy[t & 1].arrive(t >> 1, tx=LOAD)
+                sim.copy(rdy[t & 1], t >> 1, LOAD, setter(s, t))
+                yield None
+            # never leave with copies in flight: the row tile, then the last stages' tiles
+            yield (bar_a, 0)
+            for t in range(max(0, nt - stages), nt):
+                yield (rdy[t & 1], t >> 1)
+
+        def mma(s, b, t, st=st):
+            def run():
+                if st["acc_reading"][b]:
+                    raise ProtocolError("accumulator overwritten while an epilogue warp reads it")
+                st["acc_tile"][b] = t
+                st["b_reads"][s] -= 1
+            return run
+
+        def issuer(nt=nt, st=st, bar_a=bar_a, empty=empty, rdy=rdy, accf=accf):
+            yield (bar_a, 0)
+            if not st["a_loaded"]:
+                raise ProtocolError("MMAs issued on a row tile that has not landed")
+            for t in range(nt):
+                s, b = t % stages, t & 1
+                yield (rdy[b], t >> 1)
+                if st["b_loaded"][s] != t:
+                    raise ProtocolError(f"MMAs of tile {t} issued before its column tile landed")
+                if t >= 2 and min(st["released"]) < t - 2:
+                    raise ProtocolError("accumulator reused before every epilogue warp released it")
+                st["b_reads"][s] += 1
+                sim.tc.append(("mma", mma(s, b, t)))
+                commits = [("commit", empty[s], t // stages), ("commit", accf[b], t >> 1)]
+                sim.tc.extend(commits[::-1] if accf_first else commits)
+                yield None
+            if nt > 0:   # every MMA complete before the unit ends
+                yield (accf[(nt - 1) & 1], (nt - 1) >> 1)
+
+        def epilogue(w, nt=nt, st=st, rdy=rdy, accf=accf):
+            rdy[0].arrive(0)
+            rdy[1].arrive(0)
+            for t in range(nt):
+                b = t & 1
+                yield (accf[b], t >> 1)
+                if st["acc_tile"][b] != t:
+                    raise ProtocolError(f"warp {w} finds tile {st['acc_tile'][b]} for tile {t}")
+                st["acc_reading"][b] += 1
+                yield None                               # the tile's TMEM loads
+                st["acc_reading"][b] -= 1
+                st["released"][w] = t
+                rdy[b].arrive((t >> 1) + 1)              # then the chunk arithmetic
+                yield None
+                st["seen"][w].append(t)
+
+        actors = [producer(), issuer()] + [epilogue(w) for w in range(warps)]
+        sim.run(actors, drain=False)
+        if sim.copies or sim.tc:
+            raise ProtocolError(f"unit {u} ends with {len(sim.copies)} copies and {len(sim.tc)} "
+                                f"tensor-core operations in flight; its barriers are initialised again")
+        assert all(x == list(range(nt)) for x in st["seen"])
+
+
 def _score_units(rng):
     return [rng.choice([0, 1, 1, 2, 3, 5]) for _ in range(rng.randrange(1, 8))]
 
@@ -356,6 +449,12 @@ def test_score_pass_protocol(seed):
 def test_crossing_pass_protocol(seed):
     rng = random.Random(1000 + seed)
     cross_dual_model(Sim(rng), _cross_units(rng))
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_persistent_row_passes_protocol(seed):
+    rng = random.Random(2000 + seed)
+    pairs_loop_model(Sim(rng), [rng.randrange(1, 7) for _ in range(rng.randrange(1, 6))])
 
 
 def test_long_units_both_passes():
@@ -379,6 +478,13 @@ def test_planted_four_stages_with_accumulator_barrier_is_caught():
     assert _caught(lambda s: cross_dual_model(Sim(random.Random(s)), [(8, True), (6, False)], stages=4),
                    range(40))
     assert _caught(lambda s: score_wide_model(Sim(random.Random(s)), [8, 6], stages=4), range(40))
+
+
+def test_planted_commit_order_is_caught():
+    """The last waits of a unit are on the accumulator barrier of its last tile (the
+    epilogue's and the issuer's); with that tile's two commits issued accumulator first,
+    the stage barrier's commit can still be in flight when the next unit initialises it."""
+    assert _caught(lambda s: pairs_loop_model(Sim(random.Random(s)), [3, 2], accf_first=True), range(300))
 
 
 def test_planted_early_release_is_caught():
