@@ -5,7 +5,9 @@ and the persistent crossing pass (two 128-row bank tiles per unit, 128-column ca
 tiles) each run one TMA-producer thread, one MMA-issuing thread and 16 epilogue warps
 that meet only at mbarriers, whose phases run on across units.  The persistent
 projection, survivor and new-baseline passes initialise their barriers again for every
-unit, so each unit must end with nothing in flight.  A mistake there shows up
+unit, so each unit must end with nothing in flight.  The attention kernel with two query
+tiles per CTA runs a producer, the issuing thread and two softmax groups whose S, P and
+O live in TMEM.  A mistake there shows up
 on the GPU as a hang or an exception, not as a wrong number, so the protocol is replayed
 here on the host:
 
@@ -22,12 +24,13 @@ here on the host:
   while a reader still needs it, and every reader finds the tile it expects;
 - every run ends (no deadlock), and every epilogue warp sees every tile in order.
 
-Three planted variants must be caught: four column stages with the combined "tile
+Four planted variants must be caught: four column stages with the combined "tile
 landed and accumulator free" barrier still indexed by accumulator (the form that raised
 a GPU exception: the producer arms the barrier for tile T + 2 while tile T's phase is
-open), an epilogue that releases its accumulator before its TMEM loads are done, and,
-in the re-initialising passes, a tile's two MMA commits issued in the other order (the
-stage barrier's commit then outlives the unit).
+open), an epilogue that releases its accumulator before its TMEM loads are done, in the
+re-initialising passes a tile's two MMA commits issued in the other order (the stage
+barrier's commit then outlives the unit), and attention with one group-0 barrier
+instead of one per tile parity.
 """
 import random
 
@@ -431,6 +434,155 @@ def pairs_loop_model(sim, units, stages=2, accf_first=False):
         assert all(x == list(range(nt)) for x in st["seen"])
 
 
+def attend2_model(sim, nt, G, pf0_single=False):
+    """Attention with two query tiles per CTA: a producer, the MMA-issuing thread and two
+    softmax groups of four warps (group g over query tile g; G = 1 when only one query
+    tile is valid).  Per key tile i the issuer, after group 0's barrier, issues
+    PV_0(i) and S_0(i + 1), then after group 1's barrier PV_1(i) and S_1(i + 1).  Group g's
+    S and P share one TMEM region (P(i) overwrites S(i), S(i + 1) overwrites P(i)); O is
+    rescaled in place by the softmax warps.  Key slots: 2 (K(0) through its own barrier,
+    K(i + 1) with tile i); value slots: 3.  pf0 is one barrier per tile parity (group 0's
+    softmax warps + the producer with V(i), K(i + 1)); pf1 one barrier (group 1)."""
+    TB = 32768
+    npf = 1 if pf0_single else 2
+    q_full, k0_full = Bar("q_full", 1), Bar("k0_full", 1)
+    pf0 = [Bar(f"pf0_{p}", 5) for p in range(npf)]
+    pf1 = Bar("pf1", 4)
+    k_empty = [Bar(f"k_empty{s}", 1) for s in range(2)]
+    v_empty = [Bar(f"v_empty{s}", 1) for s in range(3)]
+    s_full = [Bar(f"s_full{g}", 1) for g in range(2)]
+    pv_done = [Bar(f"pv_done{g}", 1) for g in range(2)]
+    st = dict(q=False, k=[-1, -1], k_reads=[0, 0], v=[-1, -1, -1], v_reads=[0, 0, 0],
+              region=[("none", -1)] * 8, busy=[0] * 8, o_through=[-1, -1],
+              pv_pending=[0, 0], seen=[[] for _ in range(8)])
+
+    def pf(i):   # the barrier and phase of group 0 for tile i
+        return (pf0[0], i) if pf0_single else (pf0[i & 1], i >> 1)
+
+    def setter(key, i, v):
+        return lambda: st[key].__setitem__(i, v)
+
+    def producer():
+        q_full.arrive(0, tx=G * TB)
+        sim.copy(q_full, 0, G * TB, lambda: st.__setitem__("q", True))
+        k0_full.arrive(0, tx=TB)
+        sim.copy(k0_full, 0, TB, setter("k", 0, 0))
+        for i in range(nt):
+            if i >= 2:   # the phase two tiles back is over (the same parity's barrier)
+                yield pf(i - 2)
+            if i >= 3:
+                yield (v_empty[i % 3], (i - 3) // 3)
+            knext = i + 1 < nt
+            if knext and i >= 1:
+                yield (k_empty[(i + 1) & 1], (i - 1) >> 1)
+            if st["v_reads"][i % 3]:
+                raise ProtocolError("value slot reloaded while P.V products read it")
+            if knext and st["k_reads"][(i + 1) & 1]:
+                raise ProtocolError("key slot reloaded while score products read it")
+            bar, idx = pf(i)
+            bar.arrive(idx, tx=(2 if knext else 1) * TB)
+            sim.copy(bar, idx, TB, setter("v", i % 3, i))
+            if knext:
+                sim.copy(bar, idx, TB, setter("k", (i + 1) & 1, i + 1))
+            yield None
+        yield (q_full, 0)
+        yield (k0_full, 0)
+        for i in range(max(0, nt - 2), nt):
+            yield pf(i)
+
+    quarter = lambda g: range(4 * g, 4 * g + 4)   # a group's warps: TMEM lane quarters
+
+    def s_mma(g, i):
+        def run():
+            if any(st["busy"][w] for w in quarter(g)):
+                raise ProtocolError(f"S_{g}({i}) written while a softmax warp of group {g} works on its lanes")
+            for w in quarter(g):
+                st["region"][w] = ("S", i)
+            st["k_reads"][i & 1] -= 1
+        return run
+
+    def pv_mma(g, i):
+        def run():
+            if any(st["region"][w] != ("P", i) for w in quarter(g)):
+                raise ProtocolError(f"PV_{g}({i}) reads {[st['region'][w] for w in quarter(g)]} instead of P({i})")
+            if any(st["busy"][w] for w in quarter(g)):
+                raise ProtocolError(f"PV_{g}({i}) while a softmax warp of group {g} works on O")
+            st["o_through"][g] = i
+            st["v_reads"][i % 3] -= 1
+            st["pv_pending"][g] -= 1
+        return run
+
+    def issue_s(g, i):
+        if st["k"][i & 1] != i:
+            raise ProtocolError(f"S_{g}({i}) issued before K({i}) landed")
+        st["k_reads"][i & 1] += 1
+        sim.tc.append(("mma", s_mma(g, i)))
+        sim.tc.append(("commit", s_full[g], i))
+        if g == G - 1:
+            sim.tc.append(("commit", k_empty[i & 1], i >> 1))
+
+    def issue_pv(g, i):
+        if st["v"][i % 3] != i:
+            raise ProtocolError(f"PV_{g}({i}) issued before V({i}) landed")
+        st["v_reads"][i % 3] += 1
+        st["pv_pending"][g] += 1
+        sim.tc.append(("mma", pv_mma(g, i)))
+        sim.tc.append(("commit", pv_done[g], i))
+        if g == G - 1:
+            sim.tc.append(("commit", v_empty[i % 3], i // 3))
+
+    def issuer():
+        yield (q_full, 0)
+        yield (k0_full, 0)
+        if not st["q"]:
+            raise ProtocolError("score products issued before the query tiles landed")
+        for g in range(G):
+            issue_s(g, 0)
+        for i in range(nt):
+            yield pf(i)
+            issue_pv(0, i)
+            if i + 1 < nt:
+                issue_s(0, i + 1)
+            if G == 2:
+                yield (pf1, i)
+                issue_pv(1, i)
+                if i + 1 < nt:
+                    issue_s(1, i + 1)
+            yield None
+        yield (pv_done[0], nt - 1)
+        if G == 2:
+            yield (pv_done[1], nt - 1)
+
+    def softmax(w):
+        g = w // 4
+        ng = nt if g < G else 0
+        for i in range(ng):
+            yield (s_full[g], i)
+            if st["region"][w] != ("S", i):
+                raise ProtocolError(f"warp {w} finds {st['region'][w]} for S({i})")
+            st["busy"][w] += 1
+            yield None                               # S loads, P stores, O rescale
+            if st["pv_pending"][g] or st["o_through"][g] != i - 1:
+                raise ProtocolError(f"group {g} rescales O with P.V products of earlier tiles in flight")
+            st["busy"][w] -= 1
+            st["region"][w] = ("P", i)
+            if g == 0:
+                bar, idx = pf(i)
+                bar.arrive(idx)
+            else:
+                pf1.arrive(i)
+            st["seen"][w].append(i)
+            yield None
+        if ng:
+            yield (pv_done[g], ng - 1)
+            if st["o_through"][g] != ng - 1:
+                raise ProtocolError(f"group {g} reads O before the last P.V product")
+
+    actors = [producer(), issuer()] + [softmax(w) for w in range(8)]
+    sim.run(actors)
+    assert all(st["seen"][w] == (list(range(nt)) if w // 4 < G else []) for w in range(8))
+
+
 def _score_units(rng):
     return [rng.choice([0, 1, 1, 2, 3, 5]) for _ in range(rng.randrange(1, 8))]
 
@@ -455,6 +607,12 @@ def test_crossing_pass_protocol(seed):
 def test_persistent_row_passes_protocol(seed):
     rng = random.Random(2000 + seed)
     pairs_loop_model(Sim(rng), [rng.randrange(1, 7) for _ in range(rng.randrange(1, 6))])
+
+
+@pytest.mark.parametrize("seed", range(60))
+def test_attention_protocol(seed):
+    rng = random.Random(3000 + seed)
+    attend2_model(Sim(rng), rng.randrange(1, 9), rng.choice([1, 2, 2]))
 
 
 def test_long_units_both_passes():
@@ -485,6 +643,12 @@ def test_planted_commit_order_is_caught():
     epilogue's and the issuer's); with that tile's two commits issued accumulator first,
     the stage barrier's commit can still be in flight when the next unit initialises it."""
     assert _caught(lambda s: pairs_loop_model(Sim(random.Random(s)), [3, 2], accf_first=True), range(300))
+
+
+def test_planted_single_attention_barrier_is_caught():
+    """Attention with one group-0 barrier for all tiles instead of one per tile parity:
+    the producer arms tile i + 1 while tile i's phase is still open."""
+    assert _caught(lambda s: attend2_model(Sim(random.Random(s)), 6, 2, pf0_single=True), range(40))
 
 
 def test_planted_early_release_is_caught():
