@@ -5,9 +5,10 @@ and the persistent crossing pass (two 128-row bank tiles per unit, 128-column ca
 tiles) each run one TMA-producer thread, one MMA-issuing thread and 16 epilogue warps
 that meet only at mbarriers, whose phases run on across units.  The persistent
 projection, survivor and new-baseline passes initialise their barriers again for every
-unit, so each unit must end with nothing in flight.  The attention kernel with two query
-tiles per CTA runs a producer, the issuing thread and two softmax groups whose S, P and
-O live in TMEM.  A mistake there shows up
+unit, so each unit must end with nothing in flight.  Both attention schedules (two query
+tiles per CTA; one query tile with its key tiles split over two groups) run a producer,
+the issuing thread and two softmax groups whose S, P and O live in TMEM.  A mistake
+there shows up
 on the GPU as a hang or an exception, not as a wrong number, so the protocol is replayed
 here on the host:
 
@@ -24,13 +25,14 @@ here on the host:
   while a reader still needs it, and every reader finds the tile it expects;
 - every run ends (no deadlock), and every epilogue warp sees every tile in order.
 
-Four planted variants must be caught: four column stages with the combined "tile
+Five planted variants must be caught: four column stages with the combined "tile
 landed and accumulator free" barrier still indexed by accumulator (the form that raised
 a GPU exception: the producer arms the barrier for tile T + 2 while tile T's phase is
 open), an epilogue that releases its accumulator before its TMEM loads are done, in the
 re-initialising passes a tile's two MMA commits issued in the other order (the stage
-barrier's commit then outlives the unit), and attention with one group-0 barrier
-instead of one per tile parity.
+barrier's commit then outlives the unit), attention with one group-0 barrier instead of
+one per tile parity, and key-split attention reloading a group's value slot without
+waiting for the previous tile's P.V products.
 """
 import random
 
@@ -583,6 +585,143 @@ def attend2_model(sim, nt, G, pf0_single=False):
     assert all(st["seen"][w] == (list(range(nt)) if w // 4 < G else []) for w in range(8))
 
 
+def attend_split_model(sim, nt, skip_v_wait=False):
+    """Attention with the key tiles of one query tile split over two softmax groups
+    (group 0 the first (nt + 1) / 2 tiles, group 1 the rest).  Per group: its first key
+    tile through its own barrier, two key slots, one value slot; p_full_g (four softmax
+    warps + the producer with V(i) and K(i + 1)) has one phase per tile; the producer
+    reloads the group's value slot only after PV_g(i - 1) is complete."""
+    TB = 32768
+    n = [(nt + 1) // 2, nt - (nt + 1) // 2]
+    q_full = Bar("q_full", 1)
+    k0_full = [Bar(f"k0_full{g}", 1) for g in range(2)]
+    k_empty = [[Bar(f"k_empty{g}{s}", 1) for s in range(2)] for g in range(2)]
+    v_empty = [Bar(f"v_empty{g}", 1) for g in range(2)]
+    s_full = [Bar(f"s_full{g}", 1) for g in range(2)]
+    p_full = [Bar(f"p_full{g}", 5) for g in range(2)]
+    pv_done = [Bar(f"pv_done{g}", 1) for g in range(2)]
+    st = dict(q=False, k=[[-1, -1], [-1, -1]], k_reads=[[0, 0], [0, 0]], v=[-1, -1], v_reads=[0, 0],
+              region=[("none", -1)] * 8, busy=[0] * 8, o_through=[-1, -1], pv_pending=[0, 0],
+              seen=[[] for _ in range(8)])
+    quarter = lambda g: range(4 * g, 4 * g + 4)
+
+    def set_k(g, slot, i):
+        return lambda: st["k"][g].__setitem__(slot, i)
+
+    def set_v(g, i):
+        return lambda: st["v"].__setitem__(g, i)
+
+    def producer():
+        q_full.arrive(0, tx=TB)
+        sim.copy(q_full, 0, TB, lambda: st.__setitem__("q", True))
+        for g in range(2):
+            if n[g] > 0:
+                k0_full[g].arrive(0, tx=TB)
+                sim.copy(k0_full[g], 0, TB, set_k(g, 0, 0))
+        for i in range(n[0]):
+            for g in range(2):
+                if i >= n[g]:
+                    continue
+                if i > 0 and not skip_v_wait:
+                    yield (v_empty[g], i - 1)
+                knext = i + 1 < n[g]
+                if knext and i > 0:
+                    yield (k_empty[g][(i + 1) & 1], (i - 1) >> 1)
+                if st["v_reads"][g]:
+                    raise ProtocolError(f"value slot of group {g} reloaded while P.V products read it")
+                if knext and st["k_reads"][g][(i + 1) & 1]:
+                    raise ProtocolError(f"key slot of group {g} reloaded while score products read it")
+                p_full[g].arrive(i, tx=(2 if knext else 1) * TB)
+                sim.copy(p_full[g], i, TB, set_v(g, i))
+                if knext:
+                    sim.copy(p_full[g], i, TB, set_k(g, (i + 1) & 1, i + 1))
+                yield None
+        yield (q_full, 0)
+        for g in range(2):
+            if n[g] > 0:
+                yield (k0_full[g], 0)
+                yield (p_full[g], n[g] - 1)
+
+    def s_mma(g, i):
+        def run():
+            if any(st["busy"][w] for w in quarter(g)):
+                raise ProtocolError(f"S_{g}({i}) written while a softmax warp of group {g} works on its lanes")
+            for w in quarter(g):
+                st["region"][w] = ("S", i)
+            st["k_reads"][g][i & 1] -= 1
+        return run
+
+    def pv_mma(g, i):
+        def run():
+            if any(st["region"][w] != ("P", i) for w in quarter(g)):
+                raise ProtocolError(f"PV_{g}({i}) does not read P({i})")
+            if any(st["busy"][w] for w in quarter(g)):
+                raise ProtocolError(f"PV_{g}({i}) while a softmax warp of group {g} works on O")
+            st["o_through"][g] = i
+            st["v_reads"][g] -= 1
+            st["pv_pending"][g] -= 1
+        return run
+
+    def issue_s(g, i):
+        if st["k"][g][i & 1] != i:
+            raise ProtocolError(f"S_{g}({i}) issued before its key tile landed")
+        st["k_reads"][g][i & 1] += 1
+        sim.tc.append(("mma", s_mma(g, i)))
+        sim.tc.append(("commit", k_empty[g][i & 1], i >> 1))
+        sim.tc.append(("commit", s_full[g], i))
+
+    def issuer():
+        yield (q_full, 0)
+        if not st["q"]:
+            raise ProtocolError("score products issued before the query tile landed")
+        for g in range(2):
+            if n[g] > 0:
+                yield (k0_full[g], 0)
+                issue_s(g, 0)
+        for i in range(n[0]):
+            for g in range(2):
+                if i >= n[g]:
+                    continue
+                yield (p_full[g], i)
+                if st["v"][g] != i:
+                    raise ProtocolError(f"PV_{g}({i}) issued before V({i}) landed")
+                st["v_reads"][g] += 1
+                st["pv_pending"][g] += 1
+                sim.tc.append(("mma", pv_mma(g, i)))
+                sim.tc.append(("commit", v_empty[g], i))
+                sim.tc.append(("commit", pv_done[g], i))
+                if i + 1 < n[g]:
+                    issue_s(g, i + 1)
+                yield None
+        for g in range(2):
+            if n[g] > 0:
+                yield (pv_done[g], n[g] - 1)
+
+    def softmax(w):
+        g = w // 4
+        for i in range(n[g]):
+            yield (s_full[g], i)
+            if st["region"][w] != ("S", i):
+                raise ProtocolError(f"warp {w} finds {st['region'][w]} for S({i})")
+            st["busy"][w] += 1
+            yield None
+            if st["pv_pending"][g] or st["o_through"][g] != i - 1:
+                raise ProtocolError(f"group {g} rescales O with P.V products of earlier tiles in flight")
+            st["busy"][w] -= 1
+            st["region"][w] = ("P", i)
+            p_full[g].arrive(i)
+            st["seen"][w].append(i)
+            yield None
+        if n[g]:
+            yield (pv_done[g], n[g] - 1)
+            if st["o_through"][g] != n[g] - 1:
+                raise ProtocolError(f"group {g} reads O before the last P.V product")
+
+    actors = [producer(), issuer()] + [softmax(w) for w in range(8)]
+    sim.run(actors)
+    assert all(st["seen"][w] == list(range(n[w // 4])) for w in range(8))
+
+
 def _score_units(rng):
     return [rng.choice([0, 1, 1, 2, 3, 5]) for _ in range(rng.randrange(1, 8))]
 
@@ -613,6 +752,12 @@ def test_persistent_row_passes_protocol(seed):
 def test_attention_protocol(seed):
     rng = random.Random(3000 + seed)
     attend2_model(Sim(rng), rng.randrange(1, 9), rng.choice([1, 2, 2]))
+
+
+@pytest.mark.parametrize("seed", range(60))
+def test_split_attention_protocol(seed):
+    rng = random.Random(4000 + seed)
+    attend_split_model(Sim(rng), rng.randrange(1, 12))
 
 
 def test_long_units_both_passes():
@@ -649,6 +794,12 @@ def test_planted_single_attention_barrier_is_caught():
     """Attention with one group-0 barrier for all tiles instead of one per tile parity:
     the producer arms tile i + 1 while tile i's phase is still open."""
     assert _caught(lambda s: attend2_model(Sim(random.Random(s)), 6, 2, pf0_single=True), range(40))
+
+
+def test_planted_missing_value_slot_wait_is_caught():
+    """Key-split attention whose producer reloads a group's one value slot without
+    waiting for the previous tile's P.V products."""
+    assert _caught(lambda s: attend_split_model(Sim(random.Random(s)), 8, skip_v_wait=True), range(40))
 
 
 def test_planted_early_release_is_caught():
