@@ -126,6 +126,22 @@ def test_host_only_entry_points():
     L.dkv_bank_destroy(None)
 
 
+def test_every_entry_point_rejects_a_missing_handle():
+    """Argument errors come back as DKV_ERR_ARG before any CUDA call, so they need no GPU:
+    every call that takes a handle, with none."""
+    L = _built_lib().lib()
+    for name, args in [("export", (None, None)), ("import", (None, None, None)), ("stats", (None, None, None)),
+                       ("occupancy", (None, None)), ("intermediates", (None, None)), ("set_timing", (None, 1)),
+                       ("kernel_times", (None, 0, None, None, None, None)), ("reset", (None, None)),
+                       ("update_sequential", (None, None, None, 1, 0, None, 0, None))]:
+        assert getattr(L, "dkv_bank_" + name)(*args) == 1, name
+    assert L.dkv_params_default(None, 128) == 1
+    assert L.dkv_candidate_order_noalloc(None, None, 1, None, 1, 128, 0, None, None, None, None) == 1
+    # scratch of the sequential update: zero for an unsupported head size
+    assert L.dkv_sequential_scratch_size(2, 96, 16, 0) == 0
+    assert L.dkv_sequential_scratch_size(2, 128, 16, 0) > 0
+
+
 def test_binding_has_no_fallback(monkeypatch):
     from paper_2608_27922_gb300 import dkv
     monkeypatch.setattr(dkv, "LIB_PATH", "/nonexistent/libdkv.so")
