@@ -252,3 +252,12 @@ def test_fullsize_headwise_budgets(dkv, sync):
     """Wan-14B-shaped layer: 40 heads with budgets drawn from {2340, 4680, 9360, 18720}."""
     wl = synth.get_workload("wan14b_headwise_l40h40", L=1)
     _run(dkv, wl, steps=4, sync_heads=sync, rows=12, cands=12)
+
+
+def test_fullsize_headwise_wide_score_pass(dkv):
+    """80 Wan-14B-shaped heads (budgets drawn from {2340, 4680, 9360, 18720}, N = 4,680):
+    2,960 candidate row tiles, so the score pass takes the persistent 256-column form
+    that the config-4 model step runs."""
+    wl = synth.get_workload("wan14b_headwise_l40h40", L=1, H=80)
+    assert wl.H * ((wl.N + 127) // 128) >= 16 * 152
+    _run(dkv, wl, steps=3, rows=8, cands=8)
