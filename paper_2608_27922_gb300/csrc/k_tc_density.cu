@@ -25,17 +25,21 @@
 //
 // Epilogue arithmetic.  Two interactions share one reciprocal:
 //   |A1|^-2 + |A2|^-2 = (A1^2 + A2^2) / (A1 A2)^2,
-// and the 16 pair terms of a 32-column chunk are summed as a fixed binary tree, so
-// there is no serial dependence inside a chunk.  The crossing pass tests each
-// chunk total against the row's threshold and rescans a chunk term by term only
-// when the threshold falls inside it (at most once per row).
+// and the 16 pair terms of a 32-column chunk are accumulated in a fixed order: two
+// independent chains of four packed fp32x2 accumulations, added at the end, so a
+// chunk's dependence chain is short.  The crossing pass tests each chunk total
+// against the row's threshold and rescans a chunk term by term only when the
+// threshold falls inside it (at most once per row).
 //
 // CTA (320 threads, 2 per SM): warp 0 TMA producer, warp 1 MMA issuer, warps 2-9
 // epilogue.  Epilogue warps w and w+4 share TMEM lanes 32 (w % 4) .. +31 (one row
 // per lane) and split each 128-column tile into halves of 64 columns; the crossing
-// and projection passes exchange half totals through shared memory every tile.  The
-// crossing pass over keys runs in a persistent form with two row tiles per CTA
-// (tc_cross_dual, below); the [K; V] descriptor keeps the one-row-tile form.
+// and projection passes exchange half totals through shared memory every tile.
+// Persistent forms (one CTA per SM, or two, taking units in turn): the crossing pass
+// over keys with two row tiles per unit (tc_cross_dual), the score pass over many
+// candidate row tiles with 256-column bank tiles (tc_score_wide), and the projection,
+// survivor and new-baseline passes over many row tiles (tc_pairs_loop); the [K; V]
+// descriptor keeps the one-row-tile form.
 #include "dkv_internal.h"
 #include "tc_ptx.cuh"
 
