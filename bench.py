@@ -804,6 +804,18 @@ TENSOR_KERNELS = ("attend_tc", "score_tc", "cross_tc", "project_tc", "subtract_t
 HBM_KERNELS = ("cand_norms", "sort_runs", "sort_rank", "rstar", "select", "commit")
 
 
+def kernel_roofs(per_kernel, steps):
+    """The per-kernel pass against its kernels' roofs: the timed kernels' time per step,
+    the time they would take at their roofs (tensor kernels' algorithmic flops at the bf16
+    peak, memory-bound kernels' algorithmic bytes at the HBM peak), and the ratio."""
+    if not per_kernel or steps <= 0:
+        return None
+    per_step = lambda r: r["avg_ms"] * r["launches"] / steps
+    t = sum(per_step(r) for r in per_kernel.values())
+    at = sum(per_step(r) * r.get("frac_of_bf16_peak", r.get("frac_of_hbm_alg", 0.0)) for r in per_kernel.values())
+    return {"ms_per_step": t, "at_roofs_ms": at, "frac": at / t if t > 0 else None}
+
+
 def kernel_work(name, d, esize, N, Nq, W, layer_of_head, Ls, hs):
     """Algorithmic work of one launch of kernel `name` over every head of a handle in one
     update step, from the step's statistics (Ls per layer, hs per head).
@@ -1197,7 +1209,7 @@ def run_stack(args):
             "wall_s_timed": wall, "step_ms": {"min": min(step_ms), "median": statistics.median(step_ms),
                                               "max": max(step_ms)},
             "e2e": e2e, "gpu_launches": launches * world, "roofline": roof, "cpu_baseline": cpu, "clocks": clk,
-            "per_kernel": per_kernel,
+            "per_kernel": per_kernel, "per_kernel_roofs": kernel_roofs(per_kernel, P),
             "per_kernel_note": f"{P} further steps on one stream with every launch timed by CUDA events (not "
                                "in value; the survivor and new-baseline passes then run one after the other); "
                                "tensor kernels against the bf16 peak, memory-bound kernels' algorithmic (and "

@@ -75,3 +75,17 @@ def test_stack_sample_heads_near_the_mean_budget():
     assert len(heads) == 2 and all(h < wl.H for h in heads)
     assert sorted(abs(wl.budgets[h] - mean) for h in heads) == sorted(
         abs(b - mean) for b in set(wl.budgets))[:2]
+
+
+def test_kernel_roofs_of_the_per_kernel_pass():
+    """The per-kernel pass against the sum of its kernels' roofs (time per step at each
+    kernel's measured fraction of its roof)."""
+    import pytest
+    pk = {"attend_tc": {"launches": 2, "avg_ms": 28.0, "share": 0.6, "frac_of_bf16_peak": 0.8},
+          "cand_norms": {"launches": 2, "avg_ms": 1.0, "share": 0.1, "frac_of_hbm_alg": 0.5},
+          "sort_runs": {"launches": 4, "avg_ms": 0.25, "share": 0.0}}
+    r = bench.kernel_roofs(pk, 2)
+    assert r["ms_per_step"] == pytest.approx(28.0 + 1.0 + 0.5)
+    assert r["at_roofs_ms"] == pytest.approx(28.0 * 0.8 + 0.5)
+    assert r["frac"] == pytest.approx((28.0 * 0.8 + 0.5) / 29.5)
+    assert bench.kernel_roofs({}, 2) is None and bench.kernel_roofs(pk, 0) is None
